@@ -1,0 +1,426 @@
+#!/usr/bin/env python3
+"""Benchmark of the JET candidate-scoring step on GB300.
+
+A step is one pass of the whole hot path - cascade attention, the recurrent
+state fork (hybrid workloads), the fused LM head with full-vocabulary
+log-sum-exp and target gather, and the decision rules - over one batch of
+synthetic requests whose inputs are already resident in HBM. The metric is
+candidate sets (requests) scored per second.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--R R]
+    python bench.py --impl reference ...   # the fp64 CPU oracle on the host cores
+
+Under torchrun (N > 1) every rank scores its own batch on its own GPU
+(independent replicas, no collective on the data path); rank 0 prints one
+JSON line with the whole-job throughput.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+_CORES = os.cpu_count() or 1
+for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, str(_CORES))
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "candidate sets scored/sec"
+UNIT = "sets/s"
+DEFAULT_WORKLOAD = "dense27b_mc"
+L2_BYTES = 129 * 1024 * 1024
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return dict(hbm=float(p["hbm_gbs"]), bf16=float(p["bf16_tflops"]),
+                    bf16_sustained=float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
+                    source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, source="fallback")
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    QUERY = ("timestamp,index,uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid: str | None):
+        self.uuid = uuid
+        self.lines = []
+        self.proc = None
+        self.t_on = self.t_off = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def mark(self, on: bool):
+        if on:
+            self.t_on = time.time()
+        else:
+            self.t_off = time.time()
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        rows = []
+        for t, line in self.lines:
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 11:
+                continue
+            if self.uuid and self.uuid not in f[2]:
+                continue
+            try:
+                rows.append(dict(t=t, sm=float(f[3]), smax=float(f[4]), active=f[6],
+                                 hw=f[7], hwt=f[8], swt=f[9], swp=f[10]))
+            except ValueError:
+                continue
+        inside = [r for r in rows if self.t_on and self.t_off and self.t_on <= r["t"] <= self.t_off + 0.1]
+        window = "timed"
+        if not inside:
+            inside, window = rows, "warmup+timed"
+        if not inside:
+            return None
+        reasons = set()
+        for r in inside:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                              ("swt", "sw_thermal_slowdown"), ("swp", "sw_power_cap")):
+                if r[key].lower().startswith("active"):
+                    reasons.add(name)
+        return dict(sm_mhz=statistics.median(r["sm"] for r in inside),
+                    sm_max_mhz=max(r["smax"] for r in inside), reasons=sorted(reasons),
+                    samples=len(inside), window=window)
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (baseline and reference arm)
+# ---------------------------------------------------------------------------
+def oracle_step(problem):
+    """The oracle's whole step on one problem: attention, fork, LM head, Eq. 3-5."""
+    import oracle as O
+    w = problem.work
+    lay = O.build_layout(problem.prefix_len, problem.n_cand, problem.cand_len,
+                         problem.target_ids, w.V)
+    O.cascade_attention(lay, problem.f32("q"), problem.f32("k_pre"), problem.f32("v_pre"),
+                        problem.f32("k_cand"), problem.f32("v_cand"), w.Hq, w.Hkv)
+    if w.Hl:
+        O.fork_state(lay, problem.f32("s_prefix"), problem.f32("lq"), problem.f32("lk"),
+                     problem.f32("lv"), problem.f32("alpha"), problem.f32("beta"))
+    mode = {"argmax": O.ARGMAX, "binary": O.BINARY, "ordinal": O.ORDINAL}[w.mode]
+    return O.score_step(lay, problem.f32("hidden"), problem.f32("w_lm"), mode)
+
+
+def oracle_sample(name: str, R: int, k: int):
+    import jet_synth
+    p = jet_synth.make_problem(name, R=min(k, R))
+    names = ["q", "k_pre", "v_pre", "k_cand", "v_cand", "hidden", "w_lm"]
+    if p.work.Hl:
+        names += ["s_prefix", "lq", "lk", "lv", "alpha", "beta"]
+    for n in names:  # draw the inputs before timing
+        p.f32(n)
+    return p
+
+
+def cpu_baseline(name: str, R: int, k: int):
+    p = oracle_sample(name, R, k)
+    t0 = time.perf_counter()
+    oracle_step(p)
+    dt = time.perf_counter() - t0
+    return dict(value=p.R / dt, unit=UNIT, cores=_CORES, kind="oracle",
+                sample=f"first {p.R} of {R} requests of workload {name}, one pass of the "
+                       f"fp64 oracle step ({dt:.1f} s), BLAS threads {_CORES}")
+
+
+# ---------------------------------------------------------------------------
+# helpers
+# ---------------------------------------------------------------------------
+def _source_hash(files):
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def _traffic(kernel_file: str, workload: str):
+    """DRAM traffic per launch of the dominant kernel from a committed ncu
+    summary, if it was taken on the current source of that kernel."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    try:
+        with open(path) as f:
+            rec = json.load(f).get(workload)
+    except (OSError, ValueError):
+        return None
+    if not rec or rec.get("source_hash") != _source_hash([kernel_file]):
+        return None
+    return rec.get("bytes_per_launch")
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+def run_gpu(args):
+    import torch
+    world, rank, local = _dist()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+
+    from paper_2609_33874_gb300 import build as _build
+    if rank == 0:
+        _build.build()
+    if world > 1:
+        torch.distributed.barrier()
+    import jet_synth
+    from paper_2609_33874_gb300 import jet
+    from paper_2609_33874_gb300.step import ScoringStep
+
+    w = jet_synth.WORKLOADS[args.workload]
+    R = args.R or w.R
+    problem = jet_synth.make_problem(w, R=R)
+    dtype = jet.DTYPE_BF16 if w.dtype == "bf16" else jet.DTYPE_F32
+    dims = jet.make_dims(dtype, Hq=w.Hq, Hkv=w.Hkv, d=w.d, D=w.D, Hl=w.Hl, dk=w.dk, dv=w.dv)
+    hl = jet.jet_layout_build(problem.prefix_len, problem.n_cand, problem.cand_len,
+                              problem.target_ids, w.V)
+    step = ScoringStep(hl, dims, jet.MODES[w.mode], device=dev, hybrid=w.Hl > 0,
+                       keep_fork_state=w.Hl > 0)
+    names = step.input_names()
+    x = {k: jet_synth.torch_tensor(problem, k, device=dev) for k in names}
+    w_lm = jet_synth.torch_tensor(problem, "w_lm", device=dev)
+    stream = torch.cuda.Stream(dev)
+
+    # --- device-resident timed region -------------------------------------
+    n_ev = args.steps
+    score_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                for _ in range(n_ev)]
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        pass
+    clocks = ClockSampler(uuid)
+    clocks.start()
+
+    def one_step(i=None):
+        d, lay = step.dims, step.layout
+        jet.jet_prefix_attend(lay, d, x["q"], x["k_pre"], x["v_pre"], x["k_cand"], x["v_cand"],
+                              step.o, step.ws, stream=stream)
+        if step.hybrid:
+            jet.jet_fork_state(lay, d, x["s_prefix"], x["lq"], x["lk"], x["lv"], x["alpha"],
+                               x["beta"], step.lo, step.s_fork, stream=stream)
+        if i is not None:
+            score_ev[i][0].record(stream)
+        jet.jet_score_candidates(lay, d, x["hidden"], w_lm, step.tok_logprob, step.cand_score,
+                                 step.ws, stream=stream)
+        if i is not None:
+            score_ev[i][1].record(stream)
+        jet.jet_decide(lay, step.mode, step.cand_score, step.q_cand, step.choice, step.value,
+                       stream=stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            one_step()
+    torch.cuda.synchronize(dev)
+    assert jet.jet_device_status(stream) == 0, "kernel reported an invalid layout index"
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize(dev)
+    clocks.mark(True)
+    t_start.record(stream)
+    with torch.cuda.stream(stream):
+        for i in range(args.steps):
+            one_step(i)
+    t_end.record(stream)
+    torch.cuda.synchronize(dev)
+    clocks.mark(False)
+    if world > 1:
+        torch.distributed.barrier()
+    total_ms = t_start.elapsed_time(t_end)
+    clk = clocks.stop()
+    score_ms = [a.elapsed_time(b) for a, b in score_ev]
+
+    # --- end to end: pinned host inputs, copies inside the timed region ---------
+    host = {k: x[k].cpu().pin_memory() for k in names}
+    words = torch.from_numpy(hl.words).pin_memory()
+    out = {k: torch.empty_like(getattr(step, k), device="cpu").pin_memory()
+           for k in ("tok_logprob", "cand_score", "q_cand", "choice", "value")}
+    e_steps = max(3, min(args.steps, 50))
+    for _ in range(max(3, args.warmup)):
+        step.run_from_host(host, words, w_lm, out, stream=stream)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    e0.record(stream)
+    for _ in range(e_steps):
+        step.run_from_host(host, words, w_lm, out, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = e0.elapsed_time(e1) / e_steps
+    h2d, d2h = step.host_bytes(host, words)
+    assert jet.jet_device_status(stream) == 0
+
+    if world > 1:
+        t = torch.tensor([total_ms, e2e_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms, e2e_ms = float(t[0]), float(t[1])
+
+    ms_per_step = total_ms / args.steps
+    value = R * world / (ms_per_step / 1e3)
+    e2e_value = R * world / (e2e_ms / 1e3)
+
+    # --- roofline of the dominant kernel (the LM head) ----------------------
+    peaks = _peaks()
+    N, T = problem.N, len(problem.target_ids)
+    es = 2 if w.dtype == "bf16" else 4
+    vtiles = (w.V + 127) // 128
+    lm_bytes = w.V * w.D * es + N * w.D * es + vtiles * N * 8 + T * 4
+    lm_flops = 2.0 * N * w.D * w.V
+    score_avg_s = statistics.mean(score_ms) / 1e3
+    ridge = peaks["bf16"] * 1e12 / (peaks["hbm"] * 1e9)
+    kernel_file = "paper_2609_33874_gb300/csrc/lmhead_tc.cu" if w.dtype == "bf16" and \
+        os.path.exists(os.path.join(ROOT, "paper_2609_33874_gb300/csrc/lmhead_tc.cu")) \
+        else "paper_2609_33874_gb300/csrc/lmhead_simt.cu"
+    traffic = _traffic(kernel_file, args.workload)
+    if w.dtype != "bf16":
+        roof = dict(bound="alu", achieved=lm_flops / score_avg_s / 1e12, peak=None, unit="TFLOP/s",
+                    frac=None, traffic=traffic)
+    elif lm_flops / lm_bytes < ridge:
+        ach = lm_bytes / score_avg_s / 1e9
+        roof = dict(bound="hbm", achieved=round(ach, 1), peak=peaks["hbm"], unit="GB/s",
+                    frac=round(ach / peaks["hbm"], 4), traffic=traffic)
+    else:
+        ach = lm_flops / score_avg_s / 1e12
+        roof = dict(bound="tensor", achieved=round(ach, 1), peak=peaks["bf16"], unit="TFLOP/s",
+                    frac=round(ach / peaks["bf16"], 4), traffic=traffic)
+    roof.update(kernel="jet_score_candidates (LM head + lse merge)",
+                algorithmic_bytes=lm_bytes, algorithmic_flops=lm_flops,
+                avg_launch_ms=round(score_avg_s * 1e3, 4), peak_source=peaks["source"])
+
+    launches_per_step = 2 + (1 if w.Hl else 0) + 3 + 1
+    result = dict(
+        metric=METRIC, value=round(value, 2), unit=UNIT, n_gpus=world, steps=args.steps,
+        warmup=args.warmup, ms_per_step=round(ms_per_step, 4), higher_is_better=True,
+        scaling="weak", vs_baseline=None, dtype="bf16" if w.dtype == "bf16" else "f32",
+        data="synthetic",
+        config=dict(workload=args.workload, R=R, N=N, T=T, C=len(problem.cand_len),
+                    total_prefix=problem.total_prefix, Hq=w.Hq, Hkv=w.Hkv, d=w.d, D=w.D, V=w.V,
+                    Hl=w.Hl, parallelism=f"replicas{world}" if world > 1 else "single",
+                    l2=f"inputs larger than L2: LM-head weights {w.V * w.D * es / 1e9:.2f} GB "
+                       f"streamed every step"),
+        clocks=clk,
+        e2e=dict(value=round(e2e_value, 2), unit=UNIT, h2d_bytes_per_step=h2d,
+                 d2h_bytes_per_step=d2h, ms_per_step=round(e2e_ms, 4)),
+        gpu_launches=launches_per_step * args.steps,
+        roofline=roof,
+    )
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(args.workload, R, args.cpu_sample)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# reference arm: the fp64 oracle on the host cores
+# ---------------------------------------------------------------------------
+def run_reference(args):
+    world, rank, _ = _dist()
+    if rank != 0:
+        return
+    import jet_synth
+    w = jet_synth.WORKLOADS[args.workload]
+    R = args.R or w.R
+    k = args.ref_sample
+    p = oracle_sample(args.workload, R, k)
+    for _ in range(args.warmup):
+        oracle_step(p)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_step(p)
+    dt = (time.perf_counter() - t0) / args.steps
+    value = p.R / dt
+    desc = (f"first {p.R} of {R} requests of workload {args.workload} per step, fp64 oracle "
+            f"step, BLAS threads {_CORES}")
+    print(json.dumps(dict(
+        impl="reference", metric=METRIC, value=round(value, 4), unit=UNIT, n_gpus=world,
+        steps=args.steps, warmup=args.warmup, ms_per_step=round(dt * 1e3, 2),
+        higher_is_better=True, scaling="weak", vs_baseline=None, dtype="f64", data="synthetic",
+        config=dict(workload=args.workload, R=R),
+        cpu_baseline=dict(value=round(value, 4), unit=UNIT, cores=_CORES, kind="oracle",
+                          sample=desc),
+        e2e=dict(value=round(value, 4), unit=UNIT, h2d_bytes_per_step=0, d2h_bytes_per_step=0),
+    )), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--R", type=int, default=0, help="requests per batch (default: the workload's)")
+    ap.add_argument("--cpu-sample", type=int, default=16,
+                    help="requests in the CPU-oracle baseline sample")
+    ap.add_argument("--ref-sample", type=int, default=1,
+                    help="requests per step of the reference arm")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(3, args.warmup)  # at least three untimed warm-up steps
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,261 @@
+/*
+ * jet.h - C ABI of the JET teacher-forced candidate-scoring step on GB300
+ * (sm_103a).
+ *
+ * JET (Justification Evaluation in Transformer) picks an answer from a
+ * finite candidate set by the candidates' teacher-forced likelihoods under a
+ * language model (Sec. 3). For a question context x, candidates
+ * y_c = (y_{c,1} .. y_{c,m_c}) and vocabulary V, one step computes
+ *
+ *   attention   shared-prefix cascade attention: every candidate row attends
+ *               to the request's prefix K/V plus its own earlier candidate
+ *               tokens (Sec. 4.1)                        -> jet_prefix_attend
+ *   fork        per-candidate continuation of an unmodified copy of the
+ *               prefix recurrent state (Sec. 4.1)        -> jet_fork_state
+ *   score       l_{c,t} = log p(y_{c,t} | x, y_{c,<t}) over the full
+ *               vocabulary (Eq. 1, Eq. 2) and s(c|x) = sum_t l_{c,t} (Eq. 3);
+ *               logits never leave the chip (Sec. 4.2)   -> jet_score_candidates
+ *   decide      q(c) = softmax over candidates (Eq. 4), argmax choice (Eq. 5),
+ *               binary q(true) or ordinal expectation (Sec. 3.3) -> jet_decide
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Every function returns a jet_status; 0 (JET_OK) means success. Nothing is
+ *   launched when a call returns an error. The library never allocates
+ *   memory, never synchronises a stream (except jet_device_status), never
+ *   prints and never exits the process.
+ * - Tensor arguments are DEVICE pointers owned by the caller, 16-byte
+ *   aligned, row-major and dense, in the element type jet_dims.dtype names
+ *   (float32 or bf16) unless stated otherwise.
+ * - A layout's int32 arrays live where the call needs them: host memory for
+ *   jet_layout_build, device memory for the compute calls (copy the words
+ *   buffer once and bind it with jet_layout_bind).
+ * - Work is enqueued on `stream` (a cudaStream_t passed as void*; NULL means
+ *   the legacy default stream) and runs asynchronously.
+ * - Kernels check every index they read from a device layout and skip an
+ *   out-of-range access instead of faulting; they then record
+ *   JET_ERR_DEVICE in a per-device status word that jet_device_status reads.
+ *
+ * Row layout (Sec. 3.1, Eq. 1; Sec. 4.1)
+ * --------------------------------------
+ * Request r owns n_r = 1 + sum_c (m_c - 1) consecutive query rows. Its first
+ * ("shared") row is the last prefix position: its logits condition on x alone
+ * and give p(y_{c,1} | x) for every candidate c. Then, candidate by candidate,
+ * one row per fed token y_{c,t}, t = 1 .. m_c - 1; the row fed with y_{c,t}
+ * predicts y_{c,t+1}. y_{c,m_c} is a target only. N = sum_r n_r rows,
+ * T = sum_c m_c targets, C = sum_r C_r candidates, F = N - R fed tokens.
+ * Candidate tensors indexed by fed token use row order with the shared rows
+ * left out: the fed token of row n of request r has index n - r - 1.
+ */
+#ifndef JET_H
+#define JET_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define JET_ABI_VERSION 1
+
+typedef int32_t jet_status;
+enum {
+  JET_OK = 0,
+  JET_ERR_ARG = 1,         /* null pointer or invalid scalar argument          */
+  JET_ERR_SHAPE = 2,       /* inconsistent sizes (Hq % Hkv != 0, m_c < 1, ...)  */
+  JET_ERR_RANGE = 3,       /* a token id outside [0, V)                          */
+  JET_ERR_ALIGN = 4,       /* a device pointer that is not 16-byte aligned       */
+  JET_ERR_WORKSPACE = 5,   /* workspace null or smaller than jet_workspace_bytes */
+  JET_ERR_CAPACITY = 6,    /* a size beyond what the kernels index (2^31 elems)  */
+  JET_ERR_UNSUPPORTED = 7, /* dtype or head dimension the kernels do not handle */
+  JET_ERR_CUDA = 8,        /* a CUDA runtime call or launch failed               */
+  JET_ERR_TIMEOUT = 9,     /* a bounded device-side wait gave up                 */
+  JET_ERR_DEVICE = 10      /* a kernel met an out-of-range index in a layout     */
+};
+
+enum { JET_DTYPE_F32 = 0, JET_DTYPE_BF16 = 1 };
+
+/* decision rules of Sec. 3.3 / Eq. 5 */
+enum { JET_DECIDE_ARGMAX = 0, JET_DECIDE_BINARY = 1, JET_DECIDE_ORDINAL = 2 };
+
+/* Sizes of one batch; filled by jet_layout_plan. */
+typedef struct jet_sizes {
+  int32_t R;            /* requests (contexts x)                          */
+  int32_t C;            /* candidates, sum_r C_r                          */
+  int32_t N;            /* query rows, sum_r n_r                          */
+  int32_t T;            /* targets, sum_c m_c                             */
+  int32_t V;            /* vocabulary size |V|                            */
+  int32_t total_prefix; /* sum_r P_r                                      */
+  int32_t max_prefix;   /* max_r P_r                                      */
+  int32_t min_cand;     /* min_r C_r                                      */
+  int32_t max_cand;     /* max_r C_r                                      */
+  int32_t max_rows;     /* max_r n_r                                      */
+  int32_t max_len;      /* max_c m_c                                      */
+  int32_t reserved;
+} jet_sizes;
+
+/*
+ * The integer layout of a batch (Sec. 3.1, Eq. 1; Sec. 4.1). All arrays are
+ * int32 and point into one "words" buffer of jet_layout_words() entries.
+ *   prefix_offset[R+1]   request r's prefix keys are [prefix_offset[r], prefix_offset[r+1])
+ *                        of the packed prefix K/V
+ *   cand_offset[R+1]     request r's candidates are [cand_offset[r], cand_offset[r+1])
+ *   row_offset[R+1]      request r's rows; row_offset[r] is its shared row
+ *   cand_row_offset[C+1] first fed row of candidate c (its m_c - 1 fed rows
+ *                        are consecutive); entry C is N
+ *   tgt_offset[C+1]      candidate c's targets y_{c,1..m_c} are
+ *                        [tgt_offset[c], tgt_offset[c+1])
+ *   target_ids[T]        y_{c,t} in candidate order
+ *   tgt_row[T]           the row whose logits predict target j
+ *   row_req[N]           request of row n
+ *   row_cand[N]          candidate of row n, -1 for a shared row
+ *   row_pos[N]           t of the token fed at row n, 0 for a shared row
+ *   row_tgt_offset[N+1], row_tgt_index[T]
+ *                        the targets predicted by row n, in increasing index
+ */
+typedef struct jet_layout {
+  jet_sizes n;
+  const int32_t* prefix_offset;
+  const int32_t* cand_offset;
+  const int32_t* row_offset;
+  const int32_t* cand_row_offset;
+  const int32_t* tgt_offset;
+  const int32_t* target_ids;
+  const int32_t* tgt_row;
+  const int32_t* row_req;
+  const int32_t* row_cand;
+  const int32_t* row_pos;
+  const int32_t* row_tgt_offset;
+  const int32_t* row_tgt_index;
+} jet_layout;
+
+/* Model dimensions of the step. */
+typedef struct jet_dims {
+  int32_t dtype; /* JET_DTYPE_*: element type of q, k, v, o, hidden, w_lm    */
+  int32_t Hq;    /* attention query heads                                    */
+  int32_t Hkv;   /* attention key/value heads; query head h uses
+                    key/value head h / (Hq / Hkv) (grouped-query attention) */
+  int32_t d;     /* attention head dimension: 64, 128 or 256                  */
+  int32_t D;     /* LM-head hidden size (multiple of 8)                       */
+  int32_t Hl;    /* linear-attention heads (0 when the model has none)        */
+  int32_t dk;    /* linear-attention key dimension: 128                       */
+  int32_t dv;    /* linear-attention value dimension: multiple of 32, <= 256 */
+} jet_dims;
+
+/* ABI version of the loaded library (JET_ABI_VERSION it was built with). */
+int32_t jet_abi_version(void);
+
+/* Static description of a status code; never NULL. */
+const char* jet_status_string(jet_status s);
+
+/*
+ * jet_layout_plan - sizes of a batch, from its structure (host only).
+ * prefix_len[R] = P_r >= 1, n_cand[R] = C_r >= 1, cand_len[C] = m_c >= 1 in
+ * request order, V >= 1. Errors: JET_ERR_ARG (null, R < 0, V < 1),
+ * JET_ERR_SHAPE (a count below 1), JET_ERR_CAPACITY (a total beyond int32).
+ */
+jet_status jet_layout_plan(int32_t R, const int32_t* prefix_len, const int32_t* n_cand,
+                           const int32_t* cand_len, int32_t V, jet_sizes* out);
+
+/* Number of int32 words a layout of these sizes occupies. */
+size_t jet_layout_words(const jet_sizes* n);
+
+/*
+ * jet_layout_build - the teacher-forced layout (host only, Sec. 3.1, Eq. 1;
+ * Sec. 4.1). target_ids[T] lists y_{c,1..m_c} for every candidate in request
+ * order; each must lie in [0, V) (else JET_ERR_RANGE). `words` is a caller
+ * buffer of n_words >= jet_layout_words() int32 (else JET_ERR_WORKSPACE);
+ * `out` is bound to it. The words may then be copied verbatim to the device
+ * and bound with jet_layout_bind.
+ */
+jet_status jet_layout_build(int32_t R, const int32_t* prefix_len, const int32_t* n_cand,
+                            const int32_t* cand_len, const int32_t* target_ids, int32_t V,
+                            int32_t* words, size_t n_words, jet_layout* out);
+
+/* jet_layout_bind - point a layout's arrays into a (host or device) copy of
+ * the words buffer. Does not read the words. */
+jet_status jet_layout_bind(const jet_sizes* n, const int32_t* words, jet_layout* out);
+
+/* Workspace bytes jet_prefix_attend and jet_score_candidates need for a batch
+ * of these sizes (the larger of the two; one buffer serves both calls when
+ * they run one after the other on a stream). 0 on invalid arguments. */
+size_t jet_workspace_bytes(const jet_sizes* n, const jet_dims* dims);
+
+/*
+ * jet_prefix_attend - shared-prefix cascade attention (Sec. 4.1, Fig. 1
+ * "KV-cache text models"; scale 1/sqrt(d), no positional encoding).
+ *   q       [N, Hq, d]           query of every row
+ *   k_pre   [total_prefix, Hkv, d], v_pre likewise: packed prefix K/V
+ *   k_cand  [F, Hkv, d], v_cand likewise: K/V of the fed candidate tokens
+ *   o       [N, Hq, d]           output
+ * The shared row of request r attends to its P_r prefix keys; the row fed
+ * with y_{c,t} attends to the prefix and to y_{c,1..t} of its own candidate.
+ * The prefix K/V of a request is read once per key/value head by all of the
+ * request's rows. Accumulation is float32; o is written in dims.dtype.
+ * ws/ws_bytes: scratch of at least jet_workspace_bytes().
+ */
+jet_status jet_prefix_attend(const jet_layout* lay, const jet_dims* dims, const void* q,
+                             const void* k_pre, const void* v_pre, const void* k_cand,
+                             const void* v_cand, void* o, void* ws, size_t ws_bytes,
+                             void* stream);
+
+/*
+ * jet_fork_state - per-candidate fork of a linear-attention recurrent state
+ * (Sec. 4.1: each candidate continues from the unchanged prefix state).
+ *   s_prefix [R, Hl, dk, dv] float32  state after the prefix (read only)
+ *   q, k     [F, Hl, dk]  dims.dtype  per fed token; k is expected unit-norm
+ *   v        [F, Hl, dv]  dims.dtype
+ *   alpha, beta [F, Hl] float32       gates
+ *   o        [F, Hl, dv]  dims.dtype  output o_t = S_t^T q_t / sqrt(dk)
+ *   s_fork   [C, Hl, dk, dv] float32  state after each candidate's last fed
+ *            token (a copy of the prefix state when m_c = 1); may be NULL
+ * Each fed token applies S <- alpha (S - beta k (k^T S)) + beta k v^T (gated
+ * delta rule; the paper does not name its recurrence). All candidates run
+ * concurrently from one read of the prefix state.
+ */
+jet_status jet_fork_state(const jet_layout* lay, const jet_dims* dims, const float* s_prefix,
+                          const void* q, const void* k, const void* v, const float* alpha,
+                          const float* beta, void* o, float* s_fork, void* stream);
+
+/*
+ * jet_score_candidates - LM head, full-vocabulary log-softmax and target
+ * gather (Eq. 1, Eq. 2), then candidate scores (Eq. 3).
+ *   hidden      [N, D]  dims.dtype  LM-head input of every row
+ *   w_lm        [V, D]  dims.dtype  LM-head weights (logit z_v = hidden . w_lm[v])
+ *   tok_logprob [T] float32         l_{c,t} in candidate order
+ *   cand_score  [C] float32         s(c|x) = sum_t l_{c,t}, summed in t order
+ * The N x V logits are reduced on chip to per-tile (max, sum of exp) pairs and
+ * never written to memory. bf16 inputs use the tensor cores with float32
+ * accumulation; float32 inputs use float32 FMA.
+ * ws/ws_bytes: scratch of at least jet_workspace_bytes().
+ */
+jet_status jet_score_candidates(const jet_layout* lay, const jet_dims* dims, const void* hidden,
+                                const void* w_lm, float* tok_logprob, float* cand_score,
+                                void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * jet_decide - decision rules (Eq. 4, Eq. 5, Sec. 3.3).
+ *   cand_score [C] float32   s(c|x)
+ *   q          [C] float32   q(c) = exp(s_c - M) / sum_d exp(s_d - M), M = max s
+ *   choice     [R] int32     argmax_c s_c, ties to the lowest candidate index
+ *   value      [R] float32   ARGMAX: q(choice); BINARY: q(true) = q of
+ *                            candidate 1 (the set is {false, true}, every
+ *                            request needs C_r = 2, else JET_ERR_SHAPE);
+ *                            ORDINAL: sum_i i q(i), zero-based levels
+ */
+jet_status jet_decide(const jet_layout* lay, int32_t mode, const float* cand_score, float* q,
+                      int32_t* choice, float* value, void* stream);
+
+/*
+ * jet_device_status - wait for `stream`, then report and clear the current
+ * device's status word: JET_OK, JET_ERR_DEVICE (a kernel skipped an
+ * out-of-range layout index) or JET_ERR_TIMEOUT (a bounded wait gave up).
+ * A failed CUDA call returns JET_ERR_CUDA.
+ */
+jet_status jet_device_status(void* stream, jet_status* out);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* JET_H */

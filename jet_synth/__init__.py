@@ -310,3 +310,19 @@ def custom_problem(work: Workload, prefix_len, n_cand, cand_len, target_ids,
     return Problem(work, seed, np.asarray(prefix_len, dtype=np.int32),
                    np.asarray(n_cand, dtype=np.int32), np.asarray(cand_len, dtype=np.int32),
                    np.asarray(target_ids, dtype=np.int32))
+
+
+def torch_tensor(problem: Problem, name: str, device=None, pin: bool = False):
+    """A tensor of the problem as a torch tensor (bf16 bit patterns become
+    torch.bfloat16 without any rounding); optionally pinned or on a device."""
+    import torch
+    a = problem.tensor(name)
+    if a.dtype == np.uint16:
+        t = torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16)
+    else:
+        t = torch.from_numpy(np.ascontiguousarray(a))
+    if pin:
+        t = t.pin_memory()
+    if device is not None:
+        t = t.to(device)
+    return t

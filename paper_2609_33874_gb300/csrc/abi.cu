@@ -1,0 +1,235 @@
+// The C entry points of libjet: argument validation, workspace plans and
+// stream-ordered launches. No entry point allocates memory, synchronises a
+// stream (except jet_device_status) or launches anything after a failed
+// check.
+#include <cstdint>
+#include <mutex>
+
+#include "jet.h"
+#include "jet_internal.h"
+
+namespace jet {
+
+// Per-device status word written by kernels that meet an out-of-range layout
+// index or give up a bounded wait.
+__device__ int g_status_word;
+
+int* device_status_ptr() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  static std::mutex mu;
+  static int* ptrs[64] = {};
+  std::lock_guard<std::mutex> lock(mu);
+  if (!ptrs[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
+    ptrs[dev] = static_cast<int*>(p);
+  }
+  return ptrs[dev];
+}
+
+cudaError_t launch_lmhead_simt(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
+                               const void* hidden, const void* w_lm, void* ws, int* status,
+                               cudaStream_t st);
+
+cudaError_t launch_lmhead(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
+                          const void* hidden, const void* w_lm, void* ws, int* status,
+                          cudaStream_t st) {
+  return launch_lmhead_simt(lay, d, plan, hidden, w_lm, ws, status, st);
+}
+
+}  // namespace jet
+
+namespace {
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// A device pointer argument: non-null and 16-byte aligned when it will be
+// touched (count > 0).
+jet_status check_ptr(const void* p, long long count) {
+  if (count <= 0) return JET_OK;
+  if (!p) return JET_ERR_ARG;
+  if (!aligned16(p)) return JET_ERR_ALIGN;
+  return JET_OK;
+}
+
+jet_status check_layout(const jet_layout* lay) {
+  if (!lay) return JET_ERR_ARG;
+  const jet_sizes& n = lay->n;
+  if (n.R < 0 || n.C < 0 || n.N < 0 || n.T < 0 || n.V < 1) return JET_ERR_SHAPE;
+  if (n.R == 0) return JET_OK;
+  if (n.C < n.R || n.N < n.R || n.T < n.C || n.total_prefix < n.R || n.max_prefix < 1 ||
+      n.max_prefix > n.total_prefix || n.min_cand < 1 || n.max_cand < n.min_cand ||
+      n.max_rows < 1 || n.max_rows > n.N || n.max_len < 1 || n.N - n.R != n.T - n.C)
+    return JET_ERR_SHAPE;
+  const void* arrays[12] = {lay->prefix_offset, lay->cand_offset,    lay->row_offset,
+                            lay->cand_row_offset, lay->tgt_offset,   lay->target_ids,
+                            lay->tgt_row,       lay->row_req,        lay->row_cand,
+                            lay->row_pos,       lay->row_tgt_offset, lay->row_tgt_index};
+  for (const void* a : arrays)
+    if (!a) return JET_ERR_ARG;
+  return JET_OK;
+}
+
+jet_status check_dtype(const jet_dims* d) {
+  if (!d) return JET_ERR_ARG;
+  if (d->dtype != JET_DTYPE_F32 && d->dtype != JET_DTYPE_BF16) return JET_ERR_UNSUPPORTED;
+  return JET_OK;
+}
+
+jet_status check_attn_dims(const jet_dims* d) {
+  jet_status s = check_dtype(d);
+  if (s) return s;
+  if (d->Hq < 1 || d->Hkv < 1 || d->Hq % d->Hkv != 0) return JET_ERR_SHAPE;
+  if (d->d != 64 && d->d != 128 && d->d != 256) return JET_ERR_UNSUPPORTED;
+  return JET_OK;
+}
+
+jet_status check_lm_dims(const jet_dims* d) {
+  jet_status s = check_dtype(d);
+  if (s) return s;
+  if (d->D < 8 || d->D % 8 != 0) return JET_ERR_SHAPE;
+  return JET_OK;
+}
+
+jet_status check_fork_dims(const jet_dims* d) {
+  jet_status s = check_dtype(d);
+  if (s) return s;
+  if (d->Hl < 1 || d->dk < 1 || d->dv < 1) return JET_ERR_SHAPE;
+  if (d->dk != 128 || d->dv % 32 != 0) return JET_ERR_UNSUPPORTED;
+  return JET_OK;
+}
+
+jet_status cuda_status(cudaError_t e) { return e == cudaSuccess ? JET_OK : JET_ERR_CUDA; }
+
+#define JET_TRY(expr)            \
+  do {                           \
+    jet_status s_ = (expr);      \
+    if (s_ != JET_OK) return s_; \
+  } while (0)
+
+}  // namespace
+
+extern "C" int32_t jet_abi_version(void) { return JET_ABI_VERSION; }
+
+extern "C" const char* jet_status_string(jet_status s) {
+  switch (s) {
+    case JET_OK: return "ok";
+    case JET_ERR_ARG: return "invalid argument (null pointer or bad scalar)";
+    case JET_ERR_SHAPE: return "inconsistent sizes";
+    case JET_ERR_RANGE: return "token id outside [0, V)";
+    case JET_ERR_ALIGN: return "device pointer not 16-byte aligned";
+    case JET_ERR_WORKSPACE: return "workspace missing or too small";
+    case JET_ERR_CAPACITY: return "size beyond kernel capacity";
+    case JET_ERR_UNSUPPORTED: return "unsupported dtype or dimension";
+    case JET_ERR_CUDA: return "CUDA runtime error";
+    case JET_ERR_TIMEOUT: return "bounded device wait gave up";
+    case JET_ERR_DEVICE: return "kernel met an out-of-range layout index";
+    default: return "unknown status";
+  }
+}
+
+extern "C" size_t jet_workspace_bytes(const jet_sizes* n, const jet_dims* d) {
+  if (!n || !d || n->R < 0 || n->N < 0 || n->V < 1) return 0;
+  size_t a = 0, b = 0;
+  if (d->Hq > 0 && d->Hkv > 0 && d->Hq % d->Hkv == 0 && d->d > 0) a = jet::attn_plan(*n, *d).bytes;
+  b = jet::score_plan(*n).bytes;
+  return a > b ? a : b;
+}
+
+extern "C" jet_status jet_prefix_attend(const jet_layout* lay, const jet_dims* dims, const void* q,
+                                        const void* k_pre, const void* v_pre, const void* k_cand,
+                                        const void* v_cand, void* o, void* ws, size_t ws_bytes,
+                                        void* stream) {
+  JET_TRY(check_layout(lay));
+  JET_TRY(check_attn_dims(dims));
+  const jet_sizes& n = lay->n;
+  if (n.R == 0) return JET_OK;
+  if ((long long)n.R * dims->Hkv > 65535) return JET_ERR_CAPACITY;
+  const long long F = n.N - n.R;
+  JET_TRY(check_ptr(q, n.N));
+  JET_TRY(check_ptr(k_pre, n.total_prefix));
+  JET_TRY(check_ptr(v_pre, n.total_prefix));
+  JET_TRY(check_ptr(k_cand, F));
+  JET_TRY(check_ptr(v_cand, F));
+  JET_TRY(check_ptr(o, n.N));
+  const jet::AttnPlan plan = jet::attn_plan(n, *dims);
+  if (!ws || ws_bytes < plan.bytes) return JET_ERR_WORKSPACE;
+  if (!aligned16(ws)) return JET_ERR_ALIGN;
+  return cuda_status(jet::launch_prefix_attend(*lay, *dims, plan, q, k_pre, v_pre, k_cand, v_cand, o,
+                                               ws, jet::device_status_ptr(),
+                                               static_cast<cudaStream_t>(stream)));
+}
+
+extern "C" jet_status jet_fork_state(const jet_layout* lay, const jet_dims* dims,
+                                     const float* s_prefix, const void* q, const void* k,
+                                     const void* v, const float* alpha, const float* beta, void* o,
+                                     float* s_fork, void* stream) {
+  JET_TRY(check_layout(lay));
+  JET_TRY(check_fork_dims(dims));
+  const jet_sizes& n = lay->n;
+  if (n.R == 0) return JET_OK;
+  if (n.R > 65535 || dims->Hl > 65535) return JET_ERR_CAPACITY;
+  const long long F = n.N - n.R;
+  JET_TRY(check_ptr(s_prefix, n.R));
+  JET_TRY(check_ptr(q, F));
+  JET_TRY(check_ptr(k, F));
+  JET_TRY(check_ptr(v, F));
+  JET_TRY(check_ptr(alpha, F));
+  JET_TRY(check_ptr(beta, F));
+  JET_TRY(check_ptr(o, F));
+  if (s_fork && !aligned16(s_fork)) return JET_ERR_ALIGN;
+  return cuda_status(jet::launch_fork_state(*lay, *dims, s_prefix, q, k, v, alpha, beta, o, s_fork,
+                                            jet::device_status_ptr(),
+                                            static_cast<cudaStream_t>(stream)));
+}
+
+extern "C" jet_status jet_score_candidates(const jet_layout* lay, const jet_dims* dims,
+                                           const void* hidden, const void* w_lm,
+                                           float* tok_logprob, float* cand_score, void* ws,
+                                           size_t ws_bytes, void* stream) {
+  JET_TRY(check_layout(lay));
+  JET_TRY(check_lm_dims(dims));
+  const jet_sizes& n = lay->n;
+  if (n.R == 0) return JET_OK;
+  const jet::ScorePlan plan = jet::score_plan(n);
+  if (plan.vtiles > 65535) return JET_ERR_CAPACITY;
+  JET_TRY(check_ptr(hidden, n.N));
+  JET_TRY(check_ptr(w_lm, n.V));
+  JET_TRY(check_ptr(tok_logprob, n.T));
+  JET_TRY(check_ptr(cand_score, n.C));
+  if (!ws || ws_bytes < plan.bytes) return JET_ERR_WORKSPACE;
+  if (!aligned16(ws)) return JET_ERR_ALIGN;
+  int* status = jet::device_status_ptr();
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  JET_TRY(cuda_status(jet::launch_lmhead(*lay, *dims, plan, hidden, w_lm, ws, status, st)));
+  return cuda_status(jet::launch_score_finish(*lay, plan, ws, tok_logprob, cand_score, status, st));
+}
+
+extern "C" jet_status jet_decide(const jet_layout* lay, int32_t mode, const float* cand_score,
+                                 float* q, int32_t* choice, float* value, void* stream) {
+  JET_TRY(check_layout(lay));
+  if (mode != JET_DECIDE_ARGMAX && mode != JET_DECIDE_BINARY && mode != JET_DECIDE_ORDINAL)
+    return JET_ERR_ARG;
+  const jet_sizes& n = lay->n;
+  if (n.R == 0) return JET_OK;
+  if (mode == JET_DECIDE_BINARY && (n.min_cand != 2 || n.max_cand != 2)) return JET_ERR_SHAPE;
+  JET_TRY(check_ptr(cand_score, n.C));
+  JET_TRY(check_ptr(q, n.C));
+  JET_TRY(check_ptr(choice, n.R));
+  JET_TRY(check_ptr(value, n.R));
+  return cuda_status(jet::launch_decide(*lay, mode, cand_score, q, choice, value,
+                                        jet::device_status_ptr(),
+                                        static_cast<cudaStream_t>(stream)));
+}
+
+extern "C" jet_status jet_device_status(void* stream, jet_status* out) {
+  if (!out) return JET_ERR_ARG;
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return JET_ERR_CUDA;
+  int v = 0;
+  if (cudaMemcpyFromSymbol(&v, jet::g_status_word, sizeof(int)) != cudaSuccess) return JET_ERR_CUDA;
+  const int zero = 0;
+  if (cudaMemcpyToSymbol(jet::g_status_word, &zero, sizeof(int)) != cudaSuccess) return JET_ERR_CUDA;
+  *out = v;
+  return JET_OK;
+}

@@ -1,0 +1,165 @@
+// Per-candidate fork of a linear-attention recurrent state (Sec. 4.1).
+//
+// The paper keeps one stored prefix state and restores it before each
+// candidate, evaluating candidates one after another. Here every candidate
+// of a request runs concurrently inside one CTA from a single read of the
+// prefix state: the state slice stays in registers, each candidate starts
+// from an unmodified copy of it, applies its fed tokens and writes its own
+// final state. Each fed token applies the gated delta rule
+//   S <- alpha (S - beta k (k^T S)) + beta k v^T,   o = S^T q / sqrt(dk)
+// (the paper does not state its recurrence; this is the reading used).
+// The update is column-separable: column j of S needs only k, v_j and the
+// column's own u_j = k^T S[:, j], so a CTA owns a 32-column slice of one
+// head. The kernel is bound by the writes of the forked states.
+#include "jet_device.cuh"
+#include "jet_internal.h"
+
+namespace jet {
+namespace {
+
+constexpr int kDK = 128;        // key dimension handled (rows of S)
+constexpr int kCols = 32;       // value columns per CTA
+constexpr int kThreads = 128;   // 4 warps x 32 rows
+
+__device__ __forceinline__ float4 f4_fma(float a, float4 x, float4 y) {
+  return make_float4(fmaf(a, x.x, y.x), fmaf(a, x.y, y.y), fmaf(a, x.z, y.z), fmaf(a, x.w, y.w));
+}
+
+// Reduce a per-thread float4 over the 128 rows of the slice; every thread
+// receives the 4 column sums of its column quad. `red` holds 4 x 32 floats.
+__device__ __forceinline__ float4 rows_sum(float4 v, float* red, int warp, int lane) {
+#pragma unroll
+  for (int o = 8; o <= 16; o <<= 1) {
+    v.x += __shfl_xor_sync(0xffffffffu, v.x, o);
+    v.y += __shfl_xor_sync(0xffffffffu, v.y, o);
+    v.z += __shfl_xor_sync(0xffffffffu, v.z, o);
+    v.w += __shfl_xor_sync(0xffffffffu, v.w, o);
+  }
+  const int jq = lane & 7;
+  if (lane < 8) reinterpret_cast<float4*>(red)[warp * 8 + jq] = v;
+  __syncthreads();
+  float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+  for (int w = 0; w < 4; ++w) {
+    const float4 t = reinterpret_cast<const float4*>(red)[w * 8 + jq];
+    s.x += t.x; s.y += t.y; s.z += t.z; s.w += t.w;
+  }
+  __syncthreads();
+  return s;
+}
+
+// grid (dv / 32, Hl, R); thread (warp w, lane = 8 * rg + jq) owns rows
+// 32 w + rg + 4 ii (ii < 8) and columns j0 + 4 jq .. + 3 of the slice.
+template <typename T>
+__global__ void __launch_bounds__(kThreads)
+fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__ cand_row_offset,
+            const int32_t* __restrict__ tgt_offset, int R, int C, int F, int Hl, int dv,
+            const float* __restrict__ s_prefix, const T* __restrict__ q, const T* __restrict__ k,
+            const T* __restrict__ v, const float* __restrict__ alpha, const float* __restrict__ beta,
+            T* __restrict__ o, float* __restrict__ s_fork, int* status) {
+  __shared__ __align__(16) float red[4 * kCols];
+  const int r = blockIdx.z, h = blockIdx.y, j0 = blockIdx.x * kCols;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int rg = lane >> 3, jq = lane & 7;
+  const int col = j0 + 4 * jq;
+  if (r >= R) return;
+  const int c0 = cand_offset[r], c1 = cand_offset[r + 1];
+  if (c0 < 0 || c1 < c0 || c1 > C) {
+    if (threadIdx.x == 0) flag(status, JET_ERR_DEVICE);
+    return;
+  }
+
+  // the prefix state slice: read once, reused by every candidate
+  float4 sp[8];
+  const size_t head = (size_t(r) * Hl + h) * kDK;
+#pragma unroll
+  for (int ii = 0; ii < 8; ++ii) {
+    const int i = 32 * warp + rg + 4 * ii;
+    sp[ii] = *reinterpret_cast<const float4*>(s_prefix + (head + i) * dv + col);
+  }
+  const float rs = rsqrtf(float(kDK));
+
+  for (int c = c0; c < c1; ++c) {
+    const int m = tgt_offset[c + 1] - tgt_offset[c];
+    const int f0 = cand_row_offset[c] - r - 1;  // fed-token index of y_{c,1}
+    if (m < 1 || f0 < 0 || f0 + m - 1 > F) {
+      if (threadIdx.x == 0) flag(status, JET_ERR_DEVICE);
+      continue;
+    }
+    float4 S[8];
+#pragma unroll
+    for (int ii = 0; ii < 8; ++ii) S[ii] = sp[ii];  // restore the prefix state
+    for (int t = 0; t < m - 1; ++t) {
+      const size_t fh = size_t(f0 + t) * Hl + h;
+      float kk[8], qq[8];
+#pragma unroll
+      for (int ii = 0; ii < 8; ++ii) {
+        const int i = 32 * warp + rg + 4 * ii;
+        kk[ii] = to_f32(k[fh * kDK + i]);
+        qq[ii] = to_f32(q[fh * kDK + i]);
+      }
+      const float a = alpha[fh], b = beta[fh];
+      const float4 vv = make_float4(to_f32(v[fh * dv + col]), to_f32(v[fh * dv + col + 1]),
+                                    to_f32(v[fh * dv + col + 2]), to_f32(v[fh * dv + col + 3]));
+      // u = k^T S for this column quad
+      float4 u = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int ii = 0; ii < 8; ++ii) u = f4_fma(kk[ii], S[ii], u);
+      u = rows_sum(u, red, warp, lane);
+      // S = alpha S + beta k (v - alpha u)
+      const float4 w = make_float4(b * (vv.x - a * u.x), b * (vv.y - a * u.y),
+                                   b * (vv.z - a * u.z), b * (vv.w - a * u.w));
+      float4 op = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int ii = 0; ii < 8; ++ii) {
+        float4 s = S[ii];
+        s = make_float4(fmaf(kk[ii], w.x, a * s.x), fmaf(kk[ii], w.y, a * s.y),
+                        fmaf(kk[ii], w.z, a * s.z), fmaf(kk[ii], w.w, a * s.w));
+        S[ii] = s;
+        op = f4_fma(qq[ii], s, op);
+      }
+      op = rows_sum(op, red, warp, lane);
+      if (warp == 0 && rg == 0) {
+        T* dst = o + fh * dv + col;
+        dst[0] = from_f32<T>(op.x * rs);
+        dst[1] = from_f32<T>(op.y * rs);
+        dst[2] = from_f32<T>(op.z * rs);
+        dst[3] = from_f32<T>(op.w * rs);
+      }
+    }
+    if (s_fork) {
+      const size_t fhead = (size_t(c) * Hl + h) * kDK;
+#pragma unroll
+      for (int ii = 0; ii < 8; ++ii) {
+        const int i = 32 * warp + rg + 4 * ii;
+        *reinterpret_cast<float4*>(s_fork + (fhead + i) * dv + col) = S[ii];
+      }
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, const float* s_prefix,
+                              const void* q, const void* k, const void* v, const float* alpha,
+                              const float* beta, void* o, float* s_fork, int* status,
+                              cudaStream_t st) {
+  const jet_sizes& n = lay.n;
+  dim3 grid(unsigned(d.dv / kCols), unsigned(d.Hl), unsigned(n.R));
+  const int F = n.N - n.R;
+  if (d.dtype == JET_DTYPE_F32) {
+    fork_kernel<float><<<grid, kThreads, 0, st>>>(
+        lay.cand_offset, lay.cand_row_offset, lay.tgt_offset, n.R, n.C, F, d.Hl, d.dv, s_prefix,
+        static_cast<const float*>(q), static_cast<const float*>(k), static_cast<const float*>(v),
+        alpha, beta, static_cast<float*>(o), s_fork, status);
+  } else {
+    fork_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(
+        lay.cand_offset, lay.cand_row_offset, lay.tgt_offset, n.R, n.C, F, d.Hl, d.dv, s_prefix,
+        static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k),
+        static_cast<const __nv_bfloat16*>(v), alpha, beta, static_cast<__nv_bfloat16*>(o), s_fork,
+        status);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace jet

@@ -1,0 +1,61 @@
+// Internal declarations shared by the CUDA translation units of libjet.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "jet.h"
+
+namespace jet {
+
+// ---- per-device status word -------------------------------------------------
+// Device address of the current device's status word (set up once per device);
+// nullptr when the address cannot be obtained.
+int* device_status_ptr();
+
+// ---- workspace plans -----------------------------------------------------------
+constexpr int kVocabTile = 128;  // vocabulary entries per LM-head partial
+
+struct AttnPlan {
+  int splits;    // prefix chunks per (request, key/value head)
+  int chunk;     // prefix keys per chunk (multiple of 32)
+  int qgroups;   // query-vector groups per (request, key/value head)
+  size_t bytes;  // workspace bytes
+};
+AttnPlan attn_plan(const jet_sizes& n, const jet_dims& d);
+
+struct ScorePlan {
+  int vtiles;          // ceil(V / kVocabTile)
+  size_t part_off;     // float2 partials [vtiles][N]
+  size_t ztgt_off;     // float z_tgt[T]
+  size_t lse_off;      // float lse[N]
+  size_t bytes;
+};
+ScorePlan score_plan(const jet_sizes& n);
+
+// ---- kernel launchers (stream-ordered; return the launch error) ---------------
+cudaError_t launch_prefix_attend(const jet_layout& lay, const jet_dims& d, const AttnPlan& plan,
+                                 const void* q, const void* k_pre, const void* v_pre,
+                                 const void* k_cand, const void* v_cand, void* o, void* ws,
+                                 int* status, cudaStream_t st);
+
+cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, const float* s_prefix,
+                              const void* q, const void* k, const void* v, const float* alpha,
+                              const float* beta, void* o, float* s_fork, int* status,
+                              cudaStream_t st);
+
+// logits partials: writes part[vtiles][N] (max, sum exp) and z_tgt[T]
+cudaError_t launch_lmhead(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
+                          const void* hidden, const void* w_lm, void* ws, int* status,
+                          cudaStream_t st);
+
+// lse per row, then l_{c,t} and s(c|x)
+cudaError_t launch_score_finish(const jet_layout& lay, const ScorePlan& plan, void* ws,
+                                float* tok_logprob, float* cand_score, int* status,
+                                cudaStream_t st);
+
+cudaError_t launch_decide(const jet_layout& lay, int mode, const float* cand_score, float* q,
+                          int32_t* choice, float* value, int* status, cudaStream_t st);
+
+}  // namespace jet

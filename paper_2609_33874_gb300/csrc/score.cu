@@ -1,0 +1,155 @@
+// Log-sum-exp merge, token log-probabilities, candidate scores and the
+// decision rules.
+//
+//   lse_n   = m + log sum_tiles s_i exp(m_i - m) over the per-tile partials
+//             (Eq. 2: a = max_v z, lse = a + log sum_v exp(z_v - a))
+//   l_{c,t} = z_{c,t,y} - lse of its row                      (Eq. 1, Eq. 2)
+//   s(c|x)  = sum_t l_{c,t}, summed in t order                (Eq. 3)
+//   q(c)    = exp(s_c - M) / sum_d exp(s_d - M), M = max s     (Eq. 4)
+//   choice  = argmax_c s_c, ties to the lowest index          (Eq. 5, Sec. 3.3)
+#include "jet_device.cuh"
+#include "jet_internal.h"
+
+namespace jet {
+namespace {
+
+// block (32 rows) x 8 tile slices; coalesced reads of part[vt][n]
+__global__ void __launch_bounds__(256)
+lse_kernel(const float2* __restrict__ part, int vtiles, int N, float* __restrict__ lse) {
+  __shared__ float2 red[8][33];
+  const int x = threadIdx.x & 31, y = threadIdx.x >> 5;
+  const int n = blockIdx.x * 32 + x;
+  float m = -INFINITY, s = 0.f;
+  if (n < N)
+    for (int vt = y; vt < vtiles; vt += 8) {
+      const float2 p = part[size_t(vt) * N + n];
+      ms_combine(m, s, p.x, p.y);
+    }
+  red[y][x] = make_float2(m, s);
+  __syncthreads();
+  if (y == 0 && n < N) {
+    for (int i = 1; i < 8; ++i) ms_combine(m, s, red[i][x].x, red[i][x].y);
+    lse[n] = m + __logf(s);
+  }
+}
+
+// one thread per candidate: its targets in t order
+__global__ void finish_kernel(const int32_t* __restrict__ tgt_offset, const int32_t* __restrict__ tgt_row,
+                              int C, int N, int T_, const float* __restrict__ z_tgt,
+                              const float* __restrict__ lse, float* __restrict__ tok_logprob,
+                              float* __restrict__ cand_score, int* status) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= C) return;
+  const int j0 = tgt_offset[c], j1 = tgt_offset[c + 1];
+  if (j0 < 0 || j1 < j0 || j1 > T_) {
+    flag(status, JET_ERR_DEVICE);
+    return;
+  }
+  float acc = 0.f;
+  for (int j = j0; j < j1; ++j) {
+    const int n = tgt_row[j];
+    if (n < 0 || n >= N) {
+      flag(status, JET_ERR_DEVICE);
+      continue;
+    }
+    const float ell = z_tgt[j] - lse[n];
+    tok_logprob[j] = ell;
+    acc += ell;
+  }
+  cand_score[c] = acc;
+}
+
+// one warp per request
+__global__ void __launch_bounds__(256)
+decide_kernel(const int32_t* __restrict__ cand_offset, int R, int C, int mode,
+              const float* __restrict__ s, float* __restrict__ q, int32_t* __restrict__ choice,
+              float* __restrict__ value, int* status) {
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (r >= R) return;
+  const int c0 = cand_offset[r], c1 = cand_offset[r + 1];
+  if (c0 < 0 || c1 <= c0 || c1 > C) {
+    if (lane == 0) flag(status, JET_ERR_DEVICE);
+    return;
+  }
+  // M = max s, and the lowest index attaining it
+  float best = -INFINITY;
+  int arg = 0x7fffffff;
+  for (int c = c0 + lane; c < c1; c += 32) {
+    const float v = s[c];
+    if (v > best) {  // strict: a lane keeps its lowest index among equals
+      best = v;
+      arg = c - c0;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+    const int oa = __shfl_xor_sync(0xffffffffu, arg, o);
+    if (ob > best || (ob == best && oa < arg)) {
+      best = ob;
+      arg = oa;
+    }
+  }
+  if (arg == 0x7fffffff) arg = 0;  // no finite score: fall back to the first candidate
+  float sum = 0.f;
+  for (int c = c0 + lane; c < c1; c += 32) sum += __expf(s[c] - best);
+  sum = warp_sum(sum);
+  const float inv = 1.f / sum;
+  float ev = 0.f;
+  for (int c = c0 + lane; c < c1; c += 32) {
+    const float qc = __expf(s[c] - best) * inv;
+    q[c] = qc;
+    ev += float(c - c0) * qc;
+  }
+  ev = warp_sum(ev);
+  if (lane == 0) {
+    choice[r] = arg;
+    if (mode == JET_DECIDE_BINARY)
+      value[r] = (c1 - c0 == 2) ? __expf(s[c0 + 1] - best) * inv : __int_as_float(0x7fc00000);
+    else if (mode == JET_DECIDE_ORDINAL)
+      value[r] = ev;
+    else
+      value[r] = inv;  // q of the argmax: exp(0) / sum
+  }
+}
+
+}  // namespace
+
+ScorePlan score_plan(const jet_sizes& n) {
+  ScorePlan p{};
+  auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
+  p.vtiles = (n.V + kVocabTile - 1) / kVocabTile;
+  p.part_off = 0;
+  p.ztgt_off = up(size_t(p.vtiles) * n.N * sizeof(float2));
+  p.lse_off = p.ztgt_off + up(size_t(n.T) * sizeof(float));
+  p.bytes = p.lse_off + up(size_t(n.N) * sizeof(float));
+  return p;
+}
+
+cudaError_t launch_score_finish(const jet_layout& lay, const ScorePlan& plan, void* ws,
+                                float* tok_logprob, float* cand_score, int* status,
+                                cudaStream_t st) {
+  const jet_sizes& n = lay.n;
+  char* base = static_cast<char*>(ws);
+  const float2* part = reinterpret_cast<const float2*>(base + plan.part_off);
+  const float* z_tgt = reinterpret_cast<const float*>(base + plan.ztgt_off);
+  float* lse = reinterpret_cast<float*>(base + plan.lse_off);
+  lse_kernel<<<unsigned((n.N + 31) / 32), 256, 0, st>>>(part, plan.vtiles, n.N, lse);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  finish_kernel<<<unsigned((n.C + 127) / 128), 128, 0, st>>>(lay.tgt_offset, lay.tgt_row, n.C, n.N,
+                                                             n.T, z_tgt, lse, tok_logprob,
+                                                             cand_score, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decide(const jet_layout& lay, int mode, const float* cand_score, float* q,
+                          int32_t* choice, float* value, int* status, cudaStream_t st) {
+  const jet_sizes& n = lay.n;
+  decide_kernel<<<unsigned((n.R + 7) / 8), 256, 0, st>>>(lay.cand_offset, n.R, n.C, mode,
+                                                         cand_score, q, choice, value, status);
+  return cudaGetLastError();
+}
+
+}  // namespace jet

@@ -1,0 +1,109 @@
+"""One teacher-forced candidate-scoring step: attend -> (fork) -> score -> decide.
+
+:class:`ScoringStep` owns the device buffers of one batch shape (the layout,
+outputs and workspace) and strings the C entry points together on one CUDA
+stream. Inputs are torch tensors already on the device (:meth:`run`) or pinned
+host tensors that are copied in first (:meth:`run_from_host`, the end-to-end
+path: host -> device copies, the kernels, device -> host copies of the
+results).
+"""
+from __future__ import annotations
+
+from typing import Dict, Optional
+
+import torch
+
+from . import jet
+
+_TORCH_DTYPE = {jet.DTYPE_F32: torch.float32, jet.DTYPE_BF16: torch.bfloat16}
+
+# per-batch inputs of the step; the LM-head weights are model state and stay resident
+ATTN_INPUTS = ("q", "k_pre", "v_pre", "k_cand", "v_cand")
+FORK_INPUTS = ("s_prefix", "lq", "lk", "lv", "alpha", "beta")
+RESULTS = ("tok_logprob", "cand_score", "q_cand", "choice", "value")
+
+
+class ScoringStep:
+    """Device state of one batch shape.
+
+    ``layout`` is a :class:`jet.HostLayout`; ``dims`` a :class:`jet.jet_dims`;
+    ``mode`` one of ``jet.DECIDE_*``. ``hybrid`` adds the linear-attention
+    fork; ``keep_fork_state`` also writes every candidate's final recurrent
+    state. ``chain`` feeds the attention output to the LM head (requires
+    Hq * d == D).
+    """
+
+    def __init__(self, layout: "jet.HostLayout", dims: "jet.jet_dims", mode: int,
+                 device="cuda", hybrid: bool = False, keep_fork_state: bool = False,
+                 chain: bool = False):
+        self.dev = torch.device(device)
+        self.host_layout = layout
+        self.layout = layout.to_device(self.dev)
+        self.dims, self.mode, self.hybrid, self.chain = dims, int(mode), hybrid, chain
+        n = layout.sizes
+        self.R, self.C, self.N, self.T = n.R, n.C, n.N, n.T
+        self.F = n.N - n.R
+        if chain and dims.Hq * dims.d != dims.D:
+            raise ValueError("chain needs Hq * d == D")
+        dt = _TORCH_DTYPE[dims.dtype]
+        z = lambda *s, dtype=torch.float32: torch.empty(*s, dtype=dtype, device=self.dev)  # noqa: E731
+        self.o = z(n.N, dims.Hq, dims.d, dtype=dt)
+        self.tok_logprob = z(n.T)
+        self.cand_score = z(n.C)
+        self.q_cand = z(n.C)
+        self.choice = z(n.R, dtype=torch.int32)
+        self.value = z(n.R)
+        ws = jet.jet_workspace_bytes(n, dims)
+        self.ws = z((ws + 15) // 16 * 4)  # float32 words, 16-byte multiple
+        if hybrid:
+            self.lo = z(self.F, dims.Hl, dims.dv, dtype=dt)
+            self.s_fork = z(n.C, dims.Hl, dims.dk, dims.dv) if keep_fork_state else None
+        self._dev_inputs: Optional[Dict[str, torch.Tensor]] = None
+
+    # ------------------------------------------------------------------
+    def run(self, x: Dict[str, torch.Tensor], w_lm: torch.Tensor, stream=None) -> None:
+        """Enqueue the whole step on ``stream`` (default: the current stream).
+
+        ``x`` holds q, k_pre, v_pre, k_cand, v_cand, hidden (unless chained)
+        and, for a hybrid step, s_prefix, lq, lk, lv, alpha, beta.
+        """
+        d, lay = self.dims, self.layout
+        jet.jet_prefix_attend(lay, d, x["q"], x["k_pre"], x["v_pre"], x["k_cand"], x["v_cand"],
+                              self.o, self.ws, stream=stream)
+        if self.hybrid:
+            jet.jet_fork_state(lay, d, x["s_prefix"], x["lq"], x["lk"], x["lv"], x["alpha"],
+                               x["beta"], self.lo, self.s_fork, stream=stream)
+        hidden = self.o.view(self.N, d.Hq * d.d) if self.chain else x["hidden"]
+        jet.jet_score_candidates(lay, d, hidden, w_lm, self.tok_logprob, self.cand_score, self.ws,
+                                 stream=stream)
+        jet.jet_decide(lay, self.mode, self.cand_score, self.q_cand, self.choice, self.value,
+                       stream=stream)
+
+    def input_names(self):
+        names = list(ATTN_INPUTS) + ([] if self.chain else ["hidden"])
+        return names + (list(FORK_INPUTS) if self.hybrid else [])
+
+    def run_from_host(self, host: Dict[str, torch.Tensor], layout_words: torch.Tensor,
+                      w_lm: torch.Tensor, out: Dict[str, torch.Tensor], stream=None) -> None:
+        """End-to-end step: copy the batch's pinned host inputs (and its layout
+        words) to the device, run the step, copy the results into the pinned
+        host tensors of ``out`` (tok_logprob, cand_score, q_cand, choice,
+        value). Everything is enqueued on ``stream``; the caller synchronises."""
+        s = torch.cuda.current_stream(self.dev) if stream is None else stream
+        with torch.cuda.stream(s):
+            if self._dev_inputs is None:
+                self._dev_inputs = {k: torch.empty_like(host[k], device=self.dev)
+                                    for k in self.input_names()}
+            self.layout.words.copy_(layout_words, non_blocking=True)
+            for k in self.input_names():
+                self._dev_inputs[k].copy_(host[k], non_blocking=True)
+            self.run(self._dev_inputs, w_lm, stream=s)
+            for k in RESULTS:
+                out[k].copy_(getattr(self, k), non_blocking=True)
+
+    def host_bytes(self, host: Dict[str, torch.Tensor], layout_words: torch.Tensor):
+        """(host->device, device->host) bytes one :meth:`run_from_host` moves."""
+        h2d = layout_words.numel() * layout_words.element_size()
+        h2d += sum(host[k].numel() * host[k].element_size() for k in self.input_names())
+        d2h = sum(getattr(self, k).numel() * getattr(self, k).element_size() for k in RESULTS)
+        return h2d, d2h

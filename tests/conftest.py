@@ -15,3 +15,12 @@ def pytest_configure(config):
 @pytest.fixture(scope="session")
 def repo_root():
     return ROOT
+
+
+@pytest.fixture(scope="session")
+def jet():
+    """The ctypes binding, building libjet.so first when it is missing or stale."""
+    from paper_2609_33874_gb300 import build as _build
+    _build.build()
+    from paper_2609_33874_gb300 import jet as _jet
+    return _jet

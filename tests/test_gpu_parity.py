@@ -1,0 +1,194 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 oracle on the
+same seeded inputs. Small cases compare every output; the full-size workloads
+(in the launch configuration the benchmark times) compare sampled requests
+and rows, plus properties that hold at any size."""
+import numpy as np
+import pytest
+
+import jet_synth
+import oracle as O
+from gpu_common import (TOL_ATTN_BF16, TOL_ATTN_F32, build_step, check_attention, check_fork,
+                        check_invariants, check_scores, oracle_layout, run_problem)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def cuda(jet):
+    import torch
+    if not torch.cuda.is_available():
+        pytest.fail("CUDA device required for -m gpu tests")
+    return jet
+
+
+def _custom(base, prefix_len, n_cand, cand_len, seed=3, **over):
+    import dataclasses
+    w = dataclasses.replace(jet_synth.WORKLOADS[base], **over)
+    rng = np.random.default_rng(seed)
+    ids = rng.integers(0, w.V, size=int(np.sum(cand_len)))
+    return jet_synth.custom_problem(w, prefix_len, n_cand, cand_len, ids, seed=seed)
+
+
+# ---------------------------------------------------------------------------
+# tiny workload (float32): every output
+# ---------------------------------------------------------------------------
+def test_tiny_full_step(cuda):
+    p = jet_synth.make_problem("tiny")
+    got, _ = run_problem(cuda, p)
+    lay = oracle_layout(p)
+    check_attention(lay, p, got["o"], list(range(p.N)), TOL_ATTN_F32)
+    check_scores(lay, p, got, [0])
+    check_invariants(lay, got)
+
+
+def test_tiny_chained(cuda):
+    # the attention output feeds the LM head (Hq * d == D)
+    p = jet_synth.make_problem("tiny")
+    got, _ = run_problem(cuda, p, chain=True)
+    lay = oracle_layout(p)
+    o = O.cascade_attention(lay, p.f32("q"), p.f32("k_pre"), p.f32("v_pre"), p.f32("k_cand"),
+                            p.f32("v_cand"), 8, 2)
+    check_scores(lay, p, got, [0], hidden=o.reshape(p.N, -1))
+
+
+# ---------------------------------------------------------------------------
+# attention: ragged prefixes, head dims, dtypes, edge cases
+# ---------------------------------------------------------------------------
+ATTN_CASES = [
+    # (base, prefix_len, n_cand, cand_len, overrides)
+    ("tiny", [1], [1], [1], {}),                                   # P = 1, one token
+    ("tiny", [33, 95, 64], [2, 1, 3], [1, 5, 2, 3, 1, 4], {}),     # ragged tails of 32-key tiles
+    ("tiny", [700], [4], [12, 1, 7, 3], dict(dtype="bf16")),
+    ("tiny", [257, 31], [3, 2], [2, 2, 2, 1, 9], dict(Hq=6, Hkv=3, d=128, dtype="bf16")),
+    ("tiny", [513, 129, 1000], [4, 4, 1], [1, 3, 1, 2, 5, 1, 1, 2, 1], dict(Hq=24, Hkv=4, d=256,
+                                                                          dtype="bf16")),
+    ("tiny", [5, 6], [1, 1], [1, 1], dict(Hq=4, Hkv=4, d=64)),     # no fed tokens at all
+]
+
+
+@pytest.mark.parametrize("case", range(len(ATTN_CASES)))
+def test_attention_cases(cuda, case):
+    base, pl, nc, cl, over = ATTN_CASES[case]
+    p = _custom(base, pl, nc, cl, seed=10 + case, **over)
+    got, _ = run_problem(cuda, p)
+    lay = oracle_layout(p)
+    tol = TOL_ATTN_BF16 if p.bf16 else TOL_ATTN_F32
+    check_attention(lay, p, got["o"], list(range(p.N)), tol)
+
+
+# ---------------------------------------------------------------------------
+# LM head: ragged vocabulary and rows, targets at the vocabulary edges
+# ---------------------------------------------------------------------------
+LM_CASES = [
+    (dict(V=1000, D=72), [4, 9], [3, 2], [1, 4, 2, 6, 3]),          # V % 128 != 0, D % 32 != 0
+    (dict(V=129, D=64, dtype="bf16"), [2], [5], [1, 1, 2, 1, 40]),  # 41 rows, one vocab tail
+    (dict(V=20000, D=256, dtype="bf16", w_std=0.05), [3] * 7, [4] * 7, [3] * 28),
+    (dict(V=8192, D=512, dtype="bf16"), [1] * 3, [1, 2, 3], [1, 12, 1, 1, 2, 3]),
+]
+
+
+@pytest.mark.parametrize("case", range(len(LM_CASES)))
+def test_lm_head_cases(cuda, case):
+    over, pl, nc, cl = LM_CASES[case]
+    p = _custom("tiny", pl, nc, cl, seed=20 + case, **over)
+    # targets at 0 and V - 1
+    p.target_ids[0] = 0
+    p.target_ids[-1] = p.work.V - 1
+    got, _ = run_problem(cuda, p)
+    lay = oracle_layout(p)
+    check_scores(lay, p, got, list(range(p.R)))
+    check_invariants(lay, got)
+
+
+def test_all_vocabulary_targets_sum_to_one(cuda):
+    # one request with every vocabulary entry as a single-token candidate:
+    # the GPU's probabilities over V sum to one (Eq. 1)
+    V = 3000
+    w = dict(V=V, D=128, dtype="bf16")
+    p = _custom("tiny", [7], [V], [1] * V, seed=30, **w)
+    p.target_ids[:] = np.arange(V)
+    got, _ = run_problem(cuda, p)
+    assert abs(np.exp(got["ell"].astype(np.float64)).sum() - 1.0) < 1e-4
+    check_scores(oracle_layout(p), p, got, [0])
+
+
+# ---------------------------------------------------------------------------
+# recurrent-state fork
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("keep", [True, False])
+def test_fork_small(cuda, keep):
+    p = _custom("ordinal_hybrid", [3, 4, 2], [10, 3, 1], [1, 2, 3, 1, 1, 3, 2, 2, 1, 3, 4, 1, 6, 1],
+                seed=40, V=4096, D=256, Hl=3, dv=64)
+    got, _ = run_problem(cuda, p, keep_fork=keep)
+    lay = oracle_layout(p)
+    check_fork(lay, p, got, list(range(p.R)))
+    check_scores(lay, p, got, list(range(p.R)))
+
+
+# ---------------------------------------------------------------------------
+# full-size workloads: sampled outputs against the oracle
+# ---------------------------------------------------------------------------
+FULL = {
+    "dense27b_mc": dict(requests=[0, 7, 15], rows=12),
+    "binary": dict(requests=[0, 31, 63], rows=12),
+    "ordinal_hybrid": dict(requests=[0, 17, 31], rows=12),
+    "moe_a3b_long": dict(requests=[0, 100, 255], rows=8),
+}
+
+
+@pytest.mark.parametrize("name", list(FULL))
+def test_full_size_workload(cuda, name):
+    p = jet_synth.make_problem(name)
+    got, _ = run_problem(cuda, p, keep_fork=True)
+    lay = oracle_layout(p)
+    check_invariants(lay, got)
+    req = FULL[name]["requests"]
+    check_scores(lay, p, got, req)
+    rng = np.random.default_rng(5)
+    rows = []
+    for r in req:
+        n0, n1 = int(lay["row_offset"][r]), int(lay["row_offset"][r + 1])
+        rows.extend(rng.choice(np.arange(n0, n1), size=min(FULL[name]["rows"] // len(req) + 1,
+                                                            n1 - n0), replace=False).tolist())
+    check_attention(lay, p, got["o"], sorted(set(rows)), TOL_ATTN_BF16)
+    if p.work.Hl:
+        check_fork(lay, p, got, req)
+
+
+# ---------------------------------------------------------------------------
+# failure detection: an invalid device layout is reported, never faults
+# ---------------------------------------------------------------------------
+def test_corrupt_device_layout_is_flagged(cuda):
+    import torch
+    p = jet_synth.make_problem("tiny")
+    step, x, w_lm = build_step(cuda, p)
+    hl = step.host_layout
+    # point one row's target index past T: the LM-head kernel must skip it
+    words = torch.from_numpy(hl.words.copy())
+    off = (hl.struct.row_tgt_index - hl.words.ctypes.data) // 4
+    words[off] = hl.sizes.T + 1000
+    step.layout.words.copy_(words.to(step.layout.words.device))
+    step.run(x, w_lm)
+    assert cuda.jet_device_status() == 10  # JET_ERR_DEVICE
+    assert cuda.jet_device_status() == 0   # cleared by the read
+    step.layout.words.copy_(torch.from_numpy(hl.words).to(step.layout.words.device))
+    step.run(x, w_lm)
+    assert cuda.jet_device_status() == 0
+
+
+def test_end_to_end_from_host(cuda):
+    import torch
+    p = jet_synth.make_problem("tiny")
+    step, _, w_lm = build_step(cuda, p)
+    host = {k: jet_synth.torch_tensor(p, k, pin=True) for k in step.input_names()}
+    words = torch.from_numpy(step.host_layout.words).pin_memory()
+    out = {k: torch.empty_like(getattr(step, k), device="cpu").pin_memory()
+           for k in ("tok_logprob", "cand_score", "q_cand", "choice", "value")}
+    step.run_from_host(host, words, w_lm, out)
+    torch.cuda.synchronize()
+    got = dict(ell=out["tok_logprob"].numpy(), s=out["cand_score"].numpy(),
+               q=out["q_cand"].numpy(), choice=out["choice"].numpy(), value=out["value"].numpy())
+    lay = oracle_layout(p)
+    check_scores(lay, p, got, [0])
+    h2d, d2h = step.host_bytes(host, words)
+    assert h2d > 0 and d2h > 0
