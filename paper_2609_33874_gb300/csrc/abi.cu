@@ -28,13 +28,13 @@ int* device_status_ptr() {
   return ptrs[dev];
 }
 
-cudaError_t launch_lmhead_simt(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
-                               const void* hidden, const void* w_lm, void* ws, int* status,
-                               cudaStream_t st);
-
+// bf16 runs on the tensor cores; float32 keeps float32 FMA (tf32 tensor-core
+// inputs would round it)
 cudaError_t launch_lmhead(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
                           const void* hidden, const void* w_lm, void* ws, int* status,
                           cudaStream_t st) {
+  if (d.dtype == JET_DTYPE_BF16)
+    return launch_lmhead_tc(lay, d, plan, hidden, w_lm, ws, status, st);
   return launch_lmhead_simt(lay, d, plan, hidden, w_lm, ws, status, st);
 }
 

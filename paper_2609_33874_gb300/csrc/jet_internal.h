@@ -45,7 +45,14 @@ cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, const fl
                               const float* beta, void* o, float* s_fork, int* status,
                               cudaStream_t st);
 
-// logits partials: writes part[vtiles][N] (max, sum exp) and z_tgt[T]
+// logits partials: writes part[vtiles][N] (m, s) in base 2 - m = max_v z log2(e),
+// s = sum_v 2^(z log2(e) - m) over the tile - and z_tgt[T]
+cudaError_t launch_lmhead_simt(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
+                               const void* hidden, const void* w_lm, void* ws, int* status,
+                               cudaStream_t st);
+cudaError_t launch_lmhead_tc(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
+                             const void* hidden, const void* w_lm, void* ws, int* status,
+                             cudaStream_t st);
 cudaError_t launch_lmhead(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
                           const void* hidden, const void* w_lm, void* ws, int* status,
                           cudaStream_t st);

@@ -63,19 +63,20 @@ lmhead_simt_kernel(const int32_t* __restrict__ target_ids, const int32_t* __rest
     }
   }
 
-  // epilogue: per row, (max, sum exp) over the tile's vocabulary, target gather
+  // epilogue: per row, base-2 (max, sum) over the tile's vocabulary, target gather
 #pragma unroll
   for (int a = 0; a < 4; ++a) {
     const int n = row0 + 4 * warp + a;
+    constexpr float kLog2e = 1.4426950408889634f;
     float mx = -INFINITY;
 #pragma unroll
     for (int b = 0; b < 4; ++b)
-      if (v0 + lane + 32 * b < V) mx = fmaxf(mx, acc[a][b]);
+      if (v0 + lane + 32 * b < V) mx = fmaxf(mx, acc[a][b] * kLog2e);
     mx = warp_max(mx);
     float s = 0.f;
 #pragma unroll
     for (int b = 0; b < 4; ++b)
-      if (v0 + lane + 32 * b < V) s += __expf(acc[a][b] - mx);
+      if (v0 + lane + 32 * b < V) s += exp2f(acc[a][b] * kLog2e - mx);
     s = warp_sum(s);
     if (n < N) {
       if (lane == 0) part[size_t(vt) * N + n] = make_float2(mx, s);

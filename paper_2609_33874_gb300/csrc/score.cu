@@ -1,8 +1,8 @@
 // Log-sum-exp merge, token log-probabilities, candidate scores and the
 // decision rules.
 //
-//   lse_n   = m + log sum_tiles s_i exp(m_i - m) over the per-tile partials
-//             (Eq. 2: a = max_v z, lse = a + log sum_v exp(z_v - a))
+//   lse_n   = ln 2 (m + log2 sum_tiles s_i 2^(m_i - m)) over the base-2 per-tile
+//             partials (Eq. 2: a = max_v z, lse = a + log sum_v exp(z_v - a))
 //   l_{c,t} = z_{c,t,y} - lse of its row                      (Eq. 1, Eq. 2)
 //   s(c|x)  = sum_t l_{c,t}, summed in t order                (Eq. 3)
 //   q(c)    = exp(s_c - M) / sum_d exp(s_d - M), M = max s     (Eq. 4)
@@ -23,13 +23,13 @@ lse_kernel(const float2* __restrict__ part, int vtiles, int N, float* __restrict
   if (n < N)
     for (int vt = y; vt < vtiles; vt += 8) {
       const float2 p = part[size_t(vt) * N + n];
-      ms_combine(m, s, p.x, p.y);
+      ms_combine2(m, s, p.x, p.y);
     }
   red[y][x] = make_float2(m, s);
   __syncthreads();
   if (y == 0 && n < N) {
-    for (int i = 1; i < 8; ++i) ms_combine(m, s, red[i][x].x, red[i][x].y);
-    lse[n] = m + __logf(s);
+    for (int i = 1; i < 8; ++i) ms_combine2(m, s, red[i][x].x, red[i][x].y);
+    lse[n] = (m + log2f(s)) * 0.6931471805599453f;  // partials are base 2
   }
 }
 

@@ -84,6 +84,11 @@ LM_CASES = [
     (dict(V=129, D=64, dtype="bf16"), [2], [5], [1, 1, 2, 1, 40]),  # 41 rows, one vocab tail
     (dict(V=20000, D=256, dtype="bf16", w_std=0.05), [3] * 7, [4] * 7, [3] * 28),
     (dict(V=8192, D=512, dtype="bf16"), [1] * 3, [1, 2, 3], [1, 12, 1, 1, 2, 3]),
+    # more than 256 rows: two token tiles; hidden size not a multiple of 64
+    (dict(V=5000, D=200, dtype="bf16"), [2] * 3, [10] * 3, [10] * 30),
+    # three token tiles, vocabulary tail of one row
+    (dict(V=1025, D=128, dtype="bf16"), [2] * 6, [10] * 6, [11] * 60),
+    (dict(V=4096, D=64, dtype="bf16"), [2], [1], [1]),                  # a single row
 ]
 
 
