@@ -1,4 +1,7 @@
-// Shared-prefix cascade attention (Sec. 4.1, Fig. 1 "KV-cache text models").
+// Shared-prefix cascade attention (Sec. 4.1, Fig. 1 "KV-cache text models"):
+// float32 prefix kernel, and the merge kernel shared with the bf16
+// tensor-core prefix kernel (attend_tc.cu). Partials are in base 2:
+// m = max of score log2(e), l = sum of 2^(score log2(e) - m).
 //
 // Every row of request r attends to the request's P_r prefix keys; a row fed
 // with y_{c,t} additionally attends to y_{c,1..t} of its own candidate. The
@@ -61,7 +64,7 @@ attend_prefix_kernel(const int32_t* __restrict__ prefix_offset, const int32_t* _
 
   const int tid = threadIdx.x;
   const int vec = tid >> 4, sub = tid & 15;
-  const float scale = rsqrtf(float(DH));
+  const float scale = 1.4426950408889634f * rsqrtf(float(DH));  // base-2 scores
   for (int i = tid; i < kQV * DH; i += kThreads) {
     const int vv = i / DH, dd = i % DH, gv = vbase + vv;
     float x = 0.f;
@@ -110,8 +113,8 @@ attend_prefix_kernel(const int32_t* __restrict__ prefix_offset, const int32_t* _
 #pragma unroll
     for (int o = 8; o > 0; o >>= 1) tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, o));
     const float mn = fmaxf(m, tmax);            // finite: key 0 of the tile is valid
-    const float corr = __expf(m - mn);          // 0 on the first tile
-    const float e0 = __expf(s0 - mn), e1 = __expf(s1 - mn);
+    const float corr = exp2f(m - mn);           // 0 on the first tile
+    const float e0 = exp2f(s0 - mn), e1 = exp2f(s1 - mn);
     float psum = e0 + e1;
 #pragma unroll
     for (int o = 8; o > 0; o >>= 1) psum += __shfl_xor_sync(0xffffffffu, psum, o);
@@ -164,7 +167,7 @@ attend_merge_kernel(const int32_t* __restrict__ row_req, const int32_t* __restri
     const float2 ml = ml_part[base];
     if (!(ml.y > 0.f)) continue;  // empty chunk
     const float mn = fmaxf(m, ml.x);
-    const float a = __expf(m - mn), b = __expf(ml.x - mn);
+    const float a = exp2f(m - mn), b = exp2f(ml.x - mn);
 #pragma unroll
     for (int i = 0; i < PER; ++i) acc[i] = acc[i] * a + o_part[base * DH + lane + 32 * i] * b;
     l = l * a + ml.y * b;
@@ -177,7 +180,7 @@ attend_merge_kernel(const int32_t* __restrict__ row_req, const int32_t* __restri
     if (first < 0 || first > n || r < 0 || first - r - 1 < 0 || n - r - 1 >= N - R) {
       if (lane == 0) flag(status, JET_ERR_DEVICE);
     } else {
-      const float scale = rsqrtf(float(DH));
+      const float scale = 1.4426950408889634f * rsqrtf(float(DH));  // base 2
       float qv[PER];
 #pragma unroll
       for (int i = 0; i < PER; ++i) qv[i] = to_f32(q[(size_t(n) * Hq + h) * DH + lane + 32 * i]) * scale;
@@ -188,7 +191,7 @@ attend_merge_kernel(const int32_t* __restrict__ row_req, const int32_t* __restri
         for (int i = 0; i < PER; ++i) sp = fmaf(qv[i], to_f32(k_cand[kb + 32 * i]), sp);
         const float sc = warp_sum(sp);
         const float mn = fmaxf(m, sc);
-        const float a = __expf(m - mn), b = __expf(sc - mn);
+        const float a = exp2f(m - mn), b = exp2f(sc - mn);
 #pragma unroll
         for (int i = 0; i < PER; ++i) acc[i] = acc[i] * a + b * to_f32(v_cand[kb + 32 * i]);
         l = l * a + b;
@@ -208,16 +211,21 @@ cudaError_t launch_typed(const jet_layout& lay, const jet_dims& d, const AttnPla
   const jet_sizes& n = lay.n;
   float* o_part = static_cast<float*>(ws);
   float2* ml_part = reinterpret_cast<float2*>(o_part + size_t(plan.splits) * n.N * d.Hq * DH);
-  const size_t smem = prefix_smem_bytes<DH>();
-  cudaError_t e = cudaFuncSetAttribute(attend_prefix_kernel<T, DH>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-  if (e != cudaSuccess) return e;
-  dim3 grid(plan.splits, plan.qgroups, unsigned(n.R * d.Hkv));
-  attend_prefix_kernel<T, DH><<<grid, kThreads, smem, st>>>(
-      lay.prefix_offset, lay.row_offset, n.R, n.N, n.total_prefix, d.Hq, d.Hkv, plan.chunk,
-      static_cast<const T*>(q), static_cast<const T*>(k_pre), static_cast<const T*>(v_pre),
-      o_part, ml_part, status);
-  e = cudaGetLastError();
+  cudaError_t e;
+  if (d.dtype == JET_DTYPE_BF16) {
+    e = launch_prefix_attend_tc(lay, d, plan, q, k_pre, v_pre, o_part, ml_part, status, st);
+  } else {
+    const size_t smem = prefix_smem_bytes<DH>();
+    e = cudaFuncSetAttribute(attend_prefix_kernel<T, DH>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    if (e != cudaSuccess) return e;
+    dim3 grid(plan.splits, plan.qgroups, unsigned(n.R * d.Hkv));
+    attend_prefix_kernel<T, DH><<<grid, kThreads, smem, st>>>(
+        lay.prefix_offset, lay.row_offset, n.R, n.N, n.total_prefix, d.Hq, d.Hkv, plan.chunk,
+        static_cast<const T*>(q), static_cast<const T*>(k_pre), static_cast<const T*>(v_pre),
+        o_part, ml_part, status);
+    e = cudaGetLastError();
+  }
   if (e != cudaSuccess) return e;
   const long long warps = (long long)n.N * d.Hq;
   attend_merge_kernel<T, DH><<<unsigned((warps + 7) / 8), 256, 0, st>>>(
@@ -233,13 +241,18 @@ AttnPlan attn_plan(const jet_sizes& n, const jet_dims& d) {
   AttnPlan p{};
   if (n.R <= 0 || n.N <= 0 || d.Hkv <= 0 || d.Hq <= 0) return p;
   const int g = d.Hq / d.Hkv;
-  p.qgroups = (n.max_rows * g + kQV - 1) / kQV;
+  const bool tc = d.dtype == JET_DTYPE_BF16;
+  const int qv = tc ? attn_tc_block() : kQV;     // query vectors per CTA
+  const int gran = tc ? 64 : kKT;                 // keys per tile
+  p.qgroups = (n.max_rows * g + qv - 1) / qv;
   const long long groups = (long long)n.R * d.Hkv * p.qgroups;
   const int max_splits = std::max(1, (n.max_prefix + 63) / 64);
-  long long want = (kTargetCtas + groups - 1) / groups;
+  // tensor-core CTAs fill an SM each: aim at two waves of them
+  const long long target = tc ? 2 * 152 : kTargetCtas;
+  long long want = (target + groups - 1) / groups;
   int splits = int(std::min<long long>(std::max<long long>(want, 1), max_splits));
   int chunk = (n.max_prefix + splits - 1) / splits;
-  chunk = (chunk + kKT - 1) / kKT * kKT;
+  chunk = (chunk + gran - 1) / gran * gran;
   p.chunk = chunk;
   p.splits = (n.max_prefix + chunk - 1) / chunk;
   const size_t vecs = size_t(p.splits) * n.N * d.Hq;

@@ -222,7 +222,7 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
       const uint32_t tph = (local >> 1) & 1;
       const int vt = u / a.n_tt;
       const int v0 = vt * kBM, t0 = (u % a.n_tt) * a.Nt;
-      const bool ok = mbar_wait(tfull + buf, tph, kWaitNs, abort_flag);
+      const bool ok = warp_mbar_wait(tfull + buf, tph, kWaitNs, abort_flag);
       if (!ok || *abort_flag) *epi_abort = 1;
       named_bar_sync(1, 128);
       if (*epi_abort) break;

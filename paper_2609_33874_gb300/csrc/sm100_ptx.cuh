@@ -67,6 +67,13 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64
   }
 }
 
+// mbar_wait by every lane of a warp, with one verdict for the whole warp
+__device__ __forceinline__ bool warp_mbar_wait(uint64_t* bar, uint32_t parity, uint64_t budget_ns,
+                                               volatile int* abort) {
+  const bool ok = mbar_wait(bar, parity, budget_ns, abort);
+  return __all_sync(0xffffffffu, ok);
+}
+
 __device__ __forceinline__ void named_bar_sync(uint32_t id, uint32_t threads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
