@@ -24,7 +24,7 @@ What each function computes, and where the paper defines it:
   head h uses key/value head floor(h / (Hq/Hkv)), no positional encoding.
 * :func:`fork_state` - every candidate continues an unmodified copy of the
   prefix recurrent state (Sec. 4.1, "Hybrid models ... restoring the unchanged
-  prefix state before each candidate"; Sec. 5.5). The recurrence itself is not
+  prefix state before each candidate"; Sec. 5.6). The recurrence itself is not
   given by the paper; the reading used is the gated delta rule
   S <- alpha (S - beta k (k^T S)) + beta k v^T, read out as o = S^T q / sqrt(dk).
 * :func:`token_logprobs` - Eq. 1 and Eq. 2: log-softmax over the full

@@ -27,7 +27,7 @@ AttnPlan attn_plan(const jet_sizes& n, const jet_dims& d);
 
 struct ScorePlan {
   int vtiles;          // ceil(V / kVocabTile)
-  size_t part_off;     // float2 partials [vtiles][N]
+  size_t part_off;     // float2 partials [N][vtiles]
   size_t ztgt_off;     // float z_tgt[T]
   size_t lse_off;      // float lse[N]
   size_t bytes;
@@ -51,7 +51,7 @@ cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, const fl
                               const float* beta, void* o, float* s_fork, int* status,
                               cudaStream_t st);
 
-// logits partials: writes part[vtiles][N] (m, s) in base 2 - m = max_v z log2(e),
+// logits partials: writes part[N][vtiles] (m, s) in base 2 - m = max_v z log2(e),
 // s = sum_v 2^(z log2(e) - m) over the tile - and z_tgt[T]
 cudaError_t launch_lmhead_simt(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
                                const void* hidden, const void* w_lm, void* ws, int* status,

@@ -79,7 +79,7 @@ lmhead_simt_kernel(const int32_t* __restrict__ target_ids, const int32_t* __rest
       if (v0 + lane + 32 * b < V) s += exp2f(acc[a][b] * kLog2e - mx);
     s = warp_sum(s);
     if (n < N) {
-      if (lane == 0) part[size_t(vt) * N + n] = make_float2(mx, s);
+      if (lane == 0) part[size_t(n) * gridDim.y + vt] = make_float2(mx, s);
       const int t0 = row_tgt_offset[n], t1 = row_tgt_offset[n + 1];
       for (int t = t0; t < t1; ++t) {
         const int j = row_tgt_index[t];

@@ -56,7 +56,7 @@ struct TcArgs {
   float* z_tgt;
   int* status;
   int N, T, V, D;
-  int Nt, n_tt, units, nkb, stages;
+  int Nt, n_tt, units, nkb, stages, vtiles;
   uint32_t tmem_cols;
 };
 
@@ -298,7 +298,7 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
         float M = red[c].x, S = red[c].y;
 #pragma unroll
         for (int w = 1; w < 4; ++w) combine(M, S, red[w * kMaxNt + c].x, red[w * kMaxNt + c].y);
-        a.part[size_t(vt) * a.N + t0 + c] = make_float2(M, S);
+        a.part[size_t(t0 + c) * a.vtiles + vt] = make_float2(M, S);
       }
       named_bar_sync(1, 128);
     }
@@ -373,6 +373,7 @@ cudaError_t launch_lmhead_tc(const jet_layout& lay, const jet_dims& d, const Sco
   a.Nt = Nt;
   a.n_tt = n_tt;
   a.units = plan.vtiles * n_tt;
+  a.vtiles = plan.vtiles;
   a.nkb = (d.D + kBK - 1) / kBK;
   a.tmem_cols = Nt <= 128 ? 256 : 512;
   const int stage_bytes = kBM * 128 + Nt * 128;

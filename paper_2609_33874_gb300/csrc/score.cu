@@ -13,22 +13,28 @@
 namespace jet {
 namespace {
 
-// block (32 rows) x 8 tile slices; coalesced reads of part[vt][n]
-__global__ void __launch_bounds__(256)
+// one block per row; coalesced reads of the row's partials part[n][0..vtiles)
+__global__ void __launch_bounds__(128)
 lse_kernel(const float2* __restrict__ part, int vtiles, int N, float* __restrict__ lse) {
-  __shared__ float2 red[8][33];
-  const int x = threadIdx.x & 31, y = threadIdx.x >> 5;
-  const int n = blockIdx.x * 32 + x;
+  __shared__ float2 red[4];
+  const int n = blockIdx.x;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const float2* p = part + size_t(n) * vtiles;
   float m = -INFINITY, s = 0.f;
-  if (n < N)
-    for (int vt = y; vt < vtiles; vt += 8) {
-      const float2 p = part[size_t(vt) * N + n];
-      ms_combine2(m, s, p.x, p.y);
-    }
-  red[y][x] = make_float2(m, s);
+  for (int vt = threadIdx.x; vt < vtiles; vt += 128) {
+    const float2 x = p[vt];
+    ms_combine2(m, s, x.x, x.y);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+    const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
+    ms_combine2(m, s, m2, s2);
+  }
+  if (lane == 0) red[warp] = make_float2(m, s);
   __syncthreads();
-  if (y == 0 && n < N) {
-    for (int i = 1; i < 8; ++i) ms_combine2(m, s, red[i][x].x, red[i][x].y);
+  if (threadIdx.x == 0) {
+    for (int i = 1; i < 4; ++i) ms_combine2(m, s, red[i].x, red[i].y);
     lse[n] = (m + log2f(s)) * 0.6931471805599453f;  // partials are base 2
   }
 }
@@ -135,7 +141,7 @@ cudaError_t launch_score_finish(const jet_layout& lay, const ScorePlan& plan, vo
   const float2* part = reinterpret_cast<const float2*>(base + plan.part_off);
   const float* z_tgt = reinterpret_cast<const float*>(base + plan.ztgt_off);
   float* lse = reinterpret_cast<float*>(base + plan.lse_off);
-  lse_kernel<<<unsigned((n.N + 31) / 32), 256, 0, st>>>(part, plan.vtiles, n.N, lse);
+  lse_kernel<<<unsigned(n.N), 128, 0, st>>>(part, plan.vtiles, n.N, lse);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   finish_kernel<<<unsigned((n.C + 127) / 128), 128, 0, st>>>(lay.tgt_offset, lay.tgt_row, n.C, n.N,

@@ -360,7 +360,7 @@ def test_toy_scores_equal_independent_recomputation():
 
 
 # ---------------------------------------------------------------------------
-# recurrent-state fork (Sec. 4.1, Sec. 5.5)
+# recurrent-state fork (Sec. 4.1, Sec. 5.6)
 # ---------------------------------------------------------------------------
 def _unit(v):
     return v / np.linalg.norm(v)
