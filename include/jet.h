@@ -235,6 +235,32 @@ jet_status jet_score_candidates(const jet_layout* lay, const jet_dims* dims, con
                                 void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * jet_score_candidates_noalloc - jet_score_candidates without caller-owned
+ * scratch memory. The paper has no counterpart to this entry point: it exists
+ * for callers that cannot call cudaMalloc, such as a host application that
+ * owns every device allocation and passes its plug-ins only the tensors they
+ * work on, or a serving loop that must not allocate (cudaMalloc can
+ * synchronise the device and can fail under memory pressure) once it runs.
+ * Arguments and results are those of jet_score_candidates minus ws/ws_bytes.
+ * - Scratch is a fixed 16 MiB array inside the library (a __device__ array that
+ *   every GPU loading the library holds until the process exits). A batch
+ *   needs N * ceil(V / 128) * 8 + T * 4 + N * 4 bytes (each term rounded up to
+ *   256); larger batches get JET_ERR_CAPACITY and nothing is launched. With
+ *   V = 151,936 that allows about 1,700 rows.
+ * - The call allocates nothing and calls no allocating library routine.
+ * - The first call on each device looks up the array's device address
+ *   (cudaGetSymbolAddress, with that device current); make that first call
+ *   before any stream capture on the device.
+ * - Every call shares the one array: calls whose work overlaps on the GPU
+ *   (other streams, other threads) race on it and must be ordered by the
+ *   caller. No part of the array needs clearing between calls: each element a
+ *   call reads is written earlier by the same call.
+ */
+jet_status jet_score_candidates_noalloc(const jet_layout* lay, const jet_dims* dims,
+                                        const void* hidden, const void* w_lm,
+                                        float* tok_logprob, float* cand_score, void* stream);
+
+/*
  * jet_decide - decision rules (Eq. 4, Eq. 5, Sec. 3.3).
  *   cand_score [C] float32   s(c|x)
  *   q          [C] float32   q(c) = exp(s_c - M) / sum_d exp(s_d - M), M = max s

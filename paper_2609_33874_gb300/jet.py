@@ -80,6 +80,8 @@ def _load() -> ctypes.CDLL:
                                P, P, P, P, P, P, P, P, P]),
         "jet_score_candidates": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
                                      P, P, P, P, P, SZ, P]),
+        "jet_score_candidates_noalloc": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
+                                             P, P, P, P, P]),
         "jet_decide": (I, [ctypes.POINTER(jet_layout), I, P, P, P, P, P]),
         "jet_device_status": (I, [P, ctypes.POINTER(ctypes.c_int32)]),
     }
@@ -93,7 +95,8 @@ def _load() -> ctypes.CDLL:
 _lib = _load()
 DECLARED = ("jet_abi_version", "jet_status_string", "jet_layout_plan", "jet_layout_words",
             "jet_layout_build", "jet_layout_bind", "jet_workspace_bytes", "jet_prefix_attend",
-            "jet_fork_state", "jet_score_candidates", "jet_decide", "jet_device_status")
+            "jet_fork_state", "jet_score_candidates", "jet_score_candidates_noalloc", "jet_decide",
+            "jet_device_status")
 
 
 def library() -> ctypes.CDLL:
@@ -231,6 +234,16 @@ def jet_score_candidates(layout, dims: jet_dims, hidden, w_lm, tok_logprob, cand
                                      _addr(hidden), _addr(w_lm), _addr(tok_logprob),
                                      _addr(cand_score), _addr(ws), int(ws_bytes),
                                      _stream(stream)), "jet_score_candidates")
+
+
+def jet_score_candidates_noalloc(layout, dims: jet_dims, hidden, w_lm, tok_logprob, cand_score,
+                                 stream=None) -> None:
+    """jet_score_candidates with the library's own fixed scratch array, for
+    callers that cannot allocate device memory (see include/jet.h)."""
+    _check(_lib.jet_score_candidates_noalloc(ctypes.byref(_lay(layout)), ctypes.byref(dims),
+                                             _addr(hidden), _addr(w_lm), _addr(tok_logprob),
+                                             _addr(cand_score), _stream(stream)),
+           "jet_score_candidates_noalloc")
 
 
 def jet_decide(layout, mode: int, cand_score, q, choice, value, stream=None) -> None:
