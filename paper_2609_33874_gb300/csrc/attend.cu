@@ -245,14 +245,18 @@ AttnPlan attn_plan(const jet_sizes& n, const jet_dims& d) {
   const int qv = tc ? attn_tc_block() : kQV;     // query vectors per CTA
   const int gran = tc ? 64 : kKT;                 // keys per tile
   p.qgroups = (n.max_rows * g + qv - 1) / qv;
-  const long long groups = (long long)n.R * d.Hkv * p.qgroups;
+  // query blocks of an average request: blocks past a request's vectors exit
+  // at once, so they do not count as work
+  const long long avg_vecs = ((long long)n.N * g + n.R - 1) / n.R;
+  const long long groups = (long long)n.R * d.Hkv * std::max<long long>(1, (avg_vecs + qv - 1) / qv);
   const int max_splits = std::max(1, (n.max_prefix + 63) / 64);
-  // tensor-core CTAs fill an SM each: aim at two waves of them
-  const long long target = tc ? 2 * 152 : kTargetCtas;
-  long long want = (target + groups - 1) / groups;
+  // about four CTAs per SM (152 SMs); tensor-core chunks keep at least 256
+  // keys so the per-chunk partials stay small next to the chunk's K/V bytes
+  long long want = (kTargetCtas + groups - 1) / groups;
   int splits = int(std::min<long long>(std::max<long long>(want, 1), max_splits));
   int chunk = (n.max_prefix + splits - 1) / splits;
   chunk = (chunk + gran - 1) / gran * gran;
+  if (tc) chunk = std::max(chunk, 256);
   p.chunk = chunk;
   p.splits = (n.max_prefix + chunk - 1) / chunk;
   const size_t vecs = size_t(p.splits) * n.N * d.Hq;

@@ -41,6 +41,7 @@ constexpr int kThreads = 192;
 constexpr uint64_t kWaitNs = 2000000000ull;
 constexpr uint64_t kDrainNs = 200000000ull;
 constexpr float kRescaleLog2 = 8.f;  // rescale O only when the max grows by > 2^8
+constexpr int kPrefetch = 4;         // key tiles prefetched into L2 ahead of the TMA loads
 
 template <int DH>
 struct Geo {
@@ -129,6 +130,15 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, u
       : "memory");
 }
 
+// 3-D TMA prefetch of the same box into L2 only
+__device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap* map, int32_t x, int32_t y,
+                                                int32_t z) {
+  asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(z)
+               : "memory");
+}
+
 template <int DH>
 __global__ void __launch_bounds__(kThreads, 1)
 attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
@@ -137,9 +147,13 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  uint64_t* kv_full = reinterpret_cast<uint64_t*>(smem + G::kOffBar);
-  uint64_t* kv_empty = kv_full + kStages;
-  uint64_t* s_full = kv_empty + kStages;   // [2]
+  // K and V of a stage fill and drain separately: K is free once S_j has been
+  // computed, V only after P_j V_j
+  uint64_t* k_full = reinterpret_cast<uint64_t*>(smem + G::kOffBar);
+  uint64_t* k_empty = k_full + kStages;
+  uint64_t* v_full = k_empty + kStages;
+  uint64_t* v_empty = v_full + kStages;
+  uint64_t* s_full = v_empty + kStages;    // [2]
   uint64_t* s_free = s_full + 2;           // [2]
   uint64_t* p_full = s_free + 2;           // [2]
   uint64_t* p_free = p_full + 2;           // [2]
@@ -148,8 +162,10 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
-  const int split = blockIdx.x, qb = blockIdx.y;
-  const int r = blockIdx.z / a.Hkv, kh = blockIdx.z % a.Hkv;
+  // query blocks are the slowest grid dimension: blocks past a request's
+  // vectors (only long requests have them) come last and exit at once
+  const int split = blockIdx.x, qb = blockIdx.z;
+  const int r = blockIdx.y / a.Hkv, kh = blockIdx.y % a.Hkv;
   const int g = a.Hq / a.Hkv;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (r >= a.R) return;
@@ -178,8 +194,10 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(kv_full + s, 1);
-      mbar_init(kv_empty + s, 1);
+      mbar_init(k_full + s, 1);
+      mbar_init(k_empty + s, 1);
+      mbar_init(v_full + s, 1);
+      mbar_init(v_empty + s, 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(s_full + b, 1);
@@ -208,33 +226,73 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
   if (warp == 0) {
     // ---------------------------------------------------------------- producer
     if (lane == 0) {
+      // K_j and V_j are issued as soon as their slots drain, whichever first
       const uint64_t pol = policy_evict_first();
-      uint32_t issued = 0, issued_par = 0;
+      uint32_t k_issued = 0, k_par = 0, v_issued = 0, v_par = 0;
+      int jk = 0, jv = 0;
       bool ok = true;
-      for (int j = 0; j < ntiles; ++j) {
-        const int s = j % kStages;
-        const uint32_t ph = (j / kStages) & 1;
-        if (!mbar_wait(kv_empty + s, ph ^ 1u, kWaitNs, abort_flag)) {
+      uint64_t t_last = global_timer_ns();
+      while (jv < ntiles) {
+        bool progressed = false;
+        if (jk < ntiles) {
+          const int s = jk % kStages;
+          const uint32_t ph = (jk / kStages) & 1;
+          if (mbar_test(k_empty + s, ph ^ 1u)) {
+            uint8_t* ks = smem + G::kOffK + s * 2 * G::kKVBytes;
+            mbar_arrive_expect_tx(k_full + s, G::kKVBytes);
+            const int key = p0 + k_begin + jk * kBN;
+#pragma unroll
+            for (int sl = 0; sl < G::kSlices; ++sl)
+              tma_load_3d(ks + sl * (kBN * 128), &tmK, k_full + s, sl * 64, kh, key, pol);
+            // keep kPrefetch further tiles on their way into L2: two shared
+            // stages alone hold too few bytes in flight to cover HBM latency
+            for (int jp = (jk == 0 ? 1 : jk + kPrefetch); jp <= jk + kPrefetch && jp < ntiles;
+                 ++jp) {
+              const int kp = p0 + k_begin + jp * kBN;
+#pragma unroll
+              for (int sl = 0; sl < G::kSlices; ++sl) {
+                tma_prefetch_3d(&tmK, sl * 64, kh, kp);
+                tma_prefetch_3d(&tmV, sl * 64, kh, kp);
+              }
+            }
+            k_issued |= 1u << s;
+            k_par = (k_par & ~(1u << s)) | (ph << s);
+            ++jk;
+            progressed = true;
+          }
+        }
+        if (jv < jk) {
+          const int s = jv % kStages;
+          const uint32_t ph = (jv / kStages) & 1;
+          if (mbar_test(v_empty + s, ph ^ 1u)) {
+            uint8_t* vs = smem + G::kOffK + s * 2 * G::kKVBytes + G::kKVBytes;
+            mbar_arrive_expect_tx(v_full + s, G::kKVBytes);
+            const int key = p0 + k_begin + jv * kBN;
+#pragma unroll
+            for (int sl = 0; sl < G::kSlices; ++sl)
+              tma_load_3d(vs + sl * (kBN * 128), &tmV, v_full + s, sl * 64, kh, key, pol);
+            v_issued |= 1u << s;
+            v_par = (v_par & ~(1u << s)) | (ph << s);
+            ++jv;
+            progressed = true;
+          }
+        }
+        const uint64_t now = global_timer_ns();
+        if (progressed) {
+          t_last = now;
+        } else if (*abort_flag || now - t_last > kWaitNs) {
           ok = false;
           break;
         }
-        uint8_t* ks = smem + G::kOffK + s * 2 * G::kKVBytes;
-        uint8_t* vs = ks + G::kKVBytes;
-        mbar_arrive_expect_tx(kv_full + s, 2 * G::kKVBytes);
-        const int key = p0 + k_begin + j * kBN;
-#pragma unroll
-        for (int sl = 0; sl < G::kSlices; ++sl) {
-          tma_load_3d(ks + sl * (kBN * 128), &tmK, kv_full + s, sl * 64, kh, key, pol);
-          tma_load_3d(vs + sl * (kBN * 128), &tmV, kv_full + s, sl * 64, kh, key, pol);
-        }
-        issued |= 1u << s;
-        issued_par = (issued_par & ~(1u << s)) | (ph << s);
       }
       if (!ok) {
         *abort_flag = 1;
         flag(a.status, JET_ERR_TIMEOUT);
-        for (int t = 0; t < kStages; ++t)
-          if (issued & (1u << t)) mbar_wait(kv_full + t, (issued_par >> t) & 1u, kDrainNs, nullptr);
+        // let every copy already issued land before the CTA can exit
+        for (int t = 0; t < kStages; ++t) {
+          if (k_issued & (1u << t)) mbar_wait(k_full + t, (k_par >> t) & 1u, kDrainNs, nullptr);
+          if (v_issued & (1u << t)) mbar_wait(v_full + t, (v_par >> t) & 1u, kDrainNs, nullptr);
+        }
       }
     }
   } else if (warp == 1) {
@@ -245,42 +303,51 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
       const uint32_t qs = smem_u32(smem);
       bool ok = mbar_wait(q_full, 0, kWaitNs, abort_flag);
       tc_fence_after();
-      for (int j = 0; ok && j <= ntiles; ++j) {
-        if (j < ntiles) {  // S_j = Q K_j^T
-          const int s = j % kStages;
-          const int b = j & 1;
-          if (!mbar_wait(kv_full + s, (j / kStages) & 1, kWaitNs, abort_flag) ||
-              !mbar_wait(s_free + b, ((j >> 1) & 1) ^ 1u, kWaitNs, abort_flag)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t ks = smem_u32(smem + G::kOffK + s * 2 * G::kKVBytes);
+      // issue S_j = Q K_j^T and O += P_j V_j in whichever order their inputs
+      // become ready; S_j always precedes P_j V_j
+      int js = 0, jo = 0;
+      uint64_t t_last = global_timer_ns();
+      while (ok && jo < ntiles) {
+        bool progressed = false;
+        if (js < ntiles) {
+          const int s = js % kStages, b = js & 1;
+          if (mbar_test(k_full + s, (js / kStages) & 1) &&
+              mbar_test(s_free + b, ((js >> 1) & 1) ^ 1u)) {
+            tc_fence_after();
+            const uint32_t ks = smem_u32(smem + G::kOffK + s * 2 * G::kKVBytes);
 #pragma unroll
-          for (int st = 0; st < DH / 16; ++st) {
-            const int sl = st >> 2, k = st & 3;
-            mma_f16(tmem + b * kBN, desc_k_sw128(qs + sl * (kBV * 128) + 32 * k),
-                    desc_k_sw128(ks + sl * (kBN * 128) + 32 * k), id_s, st != 0);
+            for (int st = 0; st < DH / 16; ++st) {
+              const int sl = st >> 2, k = st & 3;
+              mma_f16(tmem + b * kBN, desc_k_sw128(qs + sl * (kBV * 128) + 32 * k),
+                      desc_k_sw128(ks + sl * (kBN * 128) + 32 * k), id_s, st != 0);
+            }
+            mma_commit(s_full + b);
+            mma_commit(k_empty + s);
+            ++js;
+            progressed = true;
           }
-          mma_commit(s_full + b);
         }
-        if (j >= 1) {  // O += P_{j-1} V_{j-1}
-          const int jp = j - 1;
-          const int s = jp % kStages;
-          const int b = jp & 1;
-          if (!mbar_wait(p_full + b, (jp >> 1) & 1, kWaitNs, abort_flag)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t ps = smem_u32(smem + G::kOffP + b * G::kPBytes);
-          const uint32_t vs = smem_u32(smem + G::kOffK + s * 2 * G::kKVBytes + G::kKVBytes);
+        if (jo < js) {
+          const int s = jo % kStages, b = jo & 1;
+          if (mbar_test(p_full + b, (jo >> 1) & 1) && mbar_test(v_full + s, (jo / kStages) & 1)) {
+            tc_fence_after();
+            const uint32_t ps = smem_u32(smem + G::kOffP + b * G::kPBytes);
+            const uint32_t vs = smem_u32(smem + G::kOffK + s * 2 * G::kKVBytes + G::kKVBytes);
 #pragma unroll
-          for (int k = 0; k < kBN / 16; ++k)
-            mma_f16(tmem + G::kOCol, desc_k_sw128(ps + 32 * k),
-                    desc_mn_sw128(vs + k * 16 * 128, kBN * 128), id_o, (jp | k) != 0);
-          mma_commit(p_free + b);
-          mma_commit(kv_empty + s);
+            for (int k = 0; k < kBN / 16; ++k)
+              mma_f16(tmem + G::kOCol, desc_k_sw128(ps + 32 * k),
+                      desc_mn_sw128(vs + k * 16 * 128, kBN * 128), id_o, (jo | k) != 0);
+            mma_commit(p_free + b);
+            mma_commit(v_empty + s);
+            ++jo;
+            progressed = true;
+          }
+        }
+        const uint64_t now = global_timer_ns();
+        if (progressed) {
+          t_last = now;
+        } else if (*abort_flag || now - t_last > kWaitNs) {
+          ok = false;
         }
       }
       if (!ok) {
@@ -487,7 +554,7 @@ cudaError_t launch_dh(const jet_layout& lay, const jet_dims& d, const AttnPlan& 
   cudaError_t e = cudaFuncSetAttribute(attend_prefix_tc_kernel<DH>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
   if (e != cudaSuccess) return e;
-  dim3 grid(plan.splits, plan.qgroups, unsigned(n.R * d.Hkv));
+  dim3 grid(plan.splits, unsigned(n.R * d.Hkv), plan.qgroups);
   attend_prefix_tc_kernel<DH><<<grid, kThreads, smem, st>>>(tmK, tmV, a);
   return cudaGetLastError();
 }
