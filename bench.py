@@ -192,6 +192,33 @@ def _traffic(kernel_file: str, workload: str):
     return rec.get("bytes_per_launch")
 
 
+def _call(ms: float, nbytes: int, peaks) -> dict:
+    """An HBM-bound call: its time, algorithmic bytes and fraction of the copy peak."""
+    gbs = nbytes / (ms / 1e3) / 1e9
+    return dict(ms=round(ms, 4), bound="hbm", algorithmic_bytes=int(nbytes),
+                achieved_gbs=round(gbs, 1), frac=round(gbs / peaks["hbm"], 4))
+
+
+def _attend_launches(problem, w) -> int:
+    """Kernels jet_prefix_attend launches for this batch: the float32 path is
+    prefix + merge; the bf16 path is the tensor-core kernel plus a chunk
+    combine when any prefix spans more than one chunk (the library's plan:
+    about 608 CTAs, chunks of at least 256 keys)."""
+    if w.dtype != "bf16":
+        return 2
+    g = w.Hq // w.Hkv
+    R, N = problem.R, problem.N
+    max_prefix = int(problem.prefix_len.max())
+    avg_vecs = (N * g + R - 1) // R
+    qv = max(1, 128 // g) * g  # whole rows of g heads per query block
+    groups = R * w.Hkv * max(1, (avg_vecs + qv - 1) // qv)
+    splits = min(max(1, (608 + groups - 1) // groups), max(1, (max_prefix + 63) // 64))
+    chunk = (max_prefix + splits - 1) // splits
+    chunk = max(256, (chunk + 63) // 64 * 64)
+    splits = (max_prefix + chunk - 1) // chunk
+    return 1 + (1 if splits > 1 else 0)
+
+
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -236,9 +263,9 @@ def run_gpu(args):
     stream = torch.cuda.Stream(dev)
 
     # --- device-resident timed region -------------------------------------
+    # events between the calls of every timed step: attend | fork | score | decide
     n_ev = args.steps
-    score_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                for _ in range(n_ev)]
+    call_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(n_ev)]
     uuid = None
     try:
         uuid = str(torch.cuda.get_device_properties(dev).uuid)
@@ -249,19 +276,26 @@ def run_gpu(args):
 
     def one_step(i=None):
         d, lay = step.dims, step.layout
+        ev = call_ev[i] if i is not None else None
+        if ev:
+            ev[0].record(stream)
         jet.jet_prefix_attend(lay, d, x["q"], x["k_pre"], x["v_pre"], x["k_cand"], x["v_cand"],
                               step.o, step.ws, stream=stream)
+        if ev:
+            ev[1].record(stream)
         if step.hybrid:
             jet.jet_fork_state(lay, d, x["s_prefix"], x["lq"], x["lk"], x["lv"], x["alpha"],
                                x["beta"], step.lo, step.s_fork, stream=stream)
-        if i is not None:
-            score_ev[i][0].record(stream)
+        if ev:
+            ev[2].record(stream)
         jet.jet_score_candidates(lay, d, x["hidden"], w_lm, step.tok_logprob, step.cand_score,
                                  step.ws, stream=stream)
-        if i is not None:
-            score_ev[i][1].record(stream)
+        if ev:
+            ev[3].record(stream)
         jet.jet_decide(lay, step.mode, step.cand_score, step.q_cand, step.choice, step.value,
                        stream=stream)
+        if ev:
+            ev[4].record(stream)
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
@@ -284,7 +318,8 @@ def run_gpu(args):
         torch.distributed.barrier()
     total_ms = t_start.elapsed_time(t_end)
     clk = clocks.stop()
-    score_ms = [a.elapsed_time(b) for a, b in score_ev]
+    call_ms = {name: statistics.mean(ev[k].elapsed_time(ev[k + 1]) for ev in call_ev)
+               for k, name in enumerate(("attend", "fork", "score", "decide"))}
 
     # --- end to end: pinned host inputs, copies inside the timed region ---------
     host = {k: x[k].cpu().pin_memory() for k in names}
@@ -323,7 +358,7 @@ def run_gpu(args):
     vtiles = (w.V + 127) // 128
     lm_bytes = w.V * w.D * es + N * w.D * es + vtiles * N * 8 + T * 4
     lm_flops = 2.0 * N * w.D * w.V
-    score_avg_s = statistics.mean(score_ms) / 1e3
+    score_avg_s = call_ms["score"] / 1e3
     ridge = peaks["bf16"] * 1e12 / (peaks["hbm"] * 1e9)
     kernel_file = "paper_2609_33874_gb300/csrc/lmhead_tc.cu" if w.dtype == "bf16" and \
         os.path.exists(os.path.join(ROOT, "paper_2609_33874_gb300/csrc/lmhead_tc.cu")) \
@@ -344,7 +379,20 @@ def run_gpu(args):
                 algorithmic_bytes=lm_bytes, algorithmic_flops=lm_flops,
                 avg_launch_ms=round(score_avg_s * 1e3, 4), peak_source=peaks["source"])
 
-    launches_per_step = 2 + (1 if w.Hl else 0) + 3 + 1
+    # every call of the step against its own roofline (algorithmic bytes only)
+    F = N - R
+    attn_bytes = (2 * problem.total_prefix * w.Hkv * w.d * es + 2 * F * w.Hkv * w.d * es
+                  + 2 * N * w.Hq * w.d * es)
+    calls = dict(attend=_call(call_ms["attend"], attn_bytes, peaks),
+                 score=dict(ms=round(call_ms["score"], 4), bound=roof["bound"],
+                            frac=roof["frac"]),
+                 decide=dict(ms=round(call_ms["decide"], 4)))
+    if w.Hl:
+        fork_bytes = (R * w.Hl * w.dk * w.dv * 4 + len(problem.cand_len) * w.Hl * w.dk * w.dv * 4
+                      + F * w.Hl * (2 * w.dk + 2 * w.dv) * es + F * w.Hl * 8)
+        calls["fork"] = _call(call_ms["fork"], fork_bytes, peaks)
+
+    launches_per_step = _attend_launches(problem, w) + (1 if w.Hl else 0) + 3 + 1
     result = dict(
         metric=METRIC, value=round(value, 2), unit=UNIT, n_gpus=world, steps=args.steps,
         warmup=args.warmup, ms_per_step=round(ms_per_step, 4), higher_is_better=True,
@@ -360,6 +408,7 @@ def run_gpu(args):
                  d2h_bytes_per_step=d2h, ms_per_step=round(e2e_ms, 4)),
         gpu_launches=launches_per_step * args.steps,
         roofline=roof,
+        calls=calls,
     )
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(args.workload, R, args.cpu_sample)

@@ -213,7 +213,9 @@ cudaError_t launch_typed(const jet_layout& lay, const jet_dims& d, const AttnPla
   float2* ml_part = reinterpret_cast<float2*>(o_part + size_t(plan.splits) * n.N * d.Hq * DH);
   cudaError_t e;
   if (d.dtype == JET_DTYPE_BF16) {
-    e = launch_prefix_attend_tc(lay, d, plan, q, k_pre, v_pre, o_part, ml_part, status, st);
+    // the tensor-core path covers the candidates' own keys and the combine
+    return launch_attend_tc(lay, d, plan, q, k_pre, v_pre, k_cand, v_cand, o, o_part, ml_part,
+                            status, st);
   } else {
     const size_t smem = prefix_smem_bytes<DH>();
     e = cudaFuncSetAttribute(attend_prefix_kernel<T, DH>,
@@ -242,8 +244,10 @@ AttnPlan attn_plan(const jet_sizes& n, const jet_dims& d) {
   if (n.R <= 0 || n.N <= 0 || d.Hkv <= 0 || d.Hq <= 0) return p;
   const int g = d.Hq / d.Hkv;
   const bool tc = d.dtype == JET_DTYPE_BF16;
-  const int qv = tc ? attn_tc_block() : kQV;     // query vectors per CTA
   const int gran = tc ? 64 : kKT;                 // keys per tile
+  // query vectors per CTA: the tensor-core kernel takes whole rows (128 / g
+  // rows of g heads), the float32 kernel kQV vectors
+  const int qv = tc ? std::max(1, attn_tc_block() / g) * g : kQV;
   p.qgroups = (n.max_rows * g + qv - 1) / qv;
   // query blocks of an average request: blocks past a request's vectors exit
   // at once, so they do not count as work

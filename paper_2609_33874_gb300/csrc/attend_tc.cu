@@ -60,11 +60,15 @@ struct Geo {
 struct AttArgs {
   const int32_t* prefix_offset;
   const int32_t* row_offset;
+  const int32_t* row_cand;
+  const int32_t* cand_row_offset;
   const __nv_bfloat16* q;
+  __nv_bfloat16* o;  // final output, written directly by single-chunk requests
   float* o_part;
   float2* ml_part;
   int* status;
-  int R, N, total_prefix, Hq, Hkv, chunk;
+  int R, N, C, total_prefix, Hq, Hkv, chunk;
+  int has_cand;      // the batch has fed candidate tokens (F > 0)
   float scale_log2;  // log2(e) / sqrt(d)
 };
 
@@ -141,8 +145,11 @@ __device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap* map, int32_t 
 
 template <int DH>
 __global__ void __launch_bounds__(kThreads, 1)
-attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
-                        const __grid_constant__ CUtensorMap tmV, const AttArgs a) {
+attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
+                        const __grid_constant__ CUtensorMap tmK,
+                        const __grid_constant__ CUtensorMap tmV,
+                        const __grid_constant__ CUtensorMap tmKc,
+                        const __grid_constant__ CUtensorMap tmVc, const AttArgs a) {
   using G = Geo<DH>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -175,15 +182,26 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
     if (threadIdx.x == 0) flag(a.status, JET_ERR_DEVICE);
     return;
   }
-  const int nvec = nr * g;
-  const int vbase = qb * kBV;
-  if (vbase >= nvec) return;
-  const int nv = min(kBV, nvec - vbase);
+  // a query block holds whole rows: rb rows x g heads (<= 128 vectors)
+  const int rb = kBV / g;
+  const int row0 = qb * rb;  // first row of the block within the request
+  if (row0 >= nr) return;
+  const int vbase = row0 * g;
+  const int nv = min(rb, nr - row0) * g;
   const int k_begin = split * a.chunk;
   const int k_end = min(P, k_begin + a.chunk);
-  const int ntiles = k_end > k_begin ? (k_end - k_begin + kBN - 1) / kBN : 0;
+  const int npt = k_end > k_begin ? (k_end - k_begin + kBN - 1) / kBN : 0;  // prefix tiles
+  // the request's last chunk also takes its candidates' own keys: the F_r fed
+  // tokens, as extra 64-key tiles masked per row to the row's candidate and
+  // position (Sec. 4.1: a candidate attends to its own earlier tokens only)
+  const int splits_r = (P + a.chunk - 1) / a.chunk;
+  const bool last = npt > 0 && split == splits_r - 1;
+  const int f_begin = n0 - r;     // fed-token index of the request's first fed row
+  const int F_r = nr - 1;
+  const int nct = (last && a.has_cand && F_r > 0) ? (F_r + kBN - 1) / kBN : 0;
+  const int ntiles = npt + nct;
 
-  if (ntiles == 0) {  // an empty chunk: an empty partial
+  if (npt == 0) {  // an empty chunk: an empty partial
     for (int i = threadIdx.x; i < nv; i += blockDim.x) {
       const int gv = vbase + i;
       const size_t base = (size_t(split) * a.N + n0 + gv / g) * a.Hq + kh * g + gv % g;
@@ -205,7 +223,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
       mbar_init(p_full + b, 4);
       mbar_init(p_free + b, 1);
     }
-    mbar_init(q_full, 4);
+    mbar_init(q_full, 5);  // the query TMA (with its bytes) + 4 softmax warps
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -215,8 +233,13 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
     tmem_relinquish();
   }
   if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmQ);
     tma_prefetch_desc(&tmK);
     tma_prefetch_desc(&tmV);
+    if (nct > 0) {
+      tma_prefetch_desc(&tmKc);
+      tma_prefetch_desc(&tmVc);
+    }
   }
   tc_fence_before();
   __syncthreads();
@@ -226,6 +249,12 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
   if (warp == 0) {
     // ---------------------------------------------------------------- producer
     if (lane == 0) {
+      // the query block: rb rows x g heads x d of the request's group kh
+      mbar_arrive_expect_tx(q_full, uint32_t(G::kSlices) * 64 * 2 * g * rb);
+#pragma unroll
+      for (int sl = 0; sl < G::kSlices; ++sl)
+        tma_load_3d(smem + sl * (kBV * 128), &tmQ, q_full, sl * 64, kh * g, n0 + row0,
+                    policy_evict_first());
       // K_j and V_j are issued as soon as their slots drain, whichever first
       const uint64_t pol = policy_evict_first();
       uint32_t k_issued = 0, k_par = 0, v_issued = 0, v_par = 0;
@@ -240,13 +269,15 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
           if (mbar_test(k_empty + s, ph ^ 1u)) {
             uint8_t* ks = smem + G::kOffK + s * 2 * G::kKVBytes;
             mbar_arrive_expect_tx(k_full + s, G::kKVBytes);
-            const int key = p0 + k_begin + jk * kBN;
+            const bool pre = jk < npt;
+            const CUtensorMap* mk = pre ? &tmK : &tmKc;
+            const int key = pre ? p0 + k_begin + jk * kBN : f_begin + (jk - npt) * kBN;
 #pragma unroll
             for (int sl = 0; sl < G::kSlices; ++sl)
-              tma_load_3d(ks + sl * (kBN * 128), &tmK, k_full + s, sl * 64, kh, key, pol);
+              tma_load_3d(ks + sl * (kBN * 128), mk, k_full + s, sl * 64, kh, key, pol);
             // keep kPrefetch further tiles on their way into L2: two shared
             // stages alone hold too few bytes in flight to cover HBM latency
-            for (int jp = (jk == 0 ? 1 : jk + kPrefetch); jp <= jk + kPrefetch && jp < ntiles;
+            for (int jp = (jk == 0 ? 1 : jk + kPrefetch); jp <= jk + kPrefetch && jp < npt;
                  ++jp) {
               const int kp = p0 + k_begin + jp * kBN;
 #pragma unroll
@@ -267,10 +298,12 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
           if (mbar_test(v_empty + s, ph ^ 1u)) {
             uint8_t* vs = smem + G::kOffK + s * 2 * G::kKVBytes + G::kKVBytes;
             mbar_arrive_expect_tx(v_full + s, G::kKVBytes);
-            const int key = p0 + k_begin + jv * kBN;
+            const bool pre = jv < npt;
+            const CUtensorMap* mv = pre ? &tmV : &tmVc;
+            const int key = pre ? p0 + k_begin + jv * kBN : f_begin + (jv - npt) * kBN;
 #pragma unroll
             for (int sl = 0; sl < G::kSlices; ++sl)
-              tma_load_3d(vs + sl * (kBN * 128), &tmV, v_full + s, sl * 64, kh, key, pol);
+              tma_load_3d(vs + sl * (kBN * 128), mv, v_full + s, sl * 64, kh, key, pol);
             v_issued |= 1u << s;
             v_par = (v_par & ~(1u << s)) | (ph << s);
             ++jv;
@@ -364,19 +397,25 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
     const uint32_t lane_off = uint32_t(q4 * 32) << 16;
     const bool valid = i < nv;
     int n = 0, h = 0;
+    int fa = 1, fb = 0;  // fed-token indices this vector may see (none: shared row)
     if (valid) {
       const int gv = vbase + i;
       n = n0 + gv / g;
       h = kh * g + gv % g;
+      const int c = a.row_cand[n];
+      if (c >= 0 && c < a.C) {
+        fa = a.cand_row_offset[c] - r - 1;  // y_{c,1}
+        fb = n - r - 1;                     // the row's own fed token, inclusive
+      }
     }
-    // query block -> shared memory, 128-byte swizzled, zero rows past nv
+    // the query block arrives by TMA (rows [0, rb g)); zero the rows past it
+    // so that no stale shared memory enters the MMA
     {
-      const uint4* src = reinterpret_cast<const uint4*>(a.q + (size_t(n) * a.Hq + h) * DH);
-#pragma unroll 4
-      for (int c = 0; c < DH / 8; ++c) {
-        const uint4 val = valid ? src[c] : make_uint4(0, 0, 0, 0);
-        const int sl = c >> 3, cc = c & 7;
-        *reinterpret_cast<uint4*>(smem + sl * (kBV * 128) + sw128(i, cc)) = val;
+      if (i >= rb * g) {
+#pragma unroll
+        for (int c = 0; c < DH / 8; ++c)
+          *reinterpret_cast<uint4*>(smem + (c >> 3) * (kBV * 128) + sw128(i, c & 7)) =
+              make_uint4(0, 0, 0, 0);
       }
       fence_proxy_async_smem();
       __syncwarp();
@@ -406,11 +445,19 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(s_free + b);
-      const int kvalid = min(kBN, k_end - (k_begin + j * kBN));
+      // visible keys of this tile: [klo, khi) of its 64 slots
+      int klo = 0, khi;
+      if (j < npt) {
+        khi = min(kBN, k_end - (k_begin + j * kBN));
+      } else {
+        const int f0 = f_begin + (j - npt) * kBN;
+        klo = max(0, fa - f0);
+        khi = min(kBN, fb - f0 + 1);
+      }
       float mt = -INFINITY;
 #pragma unroll
       for (int c = 0; c < kBN; ++c) {
-        sv[c] = c < kvalid ? sv[c] * a.scale_log2 : -INFINITY;
+        sv[c] = (c >= klo && c < khi) ? sv[c] * a.scale_log2 : -INFINITY;
         mt = fmaxf(mt, sv[c]);
       }
       // P_j reuses buffer b: PV_{j-2} must be done reading it
@@ -473,19 +520,29 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmK,
     if (ok) {
       tc_fence_after();
       const size_t base = (size_t(split) * a.N + n) * a.Hq + h;
+      const bool direct = splits_r == 1;  // the whole row in this CTA: final output
+      const float inv = l > 0.f ? 1.f / l : 0.f;
 #pragma unroll 1
       for (int c0 = 0; c0 < DH; c0 += 32) {
         float ov[32];
         tmem_ld_32cols(tmem + lane_off + G::kOCol + c0, ov);
         tmem_wait_ld();
-        if (valid) {
+        if (valid && direct) {
+          uint4* dst = reinterpret_cast<uint4*>(a.o + (size_t(n) * a.Hq + h) * DH + c0);
+#pragma unroll
+          for (int c = 0; c < 4; ++c)
+            dst[c] = make_uint4(pack_bf16(ov[8 * c] * inv, ov[8 * c + 1] * inv),
+                                pack_bf16(ov[8 * c + 2] * inv, ov[8 * c + 3] * inv),
+                                pack_bf16(ov[8 * c + 4] * inv, ov[8 * c + 5] * inv),
+                                pack_bf16(ov[8 * c + 6] * inv, ov[8 * c + 7] * inv));
+        } else if (valid) {
           float4* dst = reinterpret_cast<float4*>(a.o_part + base * DH + c0);
 #pragma unroll
           for (int c = 0; c < 8; ++c)
             dst[c] = make_float4(ov[4 * c], ov[4 * c + 1], ov[4 * c + 2], ov[4 * c + 3]);
         }
       }
-      if (valid) a.ml_part[base] = make_float2(m_used, l);
+      if (valid && !direct) a.ml_part[base] = make_float2(m_used, l);
     } else {
       *abort_flag = 1;
       flag(a.status, JET_ERR_TIMEOUT);
@@ -515,47 +572,117 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 }
 
 // packed [keys, Hkv, DH] bf16 K or V: box of 64 d x 1 head x 64 keys
-bool encode_kv(CUtensorMap* map, const void* base, int keys, int Hkv, int DH) {
+// packed [rows, heads, DH] bf16: box of 64 d x box_heads heads x box_rows rows
+bool encode_3d(CUtensorMap* map, const void* base, int rows, int heads, int DH, int box_heads,
+               int box_rows) {
   auto fn = encode_fn();
   if (!fn) return false;
-  const cuuint64_t dims[3] = {cuuint64_t(DH), cuuint64_t(Hkv), cuuint64_t(keys)};
-  const cuuint64_t strides[2] = {cuuint64_t(DH) * 2, cuuint64_t(Hkv) * DH * 2};
-  const cuuint32_t box[3] = {64, 1, cuuint32_t(kBN)};
+  const cuuint64_t dims[3] = {cuuint64_t(DH), cuuint64_t(heads), cuuint64_t(rows)};
+  const cuuint64_t strides[2] = {cuuint64_t(DH) * 2, cuuint64_t(heads) * DH * 2};
+  const cuuint32_t box[3] = {64, cuuint32_t(box_heads), cuuint32_t(box_rows)};
   const cuuint32_t estr[3] = {1, 1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// One warp per (row, query head) of a request whose prefix spans several
+// chunks: combine the chunks' base-2 partials (the last chunk also holds the
+// candidate's own keys) and normalise. Single-chunk requests were written by
+// the attention kernel itself.
+template <int DH>
+__global__ void __launch_bounds__(256)
+attend_combine_kernel(const int32_t* __restrict__ prefix_offset, const int32_t* __restrict__ row_req,
+                      int N, int R, int Hq, int chunk, const float* __restrict__ o_part,
+                      const float2* __restrict__ ml_part, __nv_bfloat16* __restrict__ o,
+                      int* status) {
+  const int lane = threadIdx.x & 31;
+  const long long idx = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (idx >= (long long)N * Hq) return;
+  const int n = int(idx / Hq), h = int(idx % Hq);
+  const int r = row_req[n];
+  if (r < 0 || r >= R) {
+    if (lane == 0) flag(status, JET_ERR_DEVICE);
+    return;
+  }
+  const int P = prefix_offset[r + 1] - prefix_offset[r];
+  const int splits_r = (P + chunk - 1) / chunk;
+  if (splits_r <= 1) return;
+  constexpr int PER = DH / 32;
+  float acc[PER];
+#pragma unroll
+  for (int i = 0; i < PER; ++i) acc[i] = 0.f;
+  float m = -INFINITY, l = 0.f;
+  for (int s = 0; s < splits_r; ++s) {
+    const size_t base = (size_t(s) * N + n) * Hq + h;
+    const float2 ml = ml_part[base];
+    if (!(ml.y > 0.f)) continue;
+    const float mn = fmaxf(m, ml.x);
+    const float fa = exp2f(m - mn), fb = exp2f(ml.x - mn);
+#pragma unroll
+    for (int i = 0; i < PER; ++i) acc[i] = acc[i] * fa + o_part[base * DH + lane + 32 * i] * fb;
+    l = l * fa + ml.y * fb;
+    m = mn;
+  }
+  const float inv = l > 0.f ? 1.f / l : 0.f;
+#pragma unroll
+  for (int i = 0; i < PER; ++i)
+    o[(size_t(n) * Hq + h) * DH + lane + 32 * i] = __float2bfloat16_rn(acc[i] * inv);
+}
+
 template <int DH>
 cudaError_t launch_dh(const jet_layout& lay, const jet_dims& d, const AttnPlan& plan,
-                      const void* q, const void* k_pre, const void* v_pre, float* o_part,
-                      float2* ml_part, int* status, cudaStream_t st) {
+                      const void* q, const void* k_pre, const void* v_pre, const void* k_cand,
+                      const void* v_cand, void* o, float* o_part, float2* ml_part, int* status,
+                      cudaStream_t st) {
   const jet_sizes& n = lay.n;
-  CUtensorMap tmK, tmV;
-  if (!encode_kv(&tmK, k_pre, n.total_prefix, d.Hkv, DH) ||
-      !encode_kv(&tmV, v_pre, n.total_prefix, d.Hkv, DH))
+  const int F = n.N - n.R;
+  const int g = d.Hq / d.Hkv;
+  if (g > kBV) return cudaErrorInvalidValue;
+  CUtensorMap tmQ, tmK, tmV, tmKc, tmVc;
+  if (!encode_3d(&tmQ, q, n.N, d.Hq, DH, g, kBV / g) ||
+      !encode_3d(&tmK, k_pre, n.total_prefix, d.Hkv, DH, 1, kBN) ||
+      !encode_3d(&tmV, v_pre, n.total_prefix, d.Hkv, DH, 1, kBN))
     return cudaErrorInvalidValue;
+  if (F > 0) {
+    if (!encode_3d(&tmKc, k_cand, F, d.Hkv, DH, 1, kBN) ||
+        !encode_3d(&tmVc, v_cand, F, d.Hkv, DH, 1, kBN))
+      return cudaErrorInvalidValue;
+  } else {
+    tmKc = tmK;  // never read: no request has candidate tiles
+    tmVc = tmV;
+  }
   AttArgs a{};
   a.prefix_offset = lay.prefix_offset;
   a.row_offset = lay.row_offset;
+  a.row_cand = lay.row_cand;
+  a.cand_row_offset = lay.cand_row_offset;
   a.q = static_cast<const __nv_bfloat16*>(q);
+  a.o = static_cast<__nv_bfloat16*>(o);
   a.o_part = o_part;
   a.ml_part = ml_part;
   a.status = status;
   a.R = n.R;
   a.N = n.N;
+  a.C = n.C;
   a.total_prefix = n.total_prefix;
   a.Hq = d.Hq;
   a.Hkv = d.Hkv;
   a.chunk = plan.chunk;
+  a.has_cand = F > 0;
   a.scale_log2 = 1.4426950408889634f / sqrtf(float(DH));
   const size_t smem = Geo<DH>::kBytes + 1024;
   cudaError_t e = cudaFuncSetAttribute(attend_prefix_tc_kernel<DH>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
   if (e != cudaSuccess) return e;
   dim3 grid(plan.splits, unsigned(n.R * d.Hkv), plan.qgroups);
-  attend_prefix_tc_kernel<DH><<<grid, kThreads, smem, st>>>(tmK, tmV, a);
+  attend_prefix_tc_kernel<DH><<<grid, kThreads, smem, st>>>(tmQ, tmK, tmV, tmKc, tmVc, a);
+  e = cudaGetLastError();
+  if (e != cudaSuccess || plan.splits <= 1) return e;
+  const long long warps = (long long)n.N * d.Hq;
+  attend_combine_kernel<DH><<<unsigned((warps + 7) / 8), 256, 0, st>>>(
+      lay.prefix_offset, lay.row_req, n.N, n.R, d.Hq, plan.chunk, o_part, ml_part,
+      static_cast<__nv_bfloat16*>(o), status);
   return cudaGetLastError();
 }
 
@@ -563,12 +690,17 @@ cudaError_t launch_dh(const jet_layout& lay, const jet_dims& d, const AttnPlan& 
 
 int attn_tc_block() { return kBV; }
 
-cudaError_t launch_prefix_attend_tc(const jet_layout& lay, const jet_dims& d, const AttnPlan& plan,
-                                    const void* q, const void* k_pre, const void* v_pre,
-                                    float* o_part, float2* ml_part, int* status, cudaStream_t st) {
-  if (d.d == 64) return launch_dh<64>(lay, d, plan, q, k_pre, v_pre, o_part, ml_part, status, st);
-  if (d.d == 128) return launch_dh<128>(lay, d, plan, q, k_pre, v_pre, o_part, ml_part, status, st);
-  if (d.d == 256) return launch_dh<256>(lay, d, plan, q, k_pre, v_pre, o_part, ml_part, status, st);
+cudaError_t launch_attend_tc(const jet_layout& lay, const jet_dims& d, const AttnPlan& plan,
+                             const void* q, const void* k_pre, const void* v_pre,
+                             const void* k_cand, const void* v_cand, void* o, float* o_part,
+                             float2* ml_part, int* status, cudaStream_t st) {
+#define JET_TC(DH)                                                                          \
+  return launch_dh<DH>(lay, d, plan, q, k_pre, v_pre, k_cand, v_cand, o, o_part, ml_part, \
+                       status, st)
+  if (d.d == 64) JET_TC(64);
+  if (d.d == 128) JET_TC(128);
+  if (d.d == 256) JET_TC(256);
+#undef JET_TC
   return cudaErrorInvalidValue;
 }
 

@@ -2,15 +2,17 @@
 //
 // The paper keeps one stored prefix state and restores it before each
 // candidate, evaluating candidates one after another. Here every candidate
-// of a request runs concurrently inside one CTA from a single read of the
-// prefix state: the state slice stays in registers, each candidate starts
-// from an unmodified copy of it, applies its fed tokens and writes its own
-// final state. Each fed token applies the gated delta rule
+// runs concurrently: one CTA per (32-column slice, head, candidate) starts
+// from an unmodified copy of the prefix state slice (read from HBM once and
+// from L2 by the request's other candidates), applies the candidate's fed
+// tokens and writes its own final state. Each fed token applies the gated
+// delta rule
 //   S <- alpha (S - beta k (k^T S)) + beta k v^T,   o = S^T q / sqrt(dk)
 // (the paper does not state its recurrence; this is the reading used).
 // The update is column-separable: column j of S needs only k, v_j and the
 // column's own u_j = k^T S[:, j], so a CTA owns a 32-column slice of one
-// head. The kernel is bound by the writes of the forked states.
+// head. The kernel is bound by the writes of the forked states; many small
+// independent CTAs keep enough of them in flight.
 #include "jet_device.cuh"
 #include "jet_internal.h"
 
@@ -48,7 +50,7 @@ __device__ __forceinline__ float4 rows_sum(float4 v, float* red, int warp, int l
   return s;
 }
 
-// grid (dv / 32, Hl, R); thread (warp w, lane = 8 * rg + jq) owns rows
+// grid (dv / 32, Hl, C); thread (warp w, lane = 8 * rg + jq) owns rows
 // 32 w + rg + 4 ii (ii < 8) and columns j0 + 4 jq .. + 3 of the slice.
 template <typename T>
 __global__ void __launch_bounds__(kThreads)
@@ -58,37 +60,34 @@ fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__
             const T* __restrict__ v, const float* __restrict__ alpha, const float* __restrict__ beta,
             T* __restrict__ o, float* __restrict__ s_fork, int* status) {
   __shared__ __align__(16) float red[4 * kCols];
-  const int r = blockIdx.z, h = blockIdx.y, j0 = blockIdx.x * kCols;
+  const int c = blockIdx.z, h = blockIdx.y, j0 = blockIdx.x * kCols;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int rg = lane >> 3, jq = lane & 7;
   const int col = j0 + 4 * jq;
-  if (r >= R) return;
-  const int c0 = cand_offset[r], c1 = cand_offset[r + 1];
-  if (c0 < 0 || c1 < c0 || c1 > C) {
+  if (c >= C) return;
+  // the candidate's request: the last r with cand_offset[r] <= c
+  int lo = 0, hi = R - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (cand_offset[mid] <= c) lo = mid; else hi = mid - 1;
+  }
+  const int r = lo;
+  const int m = tgt_offset[c + 1] - tgt_offset[c];
+  const int f0 = cand_row_offset[c] - r - 1;  // fed-token index of y_{c,1}
+  if (cand_offset[r] > c || cand_offset[r + 1] <= c || m < 1 || f0 < 0 || f0 + m - 1 > F) {
     if (threadIdx.x == 0) flag(status, JET_ERR_DEVICE);
     return;
   }
-
-  // the prefix state slice: read once, reused by every candidate
-  float4 sp[8];
-  const size_t head = (size_t(r) * Hl + h) * kDK;
-#pragma unroll
-  for (int ii = 0; ii < 8; ++ii) {
-    const int i = 32 * warp + rg + 4 * ii;
-    sp[ii] = *reinterpret_cast<const float4*>(s_prefix + (head + i) * dv + col);
-  }
   const float rs = rsqrtf(float(kDK));
-
-  for (int c = c0; c < c1; ++c) {
-    const int m = tgt_offset[c + 1] - tgt_offset[c];
-    const int f0 = cand_row_offset[c] - r - 1;  // fed-token index of y_{c,1}
-    if (m < 1 || f0 < 0 || f0 + m - 1 > F) {
-      if (threadIdx.x == 0) flag(status, JET_ERR_DEVICE);
-      continue;
-    }
+  {
+    // restore the prefix state: an unmodified copy of the request's slice
     float4 S[8];
+    const size_t head = (size_t(r) * Hl + h) * kDK;
 #pragma unroll
-    for (int ii = 0; ii < 8; ++ii) S[ii] = sp[ii];  // restore the prefix state
+    for (int ii = 0; ii < 8; ++ii) {
+      const int i = 32 * warp + rg + 4 * ii;
+      S[ii] = *reinterpret_cast<const float4*>(s_prefix + (head + i) * dv + col);
+    }
     for (int t = 0; t < m - 1; ++t) {
       const size_t fh = size_t(f0 + t) * Hl + h;
       float kk[8], qq[8];
@@ -145,7 +144,7 @@ cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, const fl
                               const float* beta, void* o, float* s_fork, int* status,
                               cudaStream_t st) {
   const jet_sizes& n = lay.n;
-  dim3 grid(unsigned(d.dv / kCols), unsigned(d.Hl), unsigned(n.R));
+  dim3 grid(unsigned(d.dv / kCols), unsigned(d.Hl), unsigned(n.C));
   const int F = n.N - n.R;
   if (d.dtype == JET_DTYPE_F32) {
     fork_kernel<float><<<grid, kThreads, 0, st>>>(

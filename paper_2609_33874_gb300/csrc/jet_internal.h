@@ -40,11 +40,13 @@ cudaError_t launch_prefix_attend(const jet_layout& lay, const jet_dims& d, const
                                  const void* k_cand, const void* v_cand, void* o, void* ws,
                                  int* status, cudaStream_t st);
 
-// bf16 prefix part on the tensor cores (attend_tc.cu); query vectors per CTA
+// bf16 cascade attention on the tensor cores (attend_tc.cu): prefix chunks and
+// the candidates' own keys, plus the chunk combine; query vectors per CTA
 int attn_tc_block();
-cudaError_t launch_prefix_attend_tc(const jet_layout& lay, const jet_dims& d, const AttnPlan& plan,
-                                    const void* q, const void* k_pre, const void* v_pre,
-                                    float* o_part, float2* ml_part, int* status, cudaStream_t st);
+cudaError_t launch_attend_tc(const jet_layout& lay, const jet_dims& d, const AttnPlan& plan,
+                             const void* q, const void* k_pre, const void* v_pre,
+                             const void* k_cand, const void* v_cand, void* o, float* o_part,
+                             float2* ml_part, int* status, cudaStream_t st);
 
 cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, const float* s_prefix,
                               const void* q, const void* k, const void* v, const float* alpha,
