@@ -463,10 +463,24 @@ def main():
     ap.add_argument("--ref-sample", type=int, default=1,
                     help="requests per step of the reference arm")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="one line per batch size R = 1, 2, 4, ... up to the workload's R "
+                         "(one GPU; no CPU baseline)")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)  # at least three untimed warm-up steps
     if args.impl == "reference":
         run_reference(args)
+    elif args.sweep:
+        import jet_synth
+        if _dist()[0] > 1:
+            ap.error("--sweep runs on one GPU")
+        args.no_cpu_baseline = True
+        full = jet_synth.WORKLOADS[args.workload].R
+        r = 1
+        while r <= full:
+            args.R = r
+            run_gpu(args)
+            r *= 2
     else:
         run_gpu(args)
 

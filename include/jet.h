@@ -141,6 +141,11 @@ typedef struct jet_dims {
   int32_t Hl;    /* linear-attention heads (0 when the model has none)        */
   int32_t dk;    /* linear-attention key dimension: 128                       */
   int32_t dv;    /* linear-attention value dimension: multiple of 32, <= 256 */
+  int32_t max_sms; /* at most this many SMs for the persistent LM-head kernel
+                      (0: all of them). An HBM-bound LM head reaches the
+                      bandwidth roof with fewer SMs; leaving some free lets a
+                      caller run other work (the next batch's attention) on
+                      another stream at the same time. */
 } jet_dims;
 
 /* ABI version of the loaded library (JET_ABI_VERSION it was built with). */

@@ -89,6 +89,7 @@ jet_status check_lm_dims(const jet_dims* d) {
   jet_status s = check_dtype(d);
   if (s) return s;
   if (d->D < 8 || d->D % 8 != 0) return JET_ERR_SHAPE;
+  if (d->max_sms < 0) return JET_ERR_ARG;
   return JET_OK;
 }
 

@@ -1,18 +1,18 @@
 // Per-candidate fork of a linear-attention recurrent state (Sec. 4.1).
 //
 // The paper keeps one stored prefix state and restores it before each
-// candidate, evaluating candidates one after another. Here every candidate
-// runs concurrently: one CTA per (32-column slice, head, candidate) starts
-// from an unmodified copy of the prefix state slice (read from HBM once and
-// from L2 by the request's other candidates), applies the candidate's fed
-// tokens and writes its own final state. Each fed token applies the gated
-// delta rule
+// candidate, evaluating candidates one after another. Here one CTA per
+// (32-column slice, head, request) reads the prefix state slice once into
+// registers and the request's fed tokens once into shared memory; every
+// candidate then starts from an unmodified register copy of the slice,
+// applies its fed tokens and writes its own final state, so the state
+// writes of one candidate overlap the arithmetic of the next. Each fed token
+// applies the gated delta rule
 //   S <- alpha (S - beta k (k^T S)) + beta k v^T,   o = S^T q / sqrt(dk)
 // (the paper does not state its recurrence; this is the reading used).
 // The update is column-separable: column j of S needs only k, v_j and the
 // column's own u_j = k^T S[:, j], so a CTA owns a 32-column slice of one
-// head. The kernel is bound by the writes of the forked states; many small
-// independent CTAs keep enough of them in flight.
+// head. The kernel is bound by the writes of the forked states.
 #include "jet_device.cuh"
 #include "jet_internal.h"
 
@@ -22,6 +22,7 @@ namespace {
 constexpr int kDK = 128;        // key dimension handled (rows of S)
 constexpr int kCols = 32;       // value columns per CTA
 constexpr int kThreads = 128;   // 4 warps x 32 rows
+constexpr int kWin = 32;        // fed tokens staged in shared memory at a time
 
 __device__ __forceinline__ float4 f4_fma(float a, float4 x, float4 y) {
   return make_float4(fmaf(a, x.x, y.x), fmaf(a, x.y, y.y), fmaf(a, x.z, y.z), fmaf(a, x.w, y.w));
@@ -50,56 +51,87 @@ __device__ __forceinline__ float4 rows_sum(float4 v, float* red, int warp, int l
   return s;
 }
 
-// grid (dv / 32, Hl, C); thread (warp w, lane = 8 * rg + jq) owns rows
+// grid (dv / 32, Hl, R); thread (warp w, lane = 8 * rg + jq) owns rows
 // 32 w + rg + 4 ii (ii < 8) and columns j0 + 4 jq .. + 3 of the slice.
 template <typename T>
 __global__ void __launch_bounds__(kThreads)
 fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__ cand_row_offset,
-            const int32_t* __restrict__ tgt_offset, int R, int C, int F, int Hl, int dv,
-            const float* __restrict__ s_prefix, const T* __restrict__ q, const T* __restrict__ k,
-            const T* __restrict__ v, const float* __restrict__ alpha, const float* __restrict__ beta,
-            T* __restrict__ o, float* __restrict__ s_fork, int* status) {
+            const int32_t* __restrict__ tgt_offset, const int32_t* __restrict__ row_offset,
+            int R, int C, int F, int Hl, int dv, const float* __restrict__ s_prefix,
+            const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
+            const float* __restrict__ alpha, const float* __restrict__ beta, T* __restrict__ o,
+            float* __restrict__ s_fork, int* status) {
   __shared__ __align__(16) float red[4 * kCols];
-  const int c = blockIdx.z, h = blockIdx.y, j0 = blockIdx.x * kCols;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // a window of the request's fed tokens: k, q (all rows), v (this slice), gates
+  __shared__ __align__(16) float wk[kWin][kDK];
+  __shared__ __align__(16) float wq[kWin][kDK];
+  __shared__ __align__(16) float wv[kWin][kCols];
+  __shared__ float wa[kWin], wb[kWin];
+  const int r = blockIdx.z, h = blockIdx.y, j0 = blockIdx.x * kCols;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rg = lane >> 3, jq = lane & 7;
   const int col = j0 + 4 * jq;
-  if (c >= C) return;
-  // the candidate's request: the last r with cand_offset[r] <= c
-  int lo = 0, hi = R - 1;
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (cand_offset[mid] <= c) lo = mid; else hi = mid - 1;
-  }
-  const int r = lo;
-  const int m = tgt_offset[c + 1] - tgt_offset[c];
-  const int f0 = cand_row_offset[c] - r - 1;  // fed-token index of y_{c,1}
-  if (cand_offset[r] > c || cand_offset[r + 1] <= c || m < 1 || f0 < 0 || f0 + m - 1 > F) {
-    if (threadIdx.x == 0) flag(status, JET_ERR_DEVICE);
+  if (r >= R) return;
+  const int c0 = cand_offset[r], c1 = cand_offset[r + 1];
+  const int f_begin = row_offset[r] - r;                   // the request's first fed token
+  const int f_end = f_begin + row_offset[r + 1] - row_offset[r] - 1;
+  if (c0 < 0 || c1 < c0 || c1 > C || f_begin < 0 || f_end < f_begin || f_end > F) {
+    if (tid == 0) flag(status, JET_ERR_DEVICE);
     return;
   }
-  const float rs = rsqrtf(float(kDK));
-  {
-    // restore the prefix state: an unmodified copy of the request's slice
-    float4 S[8];
-    const size_t head = (size_t(r) * Hl + h) * kDK;
+
+  // the prefix state slice: read once, reused by every candidate
+  float4 sp[8];
+  const size_t head = (size_t(r) * Hl + h) * kDK;
 #pragma unroll
-    for (int ii = 0; ii < 8; ++ii) {
-      const int i = 32 * warp + rg + 4 * ii;
-      S[ii] = *reinterpret_cast<const float4*>(s_prefix + (head + i) * dv + col);
+  for (int ii = 0; ii < 8; ++ii) {
+    const int i = 32 * warp + rg + 4 * ii;
+    sp[ii] = *reinterpret_cast<const float4*>(s_prefix + (head + i) * dv + col);
+  }
+  const float rs = rsqrtf(float(kDK));
+  int w0 = f_begin, w1 = f_begin;  // fed tokens [w0, w1) are staged
+
+  for (int c = c0; c < c1; ++c) {
+    const int m = tgt_offset[c + 1] - tgt_offset[c];
+    const int f0 = cand_row_offset[c] - r - 1;  // fed-token index of y_{c,1}
+    if (m < 1 || f0 < f_begin || f0 + m - 1 > f_end) {
+      if (tid == 0) flag(status, JET_ERR_DEVICE);
+      continue;
     }
+    float4 S[8];
+#pragma unroll
+    for (int ii = 0; ii < 8; ++ii) S[ii] = sp[ii];  // restore the prefix state
     for (int t = 0; t < m - 1; ++t) {
-      const size_t fh = size_t(f0 + t) * Hl + h;
+      const int f = f0 + t;
+      if (f >= w1) {
+        // stage the next window of fed tokens with coalesced loads
+        __syncthreads();
+        w0 = f;
+        w1 = min(f + kWin, f_end);
+        const int nt = w1 - w0;
+        for (int e = tid; e < nt * kDK; e += kThreads) {
+          const size_t src = (size_t(w0 + e / kDK) * Hl + h) * kDK + e % kDK;
+          wk[e / kDK][e % kDK] = to_f32(k[src]);
+          wq[e / kDK][e % kDK] = to_f32(q[src]);
+        }
+        for (int e = tid; e < nt * kCols; e += kThreads)
+          wv[e / kCols][e % kCols] = to_f32(v[(size_t(w0 + e / kCols) * Hl + h) * dv + j0 + e % kCols]);
+        for (int e = tid; e < nt; e += kThreads) {
+          wa[e] = alpha[size_t(w0 + e) * Hl + h];
+          wb[e] = beta[size_t(w0 + e) * Hl + h];
+        }
+        __syncthreads();
+      }
+      const int wt = f - w0;
       float kk[8], qq[8];
 #pragma unroll
       for (int ii = 0; ii < 8; ++ii) {
         const int i = 32 * warp + rg + 4 * ii;
-        kk[ii] = to_f32(k[fh * kDK + i]);
-        qq[ii] = to_f32(q[fh * kDK + i]);
+        kk[ii] = wk[wt][i];
+        qq[ii] = wq[wt][i];
       }
-      const float a = alpha[fh], b = beta[fh];
-      const float4 vv = make_float4(to_f32(v[fh * dv + col]), to_f32(v[fh * dv + col + 1]),
-                                    to_f32(v[fh * dv + col + 2]), to_f32(v[fh * dv + col + 3]));
+      const float a = wa[wt], b = wb[wt];
+      const float4 vv = *reinterpret_cast<const float4*>(&wv[wt][4 * jq]);
       // u = k^T S for this column quad
       float4 u = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
@@ -119,7 +151,7 @@ fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__
       }
       op = rows_sum(op, red, warp, lane);
       if (warp == 0 && rg == 0) {
-        T* dst = o + fh * dv + col;
+        T* dst = o + (size_t(f) * Hl + h) * dv + col;
         dst[0] = from_f32<T>(op.x * rs);
         dst[1] = from_f32<T>(op.y * rs);
         dst[2] = from_f32<T>(op.z * rs);
@@ -144,16 +176,18 @@ cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, const fl
                               const float* beta, void* o, float* s_fork, int* status,
                               cudaStream_t st) {
   const jet_sizes& n = lay.n;
-  dim3 grid(unsigned(d.dv / kCols), unsigned(d.Hl), unsigned(n.C));
+  dim3 grid(unsigned(d.dv / kCols), unsigned(d.Hl), unsigned(n.R));
   const int F = n.N - n.R;
   if (d.dtype == JET_DTYPE_F32) {
     fork_kernel<float><<<grid, kThreads, 0, st>>>(
-        lay.cand_offset, lay.cand_row_offset, lay.tgt_offset, n.R, n.C, F, d.Hl, d.dv, s_prefix,
+        lay.cand_offset, lay.cand_row_offset, lay.tgt_offset, lay.row_offset, n.R, n.C, F, d.Hl,
+        d.dv, s_prefix,
         static_cast<const float*>(q), static_cast<const float*>(k), static_cast<const float*>(v),
         alpha, beta, static_cast<float*>(o), s_fork, status);
   } else {
     fork_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(
-        lay.cand_offset, lay.cand_row_offset, lay.tgt_offset, n.R, n.C, F, d.Hl, d.dv, s_prefix,
+        lay.cand_offset, lay.cand_row_offset, lay.tgt_offset, lay.row_offset, n.R, n.C, F, d.Hl,
+        d.dv, s_prefix,
         static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k),
         static_cast<const __nv_bfloat16*>(v), alpha, beta, static_cast<__nv_bfloat16*>(o), s_fork,
         status);

@@ -386,7 +386,9 @@ cudaError_t launch_lmhead_tc(const jet_layout& lay, const jet_dims& d, const Sco
   cudaError_t e = cudaFuncSetAttribute(lmhead_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        int(smem));
   if (e != cudaSuccess) return e;
-  const int grid = std::max(1, std::min(a.units, sm_count()));
+  int sms = sm_count();
+  if (d.max_sms > 0) sms = std::min(sms, d.max_sms);
+  const int grid = std::max(1, std::min(a.units, sms));
   lmhead_tc_kernel<<<grid, kThreads, smem, st>>>(tmW, tmH, a);
   return cudaGetLastError();
 }

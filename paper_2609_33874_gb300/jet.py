@@ -55,7 +55,8 @@ class jet_layout(ctypes.Structure):
 
 
 class jet_dims(ctypes.Structure):
-    _fields_ = [(n, ctypes.c_int32) for n in ("dtype", "Hq", "Hkv", "d", "D", "Hl", "dk", "dv")]
+    _fields_ = [(n, ctypes.c_int32) for n in ("dtype", "Hq", "Hkv", "d", "D", "Hl", "dk", "dv",
+                                              "max_sms")]
 
 
 def _load() -> ctypes.CDLL:
@@ -196,8 +197,9 @@ def jet_layout_build(prefix_len, n_cand, cand_len, target_ids, V: int) -> HostLa
     return HostLayout(sizes, words, struct)
 
 
-def make_dims(dtype: int, Hq=0, Hkv=0, d=0, D=0, Hl=0, dk=0, dv=0) -> jet_dims:
-    return jet_dims(int(dtype), int(Hq), int(Hkv), int(d), int(D), int(Hl), int(dk), int(dv))
+def make_dims(dtype: int, Hq=0, Hkv=0, d=0, D=0, Hl=0, dk=0, dv=0, max_sms=0) -> jet_dims:
+    return jet_dims(int(dtype), int(Hq), int(Hkv), int(d), int(D), int(Hl), int(dk), int(dv),
+                    int(max_sms))
 
 
 def jet_workspace_bytes(sizes: jet_sizes, dims: jet_dims) -> int:

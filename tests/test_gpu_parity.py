@@ -181,6 +181,26 @@ def test_corrupt_device_layout_is_flagged(cuda):
     assert cuda.jet_device_status() == 0
 
 
+def test_lm_head_sm_budget_gives_identical_results(cuda):
+    # fewer persistent CTAs change which CTA computes a tile, not the tile's arithmetic
+    import torch
+    p = jet_synth.make_problem("binary")
+    step, x, w_lm = build_step(cuda, p)
+    step.run(x, w_lm)
+    torch.cuda.synchronize()
+    ref = step.tok_logprob.clone()
+    d = step.dims
+    capped = cuda.make_dims(d.dtype, Hq=d.Hq, Hkv=d.Hkv, d=d.d, D=d.D, max_sms=37)
+    cuda.jet_score_candidates(step.layout, capped, x["hidden"], w_lm, step.tok_logprob,
+                              step.cand_score, step.ws)
+    torch.cuda.synchronize()
+    assert torch.equal(step.tok_logprob, ref)
+    bad = cuda.make_dims(d.dtype, Hq=d.Hq, Hkv=d.Hkv, d=d.d, D=d.D, max_sms=-1)
+    with pytest.raises(cuda.JetError):
+        cuda.jet_score_candidates(step.layout, bad, x["hidden"], w_lm, step.tok_logprob,
+                                  step.cand_score, step.ws)
+
+
 def test_end_to_end_from_host(cuda):
     import torch
     p = jet_synth.make_problem("tiny")
