@@ -113,6 +113,9 @@ typedef struct jet_sizes {
  *   row_pos[N]           t of the token fed at row n, 0 for a shared row
  *   row_tgt_offset[N+1], row_tgt_index[T]
  *                        the targets predicted by row n, in increasing index
+ *   req_order[R]         the requests by decreasing prefix length (ties: lower
+ *                        index first); the attention kernels hand out long
+ *                        prefixes first
  */
 typedef struct jet_layout {
   jet_sizes n;
@@ -128,9 +131,10 @@ typedef struct jet_layout {
   const int32_t* row_pos;
   const int32_t* row_tgt_offset;
   const int32_t* row_tgt_index;
+  const int32_t* req_order;
 } jet_layout;
 
-/* Model dimensions of the step. */
+/* Model dimensions of the step (and one launch limit). */
 typedef struct jet_dims {
   int32_t dtype; /* JET_DTYPE_*: element type of q, k, v, o, hidden, w_lm    */
   int32_t Hq;    /* attention query heads                                    */

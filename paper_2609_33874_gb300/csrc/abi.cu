@@ -62,10 +62,11 @@ jet_status check_layout(const jet_layout* lay) {
       n.max_prefix > n.total_prefix || n.min_cand < 1 || n.max_cand < n.min_cand ||
       n.max_rows < 1 || n.max_rows > n.N || n.max_len < 1 || n.N - n.R != n.T - n.C)
     return JET_ERR_SHAPE;
-  const void* arrays[12] = {lay->prefix_offset, lay->cand_offset,    lay->row_offset,
+  const void* arrays[13] = {lay->prefix_offset, lay->cand_offset,    lay->row_offset,
                             lay->cand_row_offset, lay->tgt_offset,   lay->target_ids,
                             lay->tgt_row,       lay->row_req,        lay->row_cand,
-                            lay->row_pos,       lay->row_tgt_offset, lay->row_tgt_index};
+                            lay->row_pos,       lay->row_tgt_offset, lay->row_tgt_index,
+                            lay->req_order};
   for (const void* a : arrays)
     if (!a) return JET_ERR_ARG;
   return JET_OK;

@@ -265,6 +265,9 @@ AttnPlan attn_plan(const jet_sizes& n, const jet_dims& d) {
   p.splits = (n.max_prefix + chunk - 1) / chunk;
   const size_t vecs = size_t(p.splits) * n.N * d.Hq;
   p.bytes = vecs * d.d * sizeof(float) + vecs * sizeof(float2);
+  // tensor-core path: a work list of (request, kv head, query block, chunk)
+  // items plus two counters, 16-byte aligned, after the partials
+  if (tc) p.bytes += 32 + 16 * size_t(n.R) * d.Hkv * p.qgroups * p.splits;
   return p;
 }
 

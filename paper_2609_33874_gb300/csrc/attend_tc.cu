@@ -52,7 +52,7 @@ struct Geo {
   static constexpr uint32_t kOffK = kQBytes;                // stage s: K at kOffK + s * 2 kKV
   static constexpr uint32_t kOffP = kQBytes + kStages * 2 * kKVBytes;
   static constexpr uint32_t kOffBar = kOffP + 2 * kPBytes;
-  static constexpr uint32_t kBytes = kOffBar + 256;
+  static constexpr uint32_t kBytes = kOffBar + 512;
   static constexpr uint32_t kTmemCols = (2 * kBN + DH) <= 256 ? 256 : 512;
   static constexpr uint32_t kOCol = 2 * kBN;                // O after the two S buffers
 };
@@ -60,6 +60,7 @@ struct Geo {
 struct AttArgs {
   const int32_t* prefix_offset;
   const int32_t* row_offset;
+  const int32_t* req_order;
   const int32_t* row_cand;
   const int32_t* cand_row_offset;
   const __nv_bfloat16* q;
@@ -67,7 +68,15 @@ struct AttArgs {
   float* o_part;
   float2* ml_part;
   int* status;
+  int4* items;       // work list (attend_items_kernel)
+  int* item_count;
+  int* item_next;    // next item to take (dynamic schedule)
   int R, N, C, total_prefix, Hq, Hkv, chunk;
+  int g, rb;         // query heads per kv head; rows per query block (128 / g)
+  int sorted;        // 1: take items from the longest-first work list; 0: static
+                     // round-robin over all (request, kv head, block, chunk) slots
+  int splits;        // chunks per request (the plan's), for the static order
+  long long n_all;   // slots in the static order
   int has_cand;      // the batch has fed candidate tokens (F > 0)
   float scale_log2;  // log2(e) / sqrt(d)
 };
@@ -143,6 +152,120 @@ __device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap* map, int32_t 
                : "memory");
 }
 
+// Geometry of one work item (request r, key/value head kh, query block qb,
+// prefix chunk split); every role derives it the same way from the item.
+struct ItemGeo {
+  int r, kh, n0, nr, p0, P, row0, vbase, nv, k_begin, k_end, npt, nct, ntiles, splits_r, f_begin;
+  int split;
+  bool ok;
+};
+
+__device__ __forceinline__ ItemGeo item_geo(const AttArgs& a, int4 it) {
+  ItemGeo e{};
+  e.r = it.x;
+  e.kh = it.y;
+  const int qb = it.z;
+  e.split = it.w;
+  e.ok = false;
+  if (e.r < 0 || e.r >= a.R || e.kh < 0 || e.kh >= a.Hkv) return e;
+  e.n0 = a.row_offset[e.r];
+  e.nr = a.row_offset[e.r + 1] - e.n0;
+  e.p0 = a.prefix_offset[e.r];
+  e.P = a.prefix_offset[e.r + 1] - e.p0;
+  if (e.n0 < 0 || e.nr < 1 || e.n0 + e.nr > a.N || e.p0 < 0 || e.P < 1 ||
+      e.p0 + e.P > a.total_prefix)
+    return e;
+  e.row0 = qb * a.rb;
+  if (e.row0 >= e.nr) return e;
+  e.vbase = e.row0 * a.g;
+  e.nv = min(a.rb, e.nr - e.row0) * a.g;
+  e.k_begin = e.split * a.chunk;
+  e.k_end = min(e.P, e.k_begin + a.chunk);
+  if (e.k_end <= e.k_begin) return e;
+  e.npt = (e.k_end - e.k_begin + kBN - 1) / kBN;
+  // the request's last chunk also takes its candidates' own keys: the F_r fed
+  // tokens, as extra 64-key tiles masked per row to the row's candidate and
+  // position (Sec. 4.1: a candidate attends to its own earlier tokens only)
+  e.splits_r = (e.P + a.chunk - 1) / a.chunk;
+  e.f_begin = e.n0 - e.r;  // fed-token index of the request's first fed row
+  const int F_r = e.nr - 1;
+  e.nct = (e.split == e.splits_r - 1 && a.has_cand && F_r > 0) ? (F_r + kBN - 1) / kBN : 0;
+  e.ntiles = e.npt + e.nct;
+  e.ok = true;
+  return e;
+}
+
+// The work list: every (request, kv head, query block, chunk) that has keys
+// and vectors, longest first (counting sort on the tile count), for the
+// persistent kernel's dynamic schedule. One block.
+constexpr int kBuckets = 256;
+
+constexpr int kItemCache = 16384;  // candidate items whose bucket stays in shared memory
+
+__device__ __forceinline__ int4 item_of(const AttArgs& a, long long idx, int splits) {
+  const int split = int(idx % splits);
+  const long long rest = idx / splits;
+  const int rk = int(rest % (a.R * a.Hkv));
+  const int qb = int(rest / (a.R * a.Hkv));
+  return make_int4(rk / a.Hkv, rk % a.Hkv, qb, split);
+}
+
+__global__ void __launch_bounds__(1024)
+attend_items_kernel(const AttArgs a, int qgroups, int splits) {
+  __shared__ int hist[kBuckets];
+  __shared__ int cursor[kBuckets];
+  __shared__ int wsum[kBuckets / 32];
+  __shared__ uint8_t bucket[kItemCache];  // 0: no item, else min(tiles, 255)
+  for (int b = threadIdx.x; b < kBuckets; b += blockDim.x) hist[b] = 0;
+  __syncthreads();
+  const long long n_all = (long long)a.R * a.Hkv * qgroups * splits;
+  for (long long idx = threadIdx.x; idx < n_all; idx += blockDim.x) {
+    const ItemGeo e = item_geo(a, item_of(a, idx, splits));
+    const int b = e.ok ? min(e.ntiles, kBuckets - 1) : 0;
+    if (idx < kItemCache) bucket[idx] = uint8_t(b);
+    if (b > 0) atomicAdd(&hist[b], 1);
+  }
+  __syncthreads();
+  // exclusive scan of the buckets from the longest down (longest items first)
+  if (threadIdx.x < kBuckets) {
+    const int t = threadIdx.x, lane = t & 31, w = t >> 5;
+    const int val = hist[kBuckets - 1 - t];
+    int inc = val;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += y;
+    }
+    if (lane == 31) wsum[w] = inc;
+    __syncwarp();
+    asm volatile("bar.sync 1, %0;" ::"r"(kBuckets) : "memory");
+    int base = 0;
+    for (int i = 0; i < w; ++i) base += wsum[i];
+    cursor[kBuckets - 1 - t] = base + inc - val;
+    if (t == kBuckets - 1) {
+      *a.item_count = base + inc;
+      *a.item_next = 0;
+    }
+  }
+  __syncthreads();
+  for (long long idx = threadIdx.x; idx < n_all; idx += blockDim.x) {
+    const int4 it = item_of(a, idx, splits);
+    int b;
+    if (idx < kItemCache) {
+      b = bucket[idx];
+    } else {
+      const ItemGeo e = item_geo(a, it);
+      b = e.ok ? min(e.ntiles, kBuckets - 1) : 0;
+    }
+    if (b > 0) a.items[atomicAdd(&cursor[b], 1)] = it;
+  }
+}
+
+// One persistent CTA per SM; items are taken from the work list one at a time
+// by the producer and handed to the other roles through a two-slot ring. All
+// barrier phases run on counters that continue across items, so the next
+// item's query block and first K/V tiles load while the current item's last
+// tiles and its output are still in flight.
 template <int DH>
 __global__ void __launch_bounds__(kThreads, 1)
 attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
@@ -154,9 +277,11 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  // K and V of a stage fill and drain separately: K is free once S_j has been
-  // computed, V only after P_j V_j
-  uint64_t* k_full = reinterpret_cast<uint64_t*>(smem + G::kOffBar);
+  // the item ring first (16-byte entries at a 1024-byte aligned offset), then
+  // the barriers. K and V of a stage fill and drain separately: K is free once
+  // S_j has been computed, V only after P_j V_j
+  int4* ring = reinterpret_cast<int4*>(smem + G::kOffBar);  // [2] items
+  uint64_t* k_full = reinterpret_cast<uint64_t*>(ring + 2);
   uint64_t* k_empty = k_full + kStages;
   uint64_t* v_full = k_empty + kStages;
   uint64_t* v_empty = v_full + kStages;
@@ -164,52 +289,18 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   uint64_t* s_free = s_full + 2;           // [2]
   uint64_t* p_full = s_free + 2;           // [2]
   uint64_t* p_free = p_full + 2;           // [2]
-  uint64_t* q_full = p_free + 2;
-  uint64_t* drain = q_full + 1;
+  uint64_t* item_full = p_free + 2;        // [2]
+  uint64_t* item_empty = item_full + 2;    // [2]
+  uint64_t* q_full = item_empty + 2;       // query block of the current item landed
+  uint64_t* q_free = q_full + 1;           // last QK^T of the previous item done
+  uint64_t* o_free = q_free + 1;           // previous item's O read out of TMEM
+  uint64_t* qz_done = o_free + 1;          // unused query rows zeroed (once)
+  uint64_t* drain = qz_done + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
-  // query blocks are the slowest grid dimension: blocks past a request's
-  // vectors (only long requests have them) come last and exit at once
-  const int split = blockIdx.x, qb = blockIdx.z;
-  const int r = blockIdx.y / a.Hkv, kh = blockIdx.y % a.Hkv;
-  const int g = a.Hq / a.Hkv;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (r >= a.R) return;
-  const int n0 = a.row_offset[r], nr = a.row_offset[r + 1] - n0;
-  const int p0 = a.prefix_offset[r], P = a.prefix_offset[r + 1] - p0;
-  if (n0 < 0 || nr < 1 || n0 + nr > a.N || p0 < 0 || P < 0 || p0 + P > a.total_prefix) {
-    if (threadIdx.x == 0) flag(a.status, JET_ERR_DEVICE);
-    return;
-  }
-  // a query block holds whole rows: rb rows x g heads (<= 128 vectors)
-  const int rb = kBV / g;
-  const int row0 = qb * rb;  // first row of the block within the request
-  if (row0 >= nr) return;
-  const int vbase = row0 * g;
-  const int nv = min(rb, nr - row0) * g;
-  const int k_begin = split * a.chunk;
-  const int k_end = min(P, k_begin + a.chunk);
-  const int npt = k_end > k_begin ? (k_end - k_begin + kBN - 1) / kBN : 0;  // prefix tiles
-  // the request's last chunk also takes its candidates' own keys: the F_r fed
-  // tokens, as extra 64-key tiles masked per row to the row's candidate and
-  // position (Sec. 4.1: a candidate attends to its own earlier tokens only)
-  const int splits_r = (P + a.chunk - 1) / a.chunk;
-  const bool last = npt > 0 && split == splits_r - 1;
-  const int f_begin = n0 - r;     // fed-token index of the request's first fed row
-  const int F_r = nr - 1;
-  const int nct = (last && a.has_cand && F_r > 0) ? (F_r + kBN - 1) / kBN : 0;
-  const int ntiles = npt + nct;
-
-  if (npt == 0) {  // an empty chunk: an empty partial
-    for (int i = threadIdx.x; i < nv; i += blockDim.x) {
-      const int gv = vbase + i;
-      const size_t base = (size_t(split) * a.N + n0 + gv / g) * a.Hq + kh * g + gv % g;
-      a.ml_part[base] = make_float2(-INFINITY, 0.f);
-    }
-    return;
-  }
-
+  const int g = a.g, rb = a.rb;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(k_full + s, 1);
@@ -222,8 +313,13 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       mbar_init(s_free + b, 4);
       mbar_init(p_full + b, 4);
       mbar_init(p_free + b, 1);
+      mbar_init(item_full + b, 1);
+      mbar_init(item_empty + b, 5);  // the MMA thread + 4 softmax warps
     }
-    mbar_init(q_full, 5);  // the query TMA (with its bytes) + 4 softmax warps
+    mbar_init(q_full, 1);
+    mbar_init(q_free, 1);
+    mbar_init(o_free, 4);
+    mbar_init(qz_done, 4);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -236,7 +332,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
     tma_prefetch_desc(&tmQ);
     tma_prefetch_desc(&tmK);
     tma_prefetch_desc(&tmV);
-    if (nct > 0) {
+    if (a.has_cand) {
       tma_prefetch_desc(&tmKc);
       tma_prefetch_desc(&tmVc);
     }
@@ -245,83 +341,138 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  const int4 kDone = make_int4(-1, -1, -1, -1);
 
   if (warp == 0) {
     // ---------------------------------------------------------------- producer
     if (lane == 0) {
-      // the query block: rb rows x g heads x d of the request's group kh
-      mbar_arrive_expect_tx(q_full, uint32_t(G::kSlices) * 64 * 2 * g * rb);
-#pragma unroll
-      for (int sl = 0; sl < G::kSlices; ++sl)
-        tma_load_3d(smem + sl * (kBV * 128), &tmQ, q_full, sl * 64, kh * g, n0 + row0,
-                    policy_evict_first());
-      // K_j and V_j are issued as soon as their slots drain, whichever first
       const uint64_t pol = policy_evict_first();
-      uint32_t k_issued = 0, k_par = 0, v_issued = 0, v_par = 0;
-      int jk = 0, jv = 0;
+      const int count = a.sorted ? *a.item_count : 0;
+      uint32_t k_issued = 0, k_par = 0, v_issued = 0, v_par = 0, q_issued = 0, q_par = 0;
+      int Tk = 0, Tv = 0, v = 0;  // K and V tiles issued so far, items processed so far
       bool ok = true;
-      uint64_t t_last = global_timer_ns();
-      while (jv < ntiles) {
-        bool progressed = false;
-        if (jk < ntiles) {
-          const int s = jk % kStages;
-          const uint32_t ph = (jk / kStages) & 1;
-          if (mbar_test(k_empty + s, ph ^ 1u)) {
-            uint8_t* ks = smem + G::kOffK + s * 2 * G::kKVBytes;
-            mbar_arrive_expect_tx(k_full + s, G::kKVBytes);
-            const bool pre = jk < npt;
-            const CUtensorMap* mk = pre ? &tmK : &tmKc;
-            const int key = pre ? p0 + k_begin + jk * kBN : f_begin + (jk - npt) * kBN;
-#pragma unroll
-            for (int sl = 0; sl < G::kSlices; ++sl)
-              tma_load_3d(ks + sl * (kBN * 128), mk, k_full + s, sl * 64, kh, key, pol);
-            // keep kPrefetch further tiles on their way into L2: two shared
-            // stages alone hold too few bytes in flight to cover HBM latency
-            for (int jp = (jk == 0 ? 1 : jk + kPrefetch); jp <= jk + kPrefetch && jp < npt;
-                 ++jp) {
-              const int kp = p0 + k_begin + jp * kBN;
-#pragma unroll
-              for (int sl = 0; sl < G::kSlices; ++sl) {
-                tma_prefetch_3d(&tmK, sl * 64, kh, kp);
-                tma_prefetch_3d(&tmV, sl * 64, kh, kp);
-              }
-            }
-            k_issued |= 1u << s;
-            k_par = (k_par & ~(1u << s)) | (ph << s);
-            ++jk;
-            progressed = true;
-          }
-        }
-        if (jv < jk) {
-          const int s = jv % kStages;
-          const uint32_t ph = (jv / kStages) & 1;
-          if (mbar_test(v_empty + s, ph ^ 1u)) {
-            uint8_t* vs = smem + G::kOffK + s * 2 * G::kKVBytes + G::kKVBytes;
-            mbar_arrive_expect_tx(v_full + s, G::kKVBytes);
-            const bool pre = jv < npt;
-            const CUtensorMap* mv = pre ? &tmV : &tmVc;
-            const int key = pre ? p0 + k_begin + jv * kBN : f_begin + (jv - npt) * kBN;
-#pragma unroll
-            for (int sl = 0; sl < G::kSlices; ++sl)
-              tma_load_3d(vs + sl * (kBN * 128), mv, v_full + s, sl * 64, kh, key, pol);
-            v_issued |= 1u << s;
-            v_par = (v_par & ~(1u << s)) | (ph << s);
-            ++jv;
-            progressed = true;
-          }
-        }
-        const uint64_t now = global_timer_ns();
-        if (progressed) {
-          t_last = now;
-        } else if (*abort_flag || now - t_last > kWaitNs) {
+      for (int u = 0; ok; ++u) {
+        const int slot = u & 1;
+        if (!mbar_wait(item_empty + slot, ((u >> 1) & 1) ^ 1u, kWaitNs, abort_flag)) {
           ok = false;
           break;
         }
+        int4 it = kDone;
+        if (a.sorted) {
+          const int idx = atomicAdd(a.item_next, 1);
+          if (idx < count) it = a.items[idx];
+        } else {
+          // the next slot that holds work, taken from a shared counter; slots
+          // run over the requests by decreasing prefix length (query blocks
+          // past the first, mostly empty, last)
+          while (true) {
+            const long long sl = atomicAdd(a.item_next, 1);
+            if (sl >= a.n_all) break;
+            const int split = int(sl % a.splits);
+            const long long rest = sl / a.splits;
+            const int kh = int(rest % a.Hkv);
+            const long long rest2 = rest / a.Hkv;
+            const int ri = int(rest2 % a.R);
+            const int qb = int(rest2 / a.R);
+            const int4 cand = make_int4(a.req_order[ri], kh, qb, split);
+            if (item_geo(a, cand).ok) {
+              it = cand;
+              break;
+            }
+          }
+        }
+        ring[slot] = it;
+        mbar_arrive(item_full + slot);
+        if (it.x < 0) break;
+        const ItemGeo e = item_geo(a, it);
+        if (!e.ok) {
+          flag(a.status, JET_ERR_DEVICE);
+          continue;
+        }
+        // the query block: rb rows x g heads x d of the group, once the last
+        // QK^T of the previous item has read the old one
+        if (v >= 1 && !mbar_wait(q_free, (v - 1) & 1, kWaitNs, abort_flag)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(q_full, uint32_t(G::kSlices) * 64 * 2 * g * rb);
+#pragma unroll
+        for (int sl = 0; sl < G::kSlices; ++sl)
+          tma_load_3d(smem + sl * (kBV * 128), &tmQ, q_full, sl * 64, e.kh * g, e.n0 + e.row0,
+                      pol);
+        q_issued = 1;
+        q_par = v & 1;
+        // K_j and V_j are issued as soon as their slots drain, whichever first
+        int jk = 0, jv = 0;
+        uint64_t t_last = global_timer_ns();
+        while (jv < e.ntiles) {
+          bool progressed = false;
+          if (jk < e.ntiles) {
+            const int T = Tk + jk;
+            const int s = T % kStages;
+            const uint32_t ph = (T / kStages) & 1;
+            if (mbar_test(k_empty + s, ph ^ 1u)) {
+              uint8_t* ks = smem + G::kOffK + s * 2 * G::kKVBytes;
+              mbar_arrive_expect_tx(k_full + s, G::kKVBytes);
+              const bool pre = jk < e.npt;
+              const CUtensorMap* mk = pre ? &tmK : &tmKc;
+              const int key = pre ? e.p0 + e.k_begin + jk * kBN : e.f_begin + (jk - e.npt) * kBN;
+#pragma unroll
+              for (int sl = 0; sl < G::kSlices; ++sl)
+                tma_load_3d(ks + sl * (kBN * 128), mk, k_full + s, sl * 64, e.kh, key, pol);
+              // keep kPrefetch further prefix tiles on their way into L2: two
+              // shared stages alone hold too few bytes in flight for HBM latency
+              for (int jp = (jk == 0 ? 1 : jk + kPrefetch); jp <= jk + kPrefetch && jp < e.npt;
+                   ++jp) {
+                const int kp = e.p0 + e.k_begin + jp * kBN;
+#pragma unroll
+                for (int sl = 0; sl < G::kSlices; ++sl) {
+                  tma_prefetch_3d(&tmK, sl * 64, e.kh, kp);
+                  tma_prefetch_3d(&tmV, sl * 64, e.kh, kp);
+                }
+              }
+              k_issued |= 1u << s;
+              k_par = (k_par & ~(1u << s)) | (ph << s);
+              ++jk;
+              progressed = true;
+            }
+          }
+          if (jv < jk) {
+            const int T = Tv + jv;
+            const int s = T % kStages;
+            const uint32_t ph = (T / kStages) & 1;
+            if (mbar_test(v_empty + s, ph ^ 1u)) {
+              uint8_t* vs = smem + G::kOffK + s * 2 * G::kKVBytes + G::kKVBytes;
+              mbar_arrive_expect_tx(v_full + s, G::kKVBytes);
+              const bool pre = jv < e.npt;
+              const CUtensorMap* mv = pre ? &tmV : &tmVc;
+              const int key = pre ? e.p0 + e.k_begin + jv * kBN : e.f_begin + (jv - e.npt) * kBN;
+#pragma unroll
+              for (int sl = 0; sl < G::kSlices; ++sl)
+                tma_load_3d(vs + sl * (kBN * 128), mv, v_full + s, sl * 64, e.kh, key, pol);
+              v_issued |= 1u << s;
+              v_par = (v_par & ~(1u << s)) | (ph << s);
+              ++jv;
+              progressed = true;
+            }
+          }
+          const uint64_t now = global_timer_ns();
+          if (progressed) {
+            t_last = now;
+          } else if (*abort_flag || now - t_last > kWaitNs) {
+            ok = false;
+            break;
+          }
+        }
+        Tk += e.ntiles;
+        Tv += e.ntiles;
+        ++v;
       }
       if (!ok) {
         *abort_flag = 1;
         flag(a.status, JET_ERR_TIMEOUT);
         // let every copy already issued land before the CTA can exit
+        if (q_issued) mbar_wait(q_full, q_par, kDrainNs, nullptr);
         for (int t = 0; t < kStages; ++t) {
           if (k_issued & (1u << t)) mbar_wait(k_full + t, (k_par >> t) & 1u, kDrainNs, nullptr);
           if (v_issued & (1u << t)) mbar_wait(v_full + t, (v_par >> t) & 1u, kDrainNs, nullptr);
@@ -334,54 +485,79 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       const uint32_t id_s = idesc_bf16_f32(kBV, kBN);
       const uint32_t id_o = idesc_bf16_f32(kBV, DH) | (1u << 16);  // B (V) is MN-major
       const uint32_t qs = smem_u32(smem);
-      bool ok = mbar_wait(q_full, 0, kWaitNs, abort_flag);
-      tc_fence_after();
-      // issue S_j = Q K_j^T and O += P_j V_j in whichever order their inputs
-      // become ready; S_j always precedes P_j V_j
-      int js = 0, jo = 0;
-      uint64_t t_last = global_timer_ns();
-      while (ok && jo < ntiles) {
-        bool progressed = false;
-        if (js < ntiles) {
-          const int s = js % kStages, b = js & 1;
-          if (mbar_test(k_full + s, (js / kStages) & 1) &&
-              mbar_test(s_free + b, ((js >> 1) & 1) ^ 1u)) {
-            tc_fence_after();
-            const uint32_t ks = smem_u32(smem + G::kOffK + s * 2 * G::kKVBytes);
-#pragma unroll
-            for (int st = 0; st < DH / 16; ++st) {
-              const int sl = st >> 2, k = st & 3;
-              mma_f16(tmem + b * kBN, desc_k_sw128(qs + sl * (kBV * 128) + 32 * k),
-                      desc_k_sw128(ks + sl * (kBN * 128) + 32 * k), id_s, st != 0);
-            }
-            mma_commit(s_full + b);
-            mma_commit(k_empty + s);
-            ++js;
-            progressed = true;
-          }
-        }
-        if (jo < js) {
-          const int s = jo % kStages, b = jo & 1;
-          if (mbar_test(p_full + b, (jo >> 1) & 1) && mbar_test(v_full + s, (jo / kStages) & 1)) {
-            tc_fence_after();
-            const uint32_t ps = smem_u32(smem + G::kOffP + b * G::kPBytes);
-            const uint32_t vs = smem_u32(smem + G::kOffK + s * 2 * G::kKVBytes + G::kKVBytes);
-#pragma unroll
-            for (int k = 0; k < kBN / 16; ++k)
-              mma_f16(tmem + G::kOCol, desc_k_sw128(ps + 32 * k),
-                      desc_mn_sw128(vs + k * 16 * 128, kBN * 128), id_o, (jo | k) != 0);
-            mma_commit(p_free + b);
-            mma_commit(v_empty + s);
-            ++jo;
-            progressed = true;
-          }
-        }
-        const uint64_t now = global_timer_ns();
-        if (progressed) {
-          t_last = now;
-        } else if (*abort_flag || now - t_last > kWaitNs) {
+      bool ok = mbar_wait(qz_done, 0, kWaitNs, abort_flag);
+      int T = 0, v = 0;  // tiles and items processed so far
+      for (int u = 0; ok; ++u) {
+        const int slot = u & 1;
+        if (!mbar_wait(item_full + slot, (u >> 1) & 1, kWaitNs, abort_flag)) {
           ok = false;
+          break;
         }
+        const int4 it = ring[slot];
+        mbar_arrive(item_empty + slot);
+        if (it.x < 0) break;
+        const ItemGeo e = item_geo(a, it);
+        if (!e.ok) continue;
+        if (!mbar_wait(q_full, v & 1, kWaitNs, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        // issue S_j = Q K_j^T and O += P_j V_j in whichever order their inputs
+        // become ready; S_j always precedes P_j V_j
+        int js = 0, jo = 0;
+        uint64_t t_last = global_timer_ns();
+        while (ok && jo < e.ntiles) {
+          bool progressed = false;
+          if (js < e.ntiles) {
+            const int Tj = T + js;
+            const int s = Tj % kStages, b = Tj & 1;
+            if (mbar_test(k_full + s, (Tj / kStages) & 1) &&
+                mbar_test(s_free + b, ((Tj >> 1) & 1) ^ 1u)) {
+              tc_fence_after();
+              const uint32_t ks = smem_u32(smem + G::kOffK + s * 2 * G::kKVBytes);
+#pragma unroll
+              for (int st = 0; st < DH / 16; ++st) {
+                const int sl = st >> 2, k = st & 3;
+                mma_f16(tmem + b * kBN, desc_k_sw128(qs + sl * (kBV * 128) + 32 * k),
+                        desc_k_sw128(ks + sl * (kBN * 128) + 32 * k), id_s, st != 0);
+              }
+              mma_commit(s_full + b);
+              mma_commit(k_empty + s);
+              if (js == e.ntiles - 1) mma_commit(q_free);  // the query block may be replaced
+              ++js;
+              progressed = true;
+            }
+          }
+          if (jo < js) {
+            const int Tj = T + jo;
+            const int s = Tj % kStages, b = Tj & 1;
+            // the item's first P V overwrites O: the previous item's O must be out
+            const bool o_ready = jo > 0 || v == 0 || mbar_test(o_free, (v - 1) & 1);
+            if (o_ready && mbar_test(p_full + b, (Tj >> 1) & 1) &&
+                mbar_test(v_full + s, (Tj / kStages) & 1)) {
+              tc_fence_after();
+              const uint32_t ps = smem_u32(smem + G::kOffP + b * G::kPBytes);
+              const uint32_t vs = smem_u32(smem + G::kOffK + s * 2 * G::kKVBytes + G::kKVBytes);
+#pragma unroll
+              for (int k = 0; k < kBN / 16; ++k)
+                mma_f16(tmem + G::kOCol, desc_k_sw128(ps + 32 * k),
+                        desc_mn_sw128(vs + k * 16 * 128, kBN * 128), id_o, (jo | k) != 0);
+              mma_commit(p_free + b);
+              mma_commit(v_empty + s);
+              ++jo;
+              progressed = true;
+            }
+          }
+          const uint64_t now = global_timer_ns();
+          if (progressed) {
+            t_last = now;
+          } else if (*abort_flag || now - t_last > kWaitNs) {
+            ok = false;
+          }
+        }
+        T += e.ntiles;
+        ++v;
       }
       if (!ok) {
         *abort_flag = 1;
@@ -395,132 +571,147 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
     const int q4 = warp & 3;
     const int i = q4 * 32 + lane;  // query vector within the block = TMEM lane
     const uint32_t lane_off = uint32_t(q4 * 32) << 16;
-    const bool valid = i < nv;
-    int n = 0, h = 0;
-    int fa = 1, fb = 0;  // fed-token indices this vector may see (none: shared row)
-    if (valid) {
-      const int gv = vbase + i;
-      n = n0 + gv / g;
-      h = kh * g + gv % g;
-      const int c = a.row_cand[n];
-      if (c >= 0 && c < a.C) {
-        fa = a.cand_row_offset[c] - r - 1;  // y_{c,1}
-        fb = n - r - 1;                     // the row's own fed token, inclusive
-      }
-    }
-    // the query block arrives by TMA (rows [0, rb g)); zero the rows past it
-    // so that no stale shared memory enters the MMA
-    {
-      if (i >= rb * g) {
+    // the query blocks arrive by TMA (rows [0, rb g)); zero the rows past them
+    // once so that no stale shared memory enters the MMA
+    if (i >= rb * g) {
 #pragma unroll
-        for (int c = 0; c < DH / 8; ++c)
-          *reinterpret_cast<uint4*>(smem + (c >> 3) * (kBV * 128) + sw128(i, c & 7)) =
-              make_uint4(0, 0, 0, 0);
-      }
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(q_full);
+      for (int c = 0; c < DH / 8; ++c)
+        *reinterpret_cast<uint4*>(smem + (c >> 3) * (kBV * 128) + sw128(i, c & 7)) =
+            make_uint4(0, 0, 0, 0);
     }
-    float m_used = -INFINITY, l = 0.f;
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(qz_done);
+
     bool ok = true;
-    for (int j = 0; j < ntiles; ++j) {
-      const int b = j & 1;
-      if (!warp_mbar_wait(s_full + b, (j >> 1) & 1, kWaitNs, abort_flag)) {
+    int T = 0;
+    for (int u = 0; ok; ++u) {
+      const int slot = u & 1;
+      if (!warp_mbar_wait(item_full + slot, (u >> 1) & 1, kWaitNs, abort_flag)) {
         ok = false;
         break;
       }
-      tc_fence_after();
-      float sv[kBN];
-      {
-        float t0[32], t1[32];
-        tmem_ld_32cols(tmem + lane_off + b * kBN, t0);
-        tmem_ld_32cols(tmem + lane_off + b * kBN + 32, t1);
-        tmem_wait_ld();
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          sv[c] = t0[c];
-          sv[c + 32] = t1[c];
+      const int4 it = ring[slot];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(item_empty + slot);
+      if (it.x < 0) break;
+      const ItemGeo e = item_geo(a, it);
+      if (!e.ok) continue;
+      const bool valid = i < e.nv;
+      int n = 0, h = 0;
+      int fa = 1, fb = 0;  // fed-token indices this vector may see (none: shared row)
+      if (valid) {
+        const int gv = e.vbase + i;
+        n = e.n0 + gv / g;
+        h = e.kh * g + gv % g;
+        const int c = a.row_cand[n];
+        if (c >= 0 && c < a.C) {
+          fa = a.cand_row_offset[c] - e.r - 1;  // y_{c,1}
+          fb = n - e.r - 1;                     // the row's own fed token, inclusive
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(s_free + b);
-      // visible keys of this tile: [klo, khi) of its 64 slots
-      int klo = 0, khi;
-      if (j < npt) {
-        khi = min(kBN, k_end - (k_begin + j * kBN));
-      } else {
-        const int f0 = f_begin + (j - npt) * kBN;
-        klo = max(0, fa - f0);
-        khi = min(kBN, fb - f0 + 1);
-      }
-      float mt = -INFINITY;
+      float m_used = -INFINITY, l = 0.f;
+      for (int j = 0; j < e.ntiles; ++j) {
+        const int Tj = T + j;
+        const int b = Tj & 1;
+        if (!warp_mbar_wait(s_full + b, (Tj >> 1) & 1, kWaitNs, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        float sv[kBN];
+        {
+          float t0[32], t1[32];
+          tmem_ld_32cols(tmem + lane_off + b * kBN, t0);
+          tmem_ld_32cols(tmem + lane_off + b * kBN + 32, t1);
+          tmem_wait_ld();
 #pragma unroll
-      for (int c = 0; c < kBN; ++c) {
-        sv[c] = (c >= klo && c < khi) ? sv[c] * a.scale_log2 : -INFINITY;
-        mt = fmaxf(mt, sv[c]);
-      }
-      // P_j reuses buffer b: PV_{j-2} must be done reading it
-      if (j >= 2 && !warp_mbar_wait(p_free + b, ((j - 2) >> 1) & 1, kWaitNs, abort_flag)) {
-        ok = false;
-        break;
-      }
-      if (mt > m_used + kRescaleLog2) {
-        const float m_new = mt;
-        if (j >= 1) {
-          // O holds PV_0 .. PV_{j-1}: wait for PV_{j-1}, then rescale it in TMEM
-          if (!warp_mbar_wait(p_free + ((j - 1) & 1), ((j - 1) >> 1) & 1, kWaitNs, abort_flag)) {
-            ok = false;
-            break;
+          for (int c = 0; c < 32; ++c) {
+            sv[c] = t0[c];
+            sv[c + 32] = t1[c];
           }
-          tc_fence_after();
-          const float f = ex2(m_used - m_new);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(s_free + b);
+        // visible keys of this tile: [klo, khi) of its 64 slots
+        int klo = 0, khi;
+        if (j < e.npt) {
+          khi = min(kBN, e.k_end - (e.k_begin + j * kBN));
+        } else {
+          const int f0 = e.f_begin + (j - e.npt) * kBN;
+          klo = max(0, fa - f0);
+          khi = min(kBN, fb - f0 + 1);
+        }
+        float mt = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < kBN; ++c) {
+          sv[c] = (c >= klo && c < khi) ? sv[c] * a.scale_log2 : -INFINITY;
+          mt = fmaxf(mt, sv[c]);
+        }
+        // P buffer b was last read by the P V of tile Tj - 2
+        if (Tj >= 2 && !warp_mbar_wait(p_free + b, ((Tj - 2) >> 1) & 1, kWaitNs, abort_flag)) {
+          ok = false;
+          break;
+        }
+        if (mt > m_used + kRescaleLog2) {
+          const float m_new = mt;
+          if (j >= 1) {
+            // O holds this item's P V so far: wait for the last one, rescale in TMEM
+            if (!warp_mbar_wait(p_free + ((Tj - 1) & 1), ((Tj - 1) >> 1) & 1, kWaitNs,
+                                abort_flag)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const float f = ex2(m_used - m_new);
 #pragma unroll 1
-          for (int c0 = 0; c0 < DH; c0 += 32) {
-            float ov[32];
-            tmem_ld_32cols(tmem + lane_off + G::kOCol + c0, ov);
-            tmem_wait_ld();
+            for (int c0 = 0; c0 < DH; c0 += 32) {
+              float ov[32];
+              tmem_ld_32cols(tmem + lane_off + G::kOCol + c0, ov);
+              tmem_wait_ld();
 #pragma unroll
-            for (int c = 0; c < 32; ++c) ov[c] *= f;
-            tmem_st_32cols(tmem + lane_off + G::kOCol + c0, ov);
+              for (int c = 0; c < 32; ++c) ov[c] *= f;
+              tmem_st_32cols(tmem + lane_off + G::kOCol + c0, ov);
+            }
+            tmem_wait_st();
+            l *= f;
           }
-          tmem_wait_st();
-          l *= f;
+          m_used = m_new;
         }
-        m_used = m_new;
-      }
-      // P_j = 2^(s - m_used) as bf16, 128-byte swizzled; the row sum uses the
-      // rounded values, which are what the tensor core multiplies
-      uint8_t* pb = smem + G::kOffP + b * G::kPBytes;
-      float psum = 0.f;
+        // P = 2^(s - m_used) as bf16, 128-byte swizzled; the row sum uses the
+        // rounded values, which are what the tensor core multiplies
+        uint8_t* pb = smem + G::kOffP + b * G::kPBytes;
+        float psum = 0.f;
 #pragma unroll
-      for (int cc = 0; cc < 8; ++cc) {
-        uint32_t w[4];
+        for (int cc = 0; cc < 8; ++cc) {
+          uint32_t w[4];
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float x0 = ex2(sv[cc * 8 + 2 * e] - m_used);
-          const float x1 = ex2(sv[cc * 8 + 2 * e + 1] - m_used);
-          w[e] = pack_bf16(x0, x1);
-          const __nv_bfloat162 hb = *reinterpret_cast<const __nv_bfloat162*>(&w[e]);
-          psum += __bfloat162float(hb.x) + __bfloat162float(hb.y);
+          for (int q = 0; q < 4; ++q) {
+            const float x0 = ex2(sv[cc * 8 + 2 * q] - m_used);
+            const float x1 = ex2(sv[cc * 8 + 2 * q + 1] - m_used);
+            w[q] = pack_bf16(x0, x1);
+            const __nv_bfloat162 hb = *reinterpret_cast<const __nv_bfloat162*>(&w[q]);
+            psum += __bfloat162float(hb.x) + __bfloat162float(hb.y);
+          }
+          *reinterpret_cast<uint4*>(pb + sw128(i, cc)) = make_uint4(w[0], w[1], w[2], w[3]);
         }
-        *reinterpret_cast<uint4*>(pb + sw128(i, cc)) = make_uint4(w[0], w[1], w[2], w[3]);
+        l += psum;
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(p_full + b);
       }
-      l += psum;
-      fence_proxy_async_smem();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(p_full + b);
-    }
-    // wait for the last PV, then write the partial
-    if (ok) {
-      const int jl = ntiles - 1;
-      ok = warp_mbar_wait(p_free + (jl & 1), (jl >> 1) & 1, kWaitNs, abort_flag);
-    }
-    if (ok) {
+      if (!ok) break;
+      // wait for the item's last P V, then write its output (or its partial)
+      const int Tl = T + e.ntiles - 1;
+      if (!warp_mbar_wait(p_free + (Tl & 1), (Tl >> 1) & 1, kWaitNs, abort_flag)) {
+        ok = false;
+        break;
+      }
       tc_fence_after();
-      const size_t base = (size_t(split) * a.N + n) * a.Hq + h;
-      const bool direct = splits_r == 1;  // the whole row in this CTA: final output
+      const size_t base = (size_t(e.split) * a.N + n) * a.Hq + h;
+      const bool direct = e.splits_r == 1;  // the whole row in this item: final output
       const float inv = l > 0.f ? 1.f / l : 0.f;
 #pragma unroll 1
       for (int c0 = 0; c0 < DH; c0 += 32) {
@@ -543,7 +734,13 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         }
       }
       if (valid && !direct) a.ml_part[base] = make_float2(m_used, l);
-    } else {
+      // O may be overwritten by the next item's first P V
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(o_free);
+      T += e.ntiles;
+    }
+    if (!ok) {
       *abort_flag = 1;
       flag(a.status, JET_ERR_TIMEOUT);
     }
@@ -655,6 +852,7 @@ cudaError_t launch_dh(const jet_layout& lay, const jet_dims& d, const AttnPlan& 
   AttArgs a{};
   a.prefix_offset = lay.prefix_offset;
   a.row_offset = lay.row_offset;
+  a.req_order = lay.req_order;
   a.row_cand = lay.row_cand;
   a.cand_row_offset = lay.cand_row_offset;
   a.q = static_cast<const __nv_bfloat16*>(q);
@@ -669,13 +867,40 @@ cudaError_t launch_dh(const jet_layout& lay, const jet_dims& d, const AttnPlan& 
   a.Hq = d.Hq;
   a.Hkv = d.Hkv;
   a.chunk = plan.chunk;
+  a.g = g;
+  a.rb = kBV / g;
   a.has_cand = F > 0;
   a.scale_log2 = 1.4426950408889634f / sqrtf(float(DH));
-  const size_t smem = Geo<DH>::kBytes + 1024;
-  cudaError_t e = cudaFuncSetAttribute(attend_prefix_tc_kernel<DH>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  // the work list follows the (m, l) partials in the workspace
+  const size_t vecs = size_t(plan.splits) * n.N * d.Hq;
+  uintptr_t ctrl = reinterpret_cast<uintptr_t>(ml_part + vecs);
+  ctrl = (ctrl + 15) & ~uintptr_t(15);
+  a.item_next = reinterpret_cast<int*>(ctrl);
+  a.item_count = a.item_next + 1;
+  a.items = reinterpret_cast<int4*>(ctrl + 16);
+  a.splits = plan.splits;
+  a.n_all = (long long)n.R * d.Hkv * plan.qgroups * plan.splits;
+  // longest-first dynamic order pays for its extra launch only when items are
+  // long and uneven (chunks of 16 key tiles or more)
+  a.sorted = plan.chunk >= 16 * kBN;
+  cudaError_t e = cudaSuccess;
+  if (a.sorted) {
+    attend_items_kernel<<<1, 1024, 0, st>>>(a, plan.qgroups, plan.splits);
+    e = cudaGetLastError();
+  } else {
+    e = cudaMemsetAsync(a.item_next, 0, sizeof(int), st);  // the shared slot counter
+  }
   if (e != cudaSuccess) return e;
-  dim3 grid(plan.splits, unsigned(n.R * d.Hkv), plan.qgroups);
+  const size_t smem = Geo<DH>::kBytes + 1024;
+  e = cudaFuncSetAttribute(attend_prefix_tc_kernel<DH>,
+                           cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  if (e != cudaSuccess) return e;
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+    return cudaErrorInvalidValue;
+  const long long max_items = (long long)n.R * d.Hkv * plan.qgroups * plan.splits;
+  const int grid = int(std::max<long long>(1, std::min<long long>(sms, max_items)));
   attend_prefix_tc_kernel<DH><<<grid, kThreads, smem, st>>>(tmQ, tmK, tmV, tmKc, tmVc, a);
   e = cudaGetLastError();
   if (e != cudaSuccess || plan.splits <= 1) return e;

@@ -5,6 +5,7 @@
 // request r's first row is its last prefix position and predicts y_{c,1} for
 // every candidate (Sec. 4.1); the row fed with y_{c,t} predicts y_{c,t+1}
 // (Eq. 1 conditions z_{c,t,.} on (x, y_{c,<t})). Pure host code: no CUDA call.
+#include <algorithm>
 #include <climits>
 #include <cstring>
 #include <vector>
@@ -16,15 +17,15 @@ namespace {
 inline size_t pad4(size_t x) { return (x + 3) & ~size_t(3); }
 
 // word offsets of the 12 arrays, plus the total, in the order of jet_layout
-void word_offsets(const jet_sizes& n, size_t off[13]) {
+void word_offsets(const jet_sizes& n, size_t off[14]) {
   const size_t R = size_t(n.R), C = size_t(n.C), N = size_t(n.N), T = size_t(n.T);
-  const size_t len[12] = {R + 1, R + 1, R + 1, C + 1, C + 1, T, T, N, N, N, N + 1, T};
+  const size_t len[13] = {R + 1, R + 1, R + 1, C + 1, C + 1, T, T, N, N, N, N + 1, T, R};
   size_t o = 0;
-  for (int i = 0; i < 12; ++i) {
+  for (int i = 0; i < 13; ++i) {
     off[i] = o;
     o += pad4(len[i]);
   }
-  off[12] = o;
+  off[13] = o;
 }
 
 }  // namespace
@@ -72,22 +73,23 @@ extern "C" jet_status jet_layout_plan(int32_t R, const int32_t* prefix_len, cons
 
 extern "C" size_t jet_layout_words(const jet_sizes* n) {
   if (!n || n->R < 0 || n->C < 0 || n->N < 0 || n->T < 0) return 0;
-  size_t off[13];
+  size_t off[14];
   word_offsets(*n, off);
-  return off[12];
+  return off[13];
 }
 
 extern "C" jet_status jet_layout_bind(const jet_sizes* n, const int32_t* words, jet_layout* out) {
   if (!n || !out || (!words && jet_layout_words(n) > 0)) return JET_ERR_ARG;
   if (n->R < 0 || n->C < 0 || n->N < 0 || n->T < 0) return JET_ERR_SHAPE;
-  size_t off[13];
+  size_t off[14];
   word_offsets(*n, off);
   out->n = *n;
-  const int32_t** slots[12] = {&out->prefix_offset, &out->cand_offset,  &out->row_offset,
+  const int32_t** slots[13] = {&out->prefix_offset, &out->cand_offset,  &out->row_offset,
                                &out->cand_row_offset, &out->tgt_offset, &out->target_ids,
                                &out->tgt_row,       &out->row_req,      &out->row_cand,
-                               &out->row_pos,       &out->row_tgt_offset, &out->row_tgt_index};
-  for (int i = 0; i < 12; ++i) *slots[i] = words + off[i];
+                               &out->row_pos,       &out->row_tgt_offset, &out->row_tgt_index,
+                               &out->req_order};
+  for (int i = 0; i < 13; ++i) *slots[i] = words + off[i];
   return JET_OK;
 }
 
@@ -105,7 +107,7 @@ extern "C" jet_status jet_layout_build(int32_t R, const int32_t* prefix_len, con
   if (need > 0 && (!words || n_words < need)) return JET_ERR_WORKSPACE;
   std::memset(words, 0, need * sizeof(int32_t));
   jet_layout_bind(&n, words, out);
-  size_t off[13];
+  size_t off[14];
   word_offsets(n, off);
   int32_t* prefix_offset = words + off[0];
   int32_t* cand_offset = words + off[1];
@@ -119,6 +121,7 @@ extern "C" jet_status jet_layout_build(int32_t R, const int32_t* prefix_len, con
   int32_t* row_pos = words + off[9];
   int32_t* row_tgt_offset = words + off[10];
   int32_t* row_tgt_index = words + off[11];
+  int32_t* req_order = words + off[12];
 
   int32_t row = 0, c = 0, j = 0;
   prefix_offset[0] = 0;
@@ -159,5 +162,11 @@ extern "C" jet_status jet_layout_build(int32_t R, const int32_t* prefix_len, con
   for (int32_t r = 0; r < n.N; ++r) row_tgt_offset[r + 1] = row_tgt_offset[r] + count[size_t(r) + 1];
   std::vector<int32_t> fill(row_tgt_offset, row_tgt_offset + n.N);
   for (int32_t t = 0; t < n.T; ++t) row_tgt_index[fill[size_t(tgt_row[t])]++] = t;
+
+  // requests by decreasing prefix length (ties: lower index first); kernels
+  // hand out long prefixes first so that their work balances across SMs
+  for (int32_t r = 0; r < R; ++r) req_order[r] = r;
+  std::stable_sort(req_order, req_order + R,
+                   [&](int32_t x, int32_t y) { return prefix_len[x] > prefix_len[y]; });
   return JET_OK;
 }

@@ -47,7 +47,7 @@ class jet_sizes(ctypes.Structure):
 
 _ARRAYS = ("prefix_offset", "cand_offset", "row_offset", "cand_row_offset", "tgt_offset",
            "target_ids", "tgt_row", "row_req", "row_cand", "row_pos", "row_tgt_offset",
-           "row_tgt_index")
+           "row_tgt_index", "req_order")
 
 
 class jet_layout(ctypes.Structure):
@@ -152,7 +152,7 @@ class HostLayout:
         lens = {"prefix_offset": n.R + 1, "cand_offset": n.R + 1, "row_offset": n.R + 1,
                 "cand_row_offset": n.C + 1, "tgt_offset": n.C + 1, "target_ids": n.T,
                 "tgt_row": n.T, "row_req": n.N, "row_cand": n.N, "row_pos": n.N,
-                "row_tgt_offset": n.N + 1, "row_tgt_index": n.T}
+                "row_tgt_offset": n.N + 1, "row_tgt_index": n.T, "req_order": n.R}
         off = (getattr(self.struct, name) - self.words.ctypes.data) // 4
         return self.words[off:off + lens[name]].copy()
 

@@ -43,6 +43,9 @@ def _compare(jet, prefix_len, n_cand, cand_len, ids, V):
         got = lay.array(f)
         assert got.dtype == np.int32
         np.testing.assert_array_equal(got, ref[f], err_msg=f)
+    # scheduling order: the requests by decreasing prefix length, ties in index order
+    order = lay.array("req_order")
+    np.testing.assert_array_equal(order, np.argsort(-np.asarray(prefix_len), kind="stable"))
 
 
 def test_layout_matches_oracle_golden(jet):
