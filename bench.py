@@ -219,6 +219,21 @@ def _attend_launches(problem, w) -> int:
     return 1 + (1 if splits > 1 else 0)
 
 
+def aggregate(total_ms: float, e2e_ms: float, R: int, steps: int, world: int, device=None):
+    """Whole-job numbers of N independent replicas: the slowest rank's timed
+    regions (max over ranks) and the sets all ranks scored per second.
+    Returns (total_ms, e2e_ms, ms_per_step, sets_per_s, e2e_sets_per_s)."""
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        t = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms, e2e_ms = float(t[0]), float(t[1])
+    ms_per_step = total_ms / steps
+    return (total_ms, e2e_ms, ms_per_step, R * world / (ms_per_step / 1e3),
+            R * world / (e2e_ms / 1e3))
+
+
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -342,14 +357,8 @@ def run_gpu(args):
     h2d, d2h = step.host_bytes(host, words)
     assert jet.jet_device_status(stream) == 0
 
-    if world > 1:
-        t = torch.tensor([total_ms, e2e_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms, e2e_ms = float(t[0]), float(t[1])
-
-    ms_per_step = total_ms / args.steps
-    value = R * world / (ms_per_step / 1e3)
-    e2e_value = R * world / (e2e_ms / 1e3)
+    total_ms, e2e_ms, ms_per_step, value, e2e_value = aggregate(
+        total_ms, e2e_ms, R, args.steps, world, device=dev)
 
     # --- roofline of the dominant kernel (the LM head) ----------------------
     peaks = _peaks()
