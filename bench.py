@@ -48,8 +48,9 @@ def _peaks():
             p = json.load(f)
         return dict(hbm=float(p["hbm_gbs"]), bf16=float(p["bf16_tflops"]),
                     bf16_sustained=float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
-                    source="measured")
-    return dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, source="fallback")
+                    sm_max_mhz=float(p.get("sm_max_mhz", 2070.0)), source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, sm_max_mhz=2070.0,
+                source="fallback")
 
 
 # ---------------------------------------------------------------------------
@@ -374,8 +375,12 @@ def run_gpu(args):
         else "paper_2609_33874_gb300/csrc/lmhead_simt.cu"
     traffic = _traffic(kernel_file, args.workload)
     if w.dtype != "bf16":
-        roof = dict(bound="alu", achieved=lm_flops / score_avg_s / 1e12, peak=None, unit="TFLOP/s",
-                    frac=None, traffic=traffic)
+        # float32 FMA: SMs x 128 lanes x 2 flop x the maximum SM clock
+        sms = torch.cuda.get_device_properties(dev).multi_processor_count
+        alu_peak = sms * 128 * 2 * peaks["sm_max_mhz"] * 1e6 / 1e12
+        ach = lm_flops / score_avg_s / 1e12
+        roof = dict(bound="alu", achieved=round(ach, 3), peak=round(alu_peak, 1), unit="TFLOP/s",
+                    frac=round(ach / alu_peak, 4), traffic=traffic)
     elif lm_flops / lm_bytes < ridge:
         ach = lm_bytes / score_avg_s / 1e9
         roof = dict(bound="hbm", achieved=round(ach, 1), peak=peaks["hbm"], unit="GB/s",
