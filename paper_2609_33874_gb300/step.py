@@ -5,7 +5,8 @@ outputs and workspace) and strings the C entry points together on one CUDA
 stream. Inputs are torch tensors already on the device (:meth:`run`) or pinned
 host tensors that are copied in first (:meth:`run_from_host`, the end-to-end
 path: host -> device copies, the kernels, device -> host copies of the
-results).
+results; :meth:`run_pipelined` does the same over a sequence of batches and
+overlaps each batch's input copies with the previous batch's kernels).
 """
 from __future__ import annotations
 
@@ -21,6 +22,9 @@ _TORCH_DTYPE = {jet.DTYPE_F32: torch.float32, jet.DTYPE_BF16: torch.bfloat16}
 ATTN_INPUTS = ("q", "k_pre", "v_pre", "k_cand", "v_cand")
 FORK_INPUTS = ("s_prefix", "lq", "lk", "lv", "alpha", "beta")
 RESULTS = ("tok_logprob", "cand_score", "q_cand", "choice", "value")
+# below this many input bytes per batch (about 5 us over the host link)
+# run_pipelined copies on the compute stream instead of overlapping
+_OVERLAP_MIN_BYTES = 1 << 20
 
 
 class ScoringStep:
@@ -59,15 +63,19 @@ class ScoringStep:
             self.lo = z(self.F, dims.Hl, dims.dv, dtype=dt)
             self.s_fork = z(n.C, dims.Hl, dims.dk, dims.dv) if keep_fork_state else None
         self._dev_inputs: Optional[Dict[str, torch.Tensor]] = None
+        self.overlap_min_bytes = _OVERLAP_MIN_BYTES
 
     # ------------------------------------------------------------------
-    def run(self, x: Dict[str, torch.Tensor], w_lm: torch.Tensor, stream=None) -> None:
+    def run(self, x: Dict[str, torch.Tensor], w_lm: torch.Tensor, stream=None,
+            layout: Optional["jet.DeviceLayout"] = None) -> None:
         """Enqueue the whole step on ``stream`` (default: the current stream).
 
         ``x`` holds q, k_pre, v_pre, k_cand, v_cand, hidden (unless chained)
-        and, for a hybrid step, s_prefix, lq, lk, lv, alpha, beta.
+        and, for a hybrid step, s_prefix, lq, lk, lv, alpha, beta. ``layout``
+        (default: the step's own) must have this step's sizes.
         """
-        d, lay = self.dims, self.layout
+        d = self.dims
+        lay = self.layout if layout is None else layout
         jet.jet_prefix_attend(lay, d, x["q"], x["k_pre"], x["v_pre"], x["k_cand"], x["v_cand"],
                               self.o, self.ws, stream=stream)
         if self.hybrid:
@@ -100,6 +108,50 @@ class ScoringStep:
             self.run(self._dev_inputs, w_lm, stream=s)
             for k in RESULTS:
                 out[k].copy_(getattr(self, k), non_blocking=True)
+
+    def run_pipelined(self, batches, w_lm: torch.Tensor, outs, stream=None) -> None:
+        """End to end over a sequence of batches of this step's shape: the
+        host -> device copies of batch i+1 run on a copy stream while the
+        kernels of batch i run on ``stream``; device inputs and layouts are
+        double-buffered. ``batches`` yields (pinned host inputs, pinned layout
+        words); ``outs[i]`` receives batch i's results (device -> host, on
+        ``stream``). Everything is enqueued; the caller synchronises."""
+        s = torch.cuda.current_stream(self.dev) if stream is None else stream
+        if getattr(self, "_pipe", None) is None:
+            self._copy_stream = torch.cuda.Stream(self.dev)
+            self._pipe = []
+            for _ in range(2):
+                words = torch.empty_like(self.layout.words)
+                self._pipe.append(dict(
+                    layout=jet.DeviceLayout(self.layout.sizes, words), inputs=None,
+                    copied=torch.cuda.Event(), consumed=torch.cuda.Event()))
+        cs = self._copy_stream
+        start = torch.cuda.Event()
+        start.record(s)
+        cs.wait_event(start)  # after everything already enqueued on ``stream``
+        for i, (host, layout_words) in enumerate(batches):
+            buf = self._pipe[i % 2]
+            # a batch whose copies take a few microseconds gains nothing from
+            # the overlap and would pay the two cross-stream waits: copy in order
+            overlap = self.host_bytes(host, layout_words)[0] >= self.overlap_min_bytes
+            with torch.cuda.stream(cs if overlap else s):
+                if overlap and i >= 2:
+                    cs.wait_event(buf["consumed"])  # batch i-2's kernels are done with it
+                if buf["inputs"] is None:
+                    buf["inputs"] = {k: torch.empty_like(host[k], device=self.dev)
+                                     for k in self.input_names()}
+                buf["layout"].words.copy_(layout_words, non_blocking=True)
+                for k in self.input_names():
+                    buf["inputs"][k].copy_(host[k], non_blocking=True)
+                if overlap:
+                    buf["copied"].record(cs)
+            if overlap:
+                s.wait_event(buf["copied"])
+            self.run(buf["inputs"], w_lm, stream=s, layout=buf["layout"])
+            buf["consumed"].record(s)
+            with torch.cuda.stream(s):
+                for k in RESULTS:
+                    outs[i][k].copy_(getattr(self, k), non_blocking=True)
 
     def host_bytes(self, host: Dict[str, torch.Tensor], layout_words: torch.Tensor):
         """(host->device, device->host) bytes one :meth:`run_from_host` moves."""

@@ -55,11 +55,11 @@ def oracle_layout(problem):
                           problem.target_ids, problem.work.V)
 
 
-def check_scores(lay, problem, got, requests, hidden=None):
+def check_scores(lay, problem, got, requests, hidden=None, w_lm=None):
     """Oracle l, s and decisions for the given requests; compare with `got`."""
     w = problem.work
     H = problem.f32("hidden") if hidden is None else hidden
-    W = problem.f32("w_lm")
+    W = problem.f32("w_lm") if w_lm is None else w_lm
     tg = []
     cands = []
     for r in requests:

@@ -217,3 +217,35 @@ def test_end_to_end_from_host(cuda):
     check_scores(lay, p, got, [0])
     h2d, d2h = step.host_bytes(host, words)
     assert h2d > 0 and d2h > 0
+
+
+@pytest.mark.parametrize("overlap", [True, False])
+def test_end_to_end_pipelined(cuda, overlap):
+    """Four batches of one shape with their own hidden states and targets,
+    copied in on the copy stream while the previous batch computes (or in
+    order on the compute stream): each batch's results must be its own (the
+    double buffers are reused from the third batch on)."""
+    import torch
+    p0 = jet_synth.make_problem("tiny")
+    rng = np.random.default_rng(7)
+    probs = [jet_synth.custom_problem(p0.work, p0.prefix_len, p0.n_cand, p0.cand_len,
+                                      rng.integers(0, p0.work.V, size=len(p0.target_ids)),
+                                      seed=1000 + i) for i in range(4)]
+    step, _, w_lm = build_step(cuda, p0)
+    step.overlap_min_bytes = 0 if overlap else 1 << 40
+    batches, outs = [], []
+    for p in probs:
+        hl = cuda.jet_layout_build(p.prefix_len, p.n_cand, p.cand_len, p.target_ids, p.work.V)
+        host = {k: jet_synth.torch_tensor(p, k, pin=True) for k in step.input_names()}
+        batches.append((host, torch.from_numpy(hl.words).pin_memory()))
+        outs.append({k: torch.empty_like(getattr(step, k), device="cpu").pin_memory()
+                     for k in ("tok_logprob", "cand_score", "q_cand", "choice", "value")})
+    step.run_pipelined(batches, w_lm, outs)
+    torch.cuda.synchronize()
+    assert cuda.jet_device_status() == 0
+    W = p0.f32("w_lm")
+    for p, out in zip(probs, outs):
+        got = dict(ell=out["tok_logprob"].numpy(), s=out["cand_score"].numpy(),
+                   q=out["q_cand"].numpy(), choice=out["choice"].numpy(),
+                   value=out["value"].numpy())
+        check_scores(oracle_layout(p), p, got, range(len(p.prefix_len)), w_lm=W)
