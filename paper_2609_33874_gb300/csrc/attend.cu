@@ -24,6 +24,8 @@ constexpr int kQV = 16;       // query vectors per CTA
 constexpr int kKT = 32;       // keys per tile
 constexpr int kThreads = 256;
 constexpr long long kTargetCtas = 608;  // about four CTAs per SM on 152 SMs
+constexpr int kPlanSMs = 152;           // GB300
+constexpr int kMinChunkTc = 640;        // keys
 
 template <int DH>
 constexpr size_t prefix_smem_bytes() {
@@ -254,13 +256,24 @@ AttnPlan attn_plan(const jet_sizes& n, const jet_dims& d) {
   const long long avg_vecs = ((long long)n.N * g + n.R - 1) / n.R;
   const long long groups = (long long)n.R * d.Hkv * std::max<long long>(1, (avg_vecs + qv - 1) / qv);
   const int max_splits = std::max(1, (n.max_prefix + 63) / 64);
-  // about four CTAs per SM (152 SMs); tensor-core chunks keep at least 256
-  // keys so the per-chunk partials stay small next to the chunk's K/V bytes
-  long long want = (kTargetCtas + groups - 1) / groups;
-  int splits = int(std::min<long long>(std::max<long long>(want, 1), max_splits));
-  int chunk = (n.max_prefix + splits - 1) / splits;
-  chunk = (chunk + gran - 1) / gran * gran;
-  if (tc) chunk = std::max(chunk, 256);
+  int chunk;
+  if (tc) {
+    // the persistent kernel (one CTA per SM, longest items first) splits a
+    // request's prefix into near-equal chunks: no shorter than kMinChunkTc keys
+    // (an item's fixed cost - query block in, f32 partial out and read back by
+    // the combine - is worth about five 64-key tiles), and no finer than half
+    // of one SM's share of all key tiles, so that the schedule can balance
+    const double avg_tiles = double(n.total_prefix) / n.R / 64.0 + 0.5;
+    const double share = double(groups) * avg_tiles / kPlanSMs;  // tiles per SM
+    chunk = std::max(kMinChunkTc, int(share / 2.0 + 0.999) * 64);
+    chunk = std::min(chunk, max_splits * 64);  // one chunk holds the longest prefix
+  } else {
+    // about four CTAs per SM
+    long long want = (kTargetCtas + groups - 1) / groups;
+    int splits = int(std::min<long long>(std::max<long long>(want, 1), max_splits));
+    chunk = (n.max_prefix + splits - 1) / splits;
+    chunk = (chunk + gran - 1) / gran * gran;
+  }
   p.chunk = chunk;
   p.splits = (n.max_prefix + chunk - 1) / chunk;
   const size_t vecs = size_t(p.splits) * n.N * d.Hq;

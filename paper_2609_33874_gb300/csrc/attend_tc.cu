@@ -16,7 +16,10 @@
 //               running max m and sum l in base 2, writes P_j = 2^(s - m) as
 //               bf16 into a 128-byte-swizzled shared tile; O is rescaled in
 //               TMEM only when the row max grows by more than 8 (a factor 256),
-//               so P stays <= 256 and rescales are rare.
+//               so P stays <= 256 and rescales are rare; at the item's end
+//               they write its output through shared memory (coalesced).
+//   warp 6      scheduler: claims work items one ahead, computes their
+//               geometry and starts their query block on the way into L2.
 // The CTA writes its unnormalised O and (m, l) as a partial; the merge kernel
 // combines the chunks with the candidates' own causal keys.
 #include <cuda.h>
@@ -37,11 +40,11 @@ using namespace sm100;
 constexpr int kBV = 128;      // query vectors per CTA (MMA M, TMEM lanes)
 constexpr int kBN = 64;       // keys per tile
 constexpr int kStages = 2;
-constexpr int kThreads = 192;
+constexpr int kThreads = 224;
+constexpr int kSchedWarp = 6;  // the work-item scheduler
 constexpr uint64_t kWaitNs = 2000000000ull;
 constexpr uint64_t kDrainNs = 200000000ull;
 constexpr float kRescaleLog2 = 8.f;  // rescale O only when the max grows by > 2^8
-constexpr int kPrefetch = 4;         // key tiles prefetched into L2 ahead of the TMA loads
 
 template <int DH>
 struct Geo {
@@ -152,6 +155,17 @@ __device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap* map, int32_t 
                : "memory");
 }
 
+// A request's P prefix keys in chunks of nearly equal length: at most
+// ceil(P / chunk) chunks of a whole number of 64-key tiles each, none empty
+// (the last also takes the candidates' own keys).
+__device__ __forceinline__ int req_splits(int P, int chunk, int* tiles_per_split) {
+  const int tiles = (P + kBN - 1) / kBN;
+  const int s0 = max(1, (P + chunk - 1) / chunk);
+  const int per = (tiles + s0 - 1) / s0;
+  *tiles_per_split = per;
+  return (tiles + per - 1) / per;
+}
+
 // Geometry of one work item (request r, key/value head kh, query block qb,
 // prefix chunk split); every role derives it the same way from the item.
 struct ItemGeo {
@@ -179,14 +193,15 @@ __device__ __forceinline__ ItemGeo item_geo(const AttArgs& a, int4 it) {
   if (e.row0 >= e.nr) return e;
   e.vbase = e.row0 * a.g;
   e.nv = min(a.rb, e.nr - e.row0) * a.g;
-  e.k_begin = e.split * a.chunk;
-  e.k_end = min(e.P, e.k_begin + a.chunk);
-  if (e.k_end <= e.k_begin) return e;
+  int per = 0;
+  e.splits_r = req_splits(e.P, a.chunk, &per);
+  if (e.split >= e.splits_r) return e;
+  e.k_begin = e.split * per * kBN;
+  e.k_end = min(e.P, e.k_begin + per * kBN);
   e.npt = (e.k_end - e.k_begin + kBN - 1) / kBN;
   // the request's last chunk also takes its candidates' own keys: the F_r fed
   // tokens, as extra 64-key tiles masked per row to the row's candidate and
   // position (Sec. 4.1: a candidate attends to its own earlier tokens only)
-  e.splits_r = (e.P + a.chunk - 1) / a.chunk;
   e.f_begin = e.n0 - e.r;  // fed-token index of the request's first fed row
   const int F_r = e.nr - 1;
   e.nct = (e.split == e.splits_r - 1 && a.has_cand && F_r > 0) ? (F_r + kBN - 1) / kBN : 0;
@@ -261,11 +276,21 @@ attend_items_kernel(const AttArgs a, int qgroups, int splits) {
   }
 }
 
-// One persistent CTA per SM; items are taken from the work list one at a time
-// by the producer and handed to the other roles through a two-slot ring. All
-// barrier phases run on counters that continue across items, so the next
-// item's query block and first K/V tiles load while the current item's last
-// tiles and its output are still in flight.
+// One work item as the scheduler warp publishes it: the item and the geometry
+// every role needs (16-byte aligned entries: the ring is read with vector loads).
+struct __align__(16) RingItem {
+  int4 it;
+  ItemGeo e;
+};
+static_assert(sizeof(RingItem) % 16 == 0, "ring entries keep 16-byte alignment");
+
+// One persistent CTA per SM. The scheduler warp claims the work items one
+// ahead of the others (the first one without touching the shared counter),
+// computes their geometry once and starts their query block on its way into
+// L2; the other roles take the items from a two-slot ring and release a slot
+// when they are done with its item. All barrier phases run on counters that
+// continue across items, so the next item's query block and first K/V tiles
+// load while the current item's last tiles and its output are still in flight.
 template <int DH>
 __global__ void __launch_bounds__(kThreads, 1)
 attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
@@ -277,10 +302,10 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  // the item ring first (16-byte entries at a 1024-byte aligned offset), then
-  // the barriers. K and V of a stage fill and drain separately: K is free once
-  // S_j has been computed, V only after P_j V_j
-  int4* ring = reinterpret_cast<int4*>(smem + G::kOffBar);  // [2] items
+  // the item ring first (16-byte aligned entries at a 1024-byte aligned
+  // offset), then the barriers. K and V of a stage fill and drain separately:
+  // K is free once S_j has been computed, V only after P_j V_j
+  RingItem* ring = reinterpret_cast<RingItem*>(smem + G::kOffBar);  // [2]
   uint64_t* k_full = reinterpret_cast<uint64_t*>(ring + 2);
   uint64_t* k_empty = k_full + kStages;
   uint64_t* v_full = k_empty + kStages;
@@ -314,7 +339,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       mbar_init(p_full + b, 4);
       mbar_init(p_free + b, 1);
       mbar_init(item_full + b, 1);
-      mbar_init(item_empty + b, 5);  // the MMA thread + 4 softmax warps
+      mbar_init(item_empty + b, 6);  // producer, MMA thread, 4 softmax warps
     }
     mbar_init(q_full, 1);
     mbar_init(q_free, 1);
@@ -343,30 +368,32 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t tmem = *tmem_slot;
   const int4 kDone = make_int4(-1, -1, -1, -1);
 
-  if (warp == 0) {
-    // ---------------------------------------------------------------- producer
+  if (warp == kSchedWarp) {
+    // ---------------------------------------------------------------- scheduler
     if (lane == 0) {
-      const uint64_t pol = policy_evict_first();
       const int count = a.sorted ? *a.item_count : 0;
-      uint32_t k_issued = 0, k_par = 0, v_issued = 0, v_par = 0, q_issued = 0, q_par = 0;
-      int Tk = 0, Tv = 0, v = 0;  // K and V tiles issued so far, items processed so far
-      bool ok = true;
-      for (int u = 0; ok; ++u) {
+      for (int u = 0;; ++u) {
         const int slot = u & 1;
         if (!mbar_wait(item_empty + slot, ((u >> 1) & 1) ^ 1u, kWaitNs, abort_flag)) {
-          ok = false;
+          *abort_flag = 1;
+          flag(a.status, JET_ERR_TIMEOUT);
           break;
         }
+        // the CTA's first item is slot blockIdx.x; later ones come from the
+        // shared counter, past the grid's first items
         int4 it = kDone;
-        if (a.sorted) {
-          const int idx = atomicAdd(a.item_next, 1);
-          if (idx < count) it = a.items[idx];
-        } else {
-          // the next slot that holds work, taken from a shared counter; slots
-          // run over the requests by decreasing prefix length (query blocks
-          // past the first, mostly empty, last)
-          while (true) {
-            const long long sl = atomicAdd(a.item_next, 1);
+        ItemGeo e{};
+        for (bool first = (u == 0);; first = false) {
+          int4 cand;
+          if (a.sorted) {
+            const int idx = first ? int(blockIdx.x) : int(gridDim.x) + atomicAdd(a.item_next, 1);
+            if (idx >= count) break;
+            cand = a.items[idx];
+          } else {
+            // slots run over the requests by decreasing prefix length (query
+            // blocks past the first, mostly empty, last)
+            const long long sl =
+                first ? (long long)blockIdx.x : (long long)gridDim.x + atomicAdd(a.item_next, 1);
             if (sl >= a.n_all) break;
             const int split = int(sl % a.splits);
             const long long rest = sl / a.splits;
@@ -374,21 +401,42 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
             const long long rest2 = rest / a.Hkv;
             const int ri = int(rest2 % a.R);
             const int qb = int(rest2 / a.R);
-            const int4 cand = make_int4(a.req_order[ri], kh, qb, split);
-            if (item_geo(a, cand).ok) {
-              it = cand;
-              break;
-            }
+            cand = make_int4(a.req_order[ri], kh, qb, split);
           }
+          const ItemGeo ce = item_geo(a, cand);
+          if (ce.ok) {
+            it = cand;
+            e = ce;
+            break;
+          }
+          if (a.sorted) flag(a.status, JET_ERR_DEVICE);  // the list holds an item the layout lacks
         }
-        ring[slot] = it;
+        ring[slot].it = it;
+        ring[slot].e = e;
         mbar_arrive(item_full + slot);
         if (it.x < 0) break;
-        const ItemGeo e = item_geo(a, it);
-        if (!e.ok) {
-          flag(a.status, JET_ERR_DEVICE);
-          continue;
+        // start the query block on its way into L2 (K/V tiles are not
+        // prefetched: extra requests in flight only delay the demand loads)
+#pragma unroll
+        for (int sl = 0; sl < G::kSlices; ++sl)
+          tma_prefetch_3d(&tmQ, sl * 64, e.kh * g, e.n0 + e.row0);
+      }
+    }
+  } else if (warp == 0) {
+    // ---------------------------------------------------------------- producer
+    if (lane == 0) {
+      const uint64_t pol = policy_evict_first();
+      uint32_t k_issued = 0, k_par = 0, v_issued = 0, v_par = 0, q_issued = 0, q_par = 0;
+      int Tk = 0, Tv = 0, v = 0;  // K and V tiles issued so far, items processed so far
+      bool ok = true;
+      for (int u = 0; ok; ++u) {
+        const int slot = u & 1;
+        if (!mbar_wait(item_full + slot, (u >> 1) & 1, kWaitNs, abort_flag)) {
+          ok = false;
+          break;
         }
+        if (ring[slot].it.x < 0) break;
+        const ItemGeo e = ring[slot].e;
         // the query block: rb rows x g heads x d of the group, once the last
         // QK^T of the previous item has read the old one
         if (v >= 1 && !mbar_wait(q_free, (v - 1) & 1, kWaitNs, abort_flag)) {
@@ -420,17 +468,6 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
 #pragma unroll
               for (int sl = 0; sl < G::kSlices; ++sl)
                 tma_load_3d(ks + sl * (kBN * 128), mk, k_full + s, sl * 64, e.kh, key, pol);
-              // keep kPrefetch further prefix tiles on their way into L2: two
-              // shared stages alone hold too few bytes in flight for HBM latency
-              for (int jp = (jk == 0 ? 1 : jk + kPrefetch); jp <= jk + kPrefetch && jp < e.npt;
-                   ++jp) {
-                const int kp = e.p0 + e.k_begin + jp * kBN;
-#pragma unroll
-                for (int sl = 0; sl < G::kSlices; ++sl) {
-                  tma_prefetch_3d(&tmK, sl * 64, e.kh, kp);
-                  tma_prefetch_3d(&tmV, sl * 64, e.kh, kp);
-                }
-              }
               k_issued |= 1u << s;
               k_par = (k_par & ~(1u << s)) | (ph << s);
               ++jk;
@@ -464,6 +501,8 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
             break;
           }
         }
+        if (!ok) break;
+        mbar_arrive(item_empty + slot);
         Tk += e.ntiles;
         Tv += e.ntiles;
         ++v;
@@ -493,11 +532,8 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
           ok = false;
           break;
         }
-        const int4 it = ring[slot];
-        mbar_arrive(item_empty + slot);
-        if (it.x < 0) break;
-        const ItemGeo e = item_geo(a, it);
-        if (!e.ok) continue;
+        if (ring[slot].it.x < 0) break;
+        const ItemGeo e = ring[slot].e;
         if (!mbar_wait(q_full, v & 1, kWaitNs, abort_flag)) {
           ok = false;
           break;
@@ -556,6 +592,8 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
             ok = false;
           }
         }
+        if (!ok) break;
+        mbar_arrive(item_empty + slot);
         T += e.ntiles;
         ++v;
       }
@@ -571,6 +609,10 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
     const int q4 = warp & 3;
     const int i = q4 * 32 + lane;  // query vector within the block = TMEM lane
     const uint32_t lane_off = uint32_t(q4 * 32) << 16;
+    // the output is transposed through this warp's own 32 rows of P buffer 0
+    // (4 KB, free once the item's last P V has completed) so that every global
+    // store covers whole 64- or 128-byte pieces of one vector's output
+    uint4* stage = reinterpret_cast<uint4*>(smem + G::kOffP + q4 * 32 * 128);
     // the query blocks arrive by TMA (rows [0, rb g)); zero the rows past them
     // once so that no stale shared memory enters the MMA
     if (i >= rb * g) {
@@ -591,19 +633,13 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         ok = false;
         break;
       }
-      const int4 it = ring[slot];
-      __syncwarp();
-      if (lane == 0) mbar_arrive(item_empty + slot);
-      if (it.x < 0) break;
-      const ItemGeo e = item_geo(a, it);
-      if (!e.ok) continue;
+      if (ring[slot].it.x < 0) break;
+      const ItemGeo e = ring[slot].e;
       const bool valid = i < e.nv;
-      int n = 0, h = 0;
       int fa = 1, fb = 0;  // fed-token indices this vector may see (none: shared row)
       if (valid) {
         const int gv = e.vbase + i;
-        n = e.n0 + gv / g;
-        h = e.kh * g + gv % g;
+        const int n = e.n0 + gv / g;
         const int c = a.row_cand[n];
         if (c >= 0 && c < a.C) {
           fa = a.cand_row_offset[c] - e.r - 1;  // y_{c,1}
@@ -710,34 +746,76 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         break;
       }
       tc_fence_after();
-      const size_t base = (size_t(e.split) * a.N + n) * a.Hq + h;
       const bool direct = e.splits_r == 1;  // the whole row in this item: final output
+      if (valid) {
+        const int gv = e.vbase + i;
+        const int n = e.n0 + gv / g, h = e.kh * g + gv % g;
+        if (!direct) a.ml_part[(size_t(e.split) * a.N + n) * a.Hq + h] = make_float2(m_used, l);
+      }
+      // the destination of the vectors this lane stores: vector 4 s + lane / 8
+      // (f32 partial, 8 lanes x 16 bytes each) or 8 s + lane / 4 (bf16 output,
+      // 4 lanes x 16 bytes each); element offsets, -1 past the block's vectors
+      long long dst[8];
+#pragma unroll
+      for (int s = 0; s < 8; ++s) {
+        const int iv = direct ? 8 * s + (lane >> 2) : 4 * s + (lane >> 3);
+        const int gi = q4 * 32 + iv;
+        dst[s] = -1;
+        if ((!direct || s < 4) && gi < e.nv) {
+          const int gv = e.vbase + gi;
+          const int n = e.n0 + gv / g, h = e.kh * g + gv % g;
+          dst[s] = direct ? (long long)(size_t(n) * a.Hq + h) * DH
+                          : (long long)((size_t(e.split) * a.N + n) * a.Hq + h) * DH;
+        }
+      }
       const float inv = l > 0.f ? 1.f / l : 0.f;
 #pragma unroll 1
       for (int c0 = 0; c0 < DH; c0 += 32) {
         float ov[32];
         tmem_ld_32cols(tmem + lane_off + G::kOCol + c0, ov);
         tmem_wait_ld();
-        if (valid && direct) {
-          uint4* dst = reinterpret_cast<uint4*>(a.o + (size_t(n) * a.Hq + h) * DH + c0);
+        if (direct) {
+          // 32 bf16 = four 16-byte pieces per vector; two vectors per 128-byte
+          // row of the stage, pieces rotated so that 8 lanes hit 8 bank groups
 #pragma unroll
-          for (int c = 0; c < 4; ++c)
-            dst[c] = make_uint4(pack_bf16(ov[8 * c] * inv, ov[8 * c + 1] * inv),
-                                pack_bf16(ov[8 * c + 2] * inv, ov[8 * c + 3] * inv),
-                                pack_bf16(ov[8 * c + 4] * inv, ov[8 * c + 5] * inv),
-                                pack_bf16(ov[8 * c + 6] * inv, ov[8 * c + 7] * inv));
-        } else if (valid) {
-          float4* dst = reinterpret_cast<float4*>(a.o_part + base * DH + c0);
+          for (int q = 0; q < 4; ++q)
+            stage[(lane >> 1) * 8 + (lane & 1) * 4 + (q ^ ((lane >> 1) & 3))] =
+                make_uint4(pack_bf16(ov[8 * q] * inv, ov[8 * q + 1] * inv),
+                           pack_bf16(ov[8 * q + 2] * inv, ov[8 * q + 3] * inv),
+                           pack_bf16(ov[8 * q + 4] * inv, ov[8 * q + 5] * inv),
+                           pack_bf16(ov[8 * q + 6] * inv, ov[8 * q + 7] * inv));
+          __syncwarp();
 #pragma unroll
-          for (int c = 0; c < 8; ++c)
-            dst[c] = make_float4(ov[4 * c], ov[4 * c + 1], ov[4 * c + 2], ov[4 * c + 3]);
+          for (int s = 0; s < 4; ++s) {
+            const int iv = 8 * s + (lane >> 2), c = lane & 3;
+            const uint4 val = stage[(iv >> 1) * 8 + (iv & 1) * 4 + (c ^ ((iv >> 1) & 3))];
+            if (dst[s] >= 0) *reinterpret_cast<uint4*>(a.o + dst[s] + c0 + c * 8) = val;
+          }
+        } else {
+          // 32 f32 = eight 16-byte pieces per vector, one vector per 128-byte
+          // row of the stage, pieces rotated by the row
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            stage[lane * 8 + (q ^ (lane & 7))] =
+                make_uint4(__float_as_uint(ov[4 * q]), __float_as_uint(ov[4 * q + 1]),
+                           __float_as_uint(ov[4 * q + 2]), __float_as_uint(ov[4 * q + 3]));
+          __syncwarp();
+#pragma unroll
+          for (int s = 0; s < 8; ++s) {
+            const int iv = 4 * s + (lane >> 3), c = lane & 7;
+            const uint4 val = stage[iv * 8 + (c ^ (iv & 7))];
+            if (dst[s] >= 0) *reinterpret_cast<uint4*>(a.o_part + dst[s] + c0 + c * 4) = val;
+          }
         }
+        __syncwarp();
       }
-      if (valid && !direct) a.ml_part[base] = make_float2(m_used, l);
-      // O may be overwritten by the next item's first P V
+      // O may be overwritten by the next item's first P V; the ring slot is free
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(o_free);
+      if (lane == 0) {
+        mbar_arrive(o_free);
+        mbar_arrive(item_empty + slot);
+      }
       T += e.ntiles;
     }
     if (!ok) {
@@ -803,7 +881,8 @@ attend_combine_kernel(const int32_t* __restrict__ prefix_offset, const int32_t* 
     return;
   }
   const int P = prefix_offset[r + 1] - prefix_offset[r];
-  const int splits_r = (P + chunk - 1) / chunk;
+  int per = 0;
+  const int splits_r = req_splits(P, chunk, &per);
   if (splits_r <= 1) return;
   constexpr int PER = DH / 32;
   float acc[PER];
