@@ -42,6 +42,7 @@ attend_prefix_kernel(const int32_t* __restrict__ prefix_offset, const int32_t* _
                      int R, int N, int total_prefix, int Hq, int Hkv, int chunk,
                      const T* __restrict__ q, const T* __restrict__ k_pre, const T* __restrict__ v_pre,
                      float* __restrict__ o_part, float2* __restrict__ ml_part, int* status) {
+  pdl_begin();
   extern __shared__ float smem[];
   float* Qs = smem;                          // [kQV][DH+1], pre-scaled by 1/sqrt(d)
   float* Ks = Qs + kQV * (DH + 1);           // [kKT][DH+1]
@@ -154,6 +155,7 @@ attend_merge_kernel(const int32_t* __restrict__ row_req, const int32_t* __restri
                     int splits, const T* __restrict__ q, const T* __restrict__ k_cand,
                     const T* __restrict__ v_cand, const float* __restrict__ o_part,
                     const float2* __restrict__ ml_part, T* __restrict__ o, int* status) {
+  pdl_begin();
   const int lane = threadIdx.x & 31;
   const long long idx = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (idx >= (long long)N * Hq) return;
@@ -224,19 +226,17 @@ cudaError_t launch_typed(const jet_layout& lay, const jet_dims& d, const AttnPla
                              cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     if (e != cudaSuccess) return e;
     dim3 grid(plan.splits, plan.qgroups, unsigned(n.R * d.Hkv));
-    attend_prefix_kernel<T, DH><<<grid, kThreads, smem, st>>>(
-        lay.prefix_offset, lay.row_offset, n.R, n.N, n.total_prefix, d.Hq, d.Hkv, plan.chunk,
-        static_cast<const T*>(q), static_cast<const T*>(k_pre), static_cast<const T*>(v_pre),
-        o_part, ml_part, status);
-    e = cudaGetLastError();
+    e = launch_pdl(attend_prefix_kernel<T, DH>, grid, dim3(kThreads), smem, st, lay.prefix_offset,
+                   lay.row_offset, n.R, n.N, n.total_prefix, d.Hq, d.Hkv, plan.chunk,
+                   static_cast<const T*>(q), static_cast<const T*>(k_pre),
+                   static_cast<const T*>(v_pre), o_part, ml_part, status);
   }
   if (e != cudaSuccess) return e;
   const long long warps = (long long)n.N * d.Hq;
-  attend_merge_kernel<T, DH><<<unsigned((warps + 7) / 8), 256, 0, st>>>(
-      lay.row_req, lay.row_cand, lay.cand_row_offset, n.N, n.R, n.C, d.Hq, d.Hkv, plan.splits,
-      static_cast<const T*>(q), static_cast<const T*>(k_cand), static_cast<const T*>(v_cand),
-      o_part, ml_part, static_cast<T*>(o), status);
-  return cudaGetLastError();
+  return launch_pdl(attend_merge_kernel<T, DH>, dim3(unsigned((warps + 7) / 8)), dim3(256), 0, st,
+                    lay.row_req, lay.row_cand, lay.cand_row_offset, n.N, n.R, n.C, d.Hq, d.Hkv,
+                    plan.splits, static_cast<const T*>(q), static_cast<const T*>(k_cand),
+                    static_cast<const T*>(v_cand), o_part, ml_part, static_cast<T*>(o), status);
 }
 
 }  // namespace

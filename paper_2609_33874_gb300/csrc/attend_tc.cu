@@ -227,6 +227,7 @@ __device__ __forceinline__ int4 item_of(const AttArgs& a, long long idx, int spl
 
 __global__ void __launch_bounds__(1024)
 attend_items_kernel(const AttArgs a, int qgroups, int splits) {
+  pdl_begin();
   __shared__ int hist[kBuckets];
   __shared__ int cursor[kBuckets];
   __shared__ int wsum[kBuckets / 32];
@@ -274,6 +275,12 @@ attend_items_kernel(const AttArgs a, int qgroups, int splits) {
     }
     if (b > 0) a.items[atomicAdd(&cursor[b], 1)] = it;
   }
+}
+
+// The shared item counter of the dynamic schedule starts at zero.
+__global__ void attend_reset_kernel(int* item_next) {
+  pdl_begin();
+  if (threadIdx.x == 0) *item_next = 0;
 }
 
 // One work item as the scheduler warp publishes it: the item and the geometry
@@ -349,10 +356,6 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
     *abort_flag = 0;
     fence_barrier_init();
   }
-  if (warp == 1) {
-    tmem_alloc(tmem_slot, G::kTmemCols);
-    tmem_relinquish();
-  }
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmQ);
     tma_prefetch_desc(&tmK);
@@ -361,6 +364,12 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       tma_prefetch_desc(&tmKc);
       tma_prefetch_desc(&tmVc);
     }
+  }
+  // global memory and TMEM only after the previous kernel of the stream is done
+  pdl_begin();
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, G::kTmemCols);
+    tmem_relinquish();
   }
   tc_fence_before();
   __syncthreads();
@@ -871,6 +880,7 @@ attend_combine_kernel(const int32_t* __restrict__ prefix_offset, const int32_t* 
                       int N, int R, int Hq, int chunk, const float* __restrict__ o_part,
                       const float2* __restrict__ ml_part, __nv_bfloat16* __restrict__ o,
                       int* status) {
+  pdl_begin();
   const int lane = threadIdx.x & 31;
   const long long idx = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (idx >= (long long)N * Hq) return;
@@ -963,12 +973,10 @@ cudaError_t launch_dh(const jet_layout& lay, const jet_dims& d, const AttnPlan& 
   // long and uneven (chunks of 16 key tiles or more)
   a.sorted = plan.chunk >= 16 * kBN;
   cudaError_t e = cudaSuccess;
-  if (a.sorted) {
-    attend_items_kernel<<<1, 1024, 0, st>>>(a, plan.qgroups, plan.splits);
-    e = cudaGetLastError();
-  } else {
-    e = cudaMemsetAsync(a.item_next, 0, sizeof(int), st);  // the shared slot counter
-  }
+  if (a.sorted)
+    e = launch_pdl(attend_items_kernel, dim3(1), dim3(1024), 0, st, a, plan.qgroups, plan.splits);
+  else
+    e = launch_pdl(attend_reset_kernel, dim3(1), dim3(32), 0, st, a.item_next);
   if (e != cudaSuccess) return e;
   const size_t smem = Geo<DH>::kBytes + 1024;
   e = cudaFuncSetAttribute(attend_prefix_tc_kernel<DH>,
@@ -980,14 +988,13 @@ cudaError_t launch_dh(const jet_layout& lay, const jet_dims& d, const AttnPlan& 
     return cudaErrorInvalidValue;
   const long long max_items = (long long)n.R * d.Hkv * plan.qgroups * plan.splits;
   const int grid = int(std::max<long long>(1, std::min<long long>(sms, max_items)));
-  attend_prefix_tc_kernel<DH><<<grid, kThreads, smem, st>>>(tmQ, tmK, tmV, tmKc, tmVc, a);
-  e = cudaGetLastError();
+  e = launch_pdl(attend_prefix_tc_kernel<DH>, dim3(grid), dim3(kThreads), smem, st, tmQ, tmK, tmV,
+                 tmKc, tmVc, a);
   if (e != cudaSuccess || plan.splits <= 1) return e;
   const long long warps = (long long)n.N * d.Hq;
-  attend_combine_kernel<DH><<<unsigned((warps + 7) / 8), 256, 0, st>>>(
-      lay.prefix_offset, lay.row_req, n.N, n.R, d.Hq, plan.chunk, o_part, ml_part,
-      static_cast<__nv_bfloat16*>(o), status);
-  return cudaGetLastError();
+  return launch_pdl(attend_combine_kernel<DH>, dim3(unsigned((warps + 7) / 8)), dim3(256), 0, st,
+                    lay.prefix_offset, lay.row_req, n.N, n.R, d.Hq, plan.chunk, o_part, ml_part,
+                    static_cast<__nv_bfloat16*>(o), status);
 }
 
 }  // namespace

@@ -61,6 +61,7 @@ fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__
             const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
             const float* __restrict__ alpha, const float* __restrict__ beta, T* __restrict__ o,
             float* __restrict__ s_fork, int* status) {
+  pdl_begin();
   __shared__ __align__(16) float red[4 * kCols];
   // a window of the request's fed tokens: k, q (all rows), v (this slice), gates
   __shared__ __align__(16) float wk[kWin][kDK];
@@ -179,20 +180,17 @@ cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, const fl
   dim3 grid(unsigned(d.dv / kCols), unsigned(d.Hl), unsigned(n.R));
   const int F = n.N - n.R;
   if (d.dtype == JET_DTYPE_F32) {
-    fork_kernel<float><<<grid, kThreads, 0, st>>>(
-        lay.cand_offset, lay.cand_row_offset, lay.tgt_offset, lay.row_offset, n.R, n.C, F, d.Hl,
-        d.dv, s_prefix,
-        static_cast<const float*>(q), static_cast<const float*>(k), static_cast<const float*>(v),
-        alpha, beta, static_cast<float*>(o), s_fork, status);
-  } else {
-    fork_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(
-        lay.cand_offset, lay.cand_row_offset, lay.tgt_offset, lay.row_offset, n.R, n.C, F, d.Hl,
-        d.dv, s_prefix,
-        static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k),
-        static_cast<const __nv_bfloat16*>(v), alpha, beta, static_cast<__nv_bfloat16*>(o), s_fork,
-        status);
+    return launch_pdl(fork_kernel<float>, grid, dim3(kThreads), 0, st, lay.cand_offset,
+                      lay.cand_row_offset, lay.tgt_offset, lay.row_offset, n.R, n.C, F, d.Hl,
+                      d.dv, s_prefix, static_cast<const float*>(q), static_cast<const float*>(k),
+                      static_cast<const float*>(v), alpha, beta, static_cast<float*>(o), s_fork,
+                      status);
   }
-  return cudaGetLastError();
+  return launch_pdl(fork_kernel<__nv_bfloat16>, grid, dim3(kThreads), 0, st, lay.cand_offset,
+                    lay.cand_row_offset, lay.tgt_offset, lay.row_offset, n.R, n.C, F, d.Hl, d.dv,
+                    s_prefix, static_cast<const __nv_bfloat16*>(q),
+                    static_cast<const __nv_bfloat16*>(k), static_cast<const __nv_bfloat16*>(v),
+                    alpha, beta, static_cast<__nv_bfloat16*>(o), s_fork, status);
 }
 
 }  // namespace jet

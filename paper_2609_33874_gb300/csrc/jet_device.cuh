@@ -21,6 +21,18 @@ __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float x) {
   return __float2bfloat16_rn(x);
 }
 
+// ---- programmatic dependent launch -------------------------------------------
+// Every kernel of libjet is launched with programmatic stream serialization
+// (launch_pdl), so it may start while the kernel before it in the stream still
+// runs. pdl_begin() lets the kernel after it start early in turn, then waits
+// until all earlier work in the stream has completed and its writes are
+// visible. A kernel touches no global memory before pdl_begin(); setting up
+// shared memory and barriers may come first.
+__device__ __forceinline__ void pdl_begin() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
 // record the first error a kernel meets; later ones keep the first code
 __device__ __forceinline__ void flag(int* status, int code) {
   if (status) atomicCAS(status, 0, code);

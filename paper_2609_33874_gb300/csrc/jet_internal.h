@@ -34,6 +34,26 @@ struct ScorePlan {
 };
 ScorePlan score_plan(const jet_sizes& n);
 
+// ---- launches ------------------------------------------------------------------
+// Stream-ordered launch with programmatic stream serialization: the kernel may
+// begin (up to its pdl_begin()) while the previous kernel of the stream ends,
+// which hides the launch latency between the dependent kernels of a step.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, Args... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr{};
+  attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr.val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // ---- kernel launchers (stream-ordered; return the launch error) ---------------
 cudaError_t launch_prefix_attend(const jet_layout& lay, const jet_dims& d, const AttnPlan& plan,
                                  const void* q, const void* k_pre, const void* v_pre,

@@ -23,6 +23,7 @@ lmhead_simt_kernel(const int32_t* __restrict__ target_ids, const int32_t* __rest
                    const int32_t* __restrict__ row_tgt_index, int N, int T_, int V, int D,
                    const T* __restrict__ hidden, const T* __restrict__ w_lm,
                    float2* __restrict__ part, float* __restrict__ z_tgt, int* status) {
+  pdl_begin();
   __shared__ float Hs[kBK][kBM + 1];
   __shared__ float Ws[kBK][kBV + 1];
   const int row0 = blockIdx.x * kBM;
@@ -108,16 +109,15 @@ cudaError_t launch_lmhead_simt(const jet_layout& lay, const jet_dims& d, const S
   float* z_tgt = reinterpret_cast<float*>(base + plan.ztgt_off);
   dim3 grid(unsigned((n.N + kBM - 1) / kBM), unsigned(plan.vtiles));
   if (d.dtype == JET_DTYPE_F32) {
-    lmhead_simt_kernel<float><<<grid, kThreads, 0, st>>>(
-        lay.target_ids, lay.row_tgt_offset, lay.row_tgt_index, n.N, n.T, n.V, d.D,
-        static_cast<const float*>(hidden), static_cast<const float*>(w_lm), part, z_tgt, status);
-  } else {
-    lmhead_simt_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(
-        lay.target_ids, lay.row_tgt_offset, lay.row_tgt_index, n.N, n.T, n.V, d.D,
-        static_cast<const __nv_bfloat16*>(hidden), static_cast<const __nv_bfloat16*>(w_lm), part,
-        z_tgt, status);
+    return launch_pdl(lmhead_simt_kernel<float>, grid, dim3(kThreads), 0, st, lay.target_ids,
+                      lay.row_tgt_offset, lay.row_tgt_index, n.N, n.T, n.V, d.D,
+                      static_cast<const float*>(hidden), static_cast<const float*>(w_lm), part,
+                      z_tgt, status);
   }
-  return cudaGetLastError();
+  return launch_pdl(lmhead_simt_kernel<__nv_bfloat16>, grid, dim3(kThreads), 0, st,
+                    lay.target_ids, lay.row_tgt_offset, lay.row_tgt_index, n.N, n.T, n.V, d.D,
+                    static_cast<const __nv_bfloat16*>(hidden),
+                    static_cast<const __nv_bfloat16*>(w_lm), part, z_tgt, status);
 }
 
 }  // namespace jet

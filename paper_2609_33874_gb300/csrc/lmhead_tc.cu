@@ -120,13 +120,15 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
     *epi_abort = 0;
     fence_barrier_init();
   }
-  if (warp == 1) {
-    tmem_alloc(tmem_slot, a.tmem_cols);
-    tmem_relinquish();
-  }
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmW);
     tma_prefetch_desc(&tmH);
+  }
+  // global memory and TMEM only after the previous kernel of the stream is done
+  pdl_begin();
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, a.tmem_cols);
+    tmem_relinquish();
   }
   tc_fence_before();
   __syncthreads();
@@ -389,8 +391,7 @@ cudaError_t launch_lmhead_tc(const jet_layout& lay, const jet_dims& d, const Sco
   int sms = sm_count();
   if (d.max_sms > 0) sms = std::min(sms, d.max_sms);
   const int grid = std::max(1, std::min(a.units, sms));
-  lmhead_tc_kernel<<<grid, kThreads, smem, st>>>(tmW, tmH, a);
-  return cudaGetLastError();
+  return launch_pdl(lmhead_tc_kernel, dim3(grid), dim3(kThreads), smem, st, tmW, tmH, a);
 }
 
 }  // namespace jet

@@ -16,6 +16,7 @@ namespace {
 // one block per row; coalesced reads of the row's partials part[n][0..vtiles)
 __global__ void __launch_bounds__(128)
 lse_kernel(const float2* __restrict__ part, int vtiles, int N, float* __restrict__ lse) {
+  pdl_begin();
   __shared__ float2 red[4];
   const int n = blockIdx.x;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -44,6 +45,7 @@ __global__ void finish_kernel(const int32_t* __restrict__ tgt_offset, const int3
                               int C, int N, int T_, const float* __restrict__ z_tgt,
                               const float* __restrict__ lse, float* __restrict__ tok_logprob,
                               float* __restrict__ cand_score, int* status) {
+  pdl_begin();
   const int c = blockIdx.x * blockDim.x + threadIdx.x;
   if (c >= C) return;
   const int j0 = tgt_offset[c], j1 = tgt_offset[c + 1];
@@ -70,6 +72,7 @@ __global__ void __launch_bounds__(256)
 decide_kernel(const int32_t* __restrict__ cand_offset, int R, int C, int mode,
               const float* __restrict__ s, float* __restrict__ q, int32_t* __restrict__ choice,
               float* __restrict__ value, int* status) {
+  pdl_begin();
   const int lane = threadIdx.x & 31;
   const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (r >= R) return;
@@ -141,21 +144,19 @@ cudaError_t launch_score_finish(const jet_layout& lay, const ScorePlan& plan, vo
   const float2* part = reinterpret_cast<const float2*>(base + plan.part_off);
   const float* z_tgt = reinterpret_cast<const float*>(base + plan.ztgt_off);
   float* lse = reinterpret_cast<float*>(base + plan.lse_off);
-  lse_kernel<<<unsigned(n.N), 128, 0, st>>>(part, plan.vtiles, n.N, lse);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e =
+      launch_pdl(lse_kernel, dim3(unsigned(n.N)), dim3(128), 0, st, part, plan.vtiles, n.N, lse);
   if (e != cudaSuccess) return e;
-  finish_kernel<<<unsigned((n.C + 127) / 128), 128, 0, st>>>(lay.tgt_offset, lay.tgt_row, n.C, n.N,
-                                                             n.T, z_tgt, lse, tok_logprob,
-                                                             cand_score, status);
-  return cudaGetLastError();
+  return launch_pdl(finish_kernel, dim3(unsigned((n.C + 127) / 128)), dim3(128), 0, st,
+                    lay.tgt_offset, lay.tgt_row, n.C, n.N, n.T, z_tgt, lse, tok_logprob,
+                    cand_score, status);
 }
 
 cudaError_t launch_decide(const jet_layout& lay, int mode, const float* cand_score, float* q,
                           int32_t* choice, float* value, int* status, cudaStream_t st) {
   const jet_sizes& n = lay.n;
-  decide_kernel<<<unsigned((n.R + 7) / 8), 256, 0, st>>>(lay.cand_offset, n.R, n.C, mode,
-                                                         cand_score, q, choice, value, status);
-  return cudaGetLastError();
+  return launch_pdl(decide_kernel, dim3(unsigned((n.R + 7) / 8)), dim3(256), 0, st,
+                    lay.cand_offset, n.R, n.C, mode, cand_score, q, choice, value, status);
 }
 
 }  // namespace jet
