@@ -23,6 +23,7 @@ constexpr int kDK = 128;        // key dimension handled (rows of S)
 constexpr int kCols = 32;       // value columns per CTA
 constexpr int kThreads = 128;   // 4 warps x 32 rows
 constexpr int kWin = 32;        // fed tokens staged in shared memory at a time
+constexpr int kMeta = 64;       // candidates whose lengths are staged at a time
 
 __device__ __forceinline__ float4 f4_fma(float a, float4 x, float4 y) {
   return make_float4(fmaf(a, x.x, y.x), fmaf(a, x.y, y.y), fmaf(a, x.z, y.z), fmaf(a, x.w, y.w));
@@ -51,6 +52,56 @@ __device__ __forceinline__ float4 rows_sum(float4 v, float* red, int warp, int l
   return s;
 }
 
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                   static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
+               "l"(src)
+               : "memory");
+}
+
+__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(
+                   static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
+               "l"(src)
+               : "memory");
+}
+
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+
+// Stage fed tokens [w0, w0 + nt) (nt <= kWin) into shared memory as they are
+// stored: their k and q rows, this slice's v columns and the gates. The
+// copies are asynchronous and all in flight at once, so a window costs one
+// memory latency and no registers; the caller synchronises the block.
+template <typename T>
+__device__ __forceinline__ void stage_window(const T* __restrict__ q, const T* __restrict__ k,
+                                             const T* __restrict__ v,
+                                             const float* __restrict__ alpha,
+                                             const float* __restrict__ beta, int Hl, int dv,
+                                             int h, int j0, int w0, int nt, int tid,
+                                             T (*wk)[kDK], T (*wq)[kDK], T (*wv)[kCols],
+                                             float* wa, float* wb) {
+  constexpr int VE = 16 / int(sizeof(T));  // elements per 16-byte piece
+  constexpr int KP = kDK / VE;             // pieces of a k (or q) row
+  constexpr int VP = kCols / VE;           // pieces of a v slice row
+  for (int e = tid; e < nt * KP; e += kThreads) {
+    const int tok = e / KP, pc = e % KP;
+    const size_t src = (size_t(w0 + tok) * Hl + h) * kDK + pc * VE;
+    cp_async16(&wk[tok][pc * VE], k + src);
+    cp_async16(&wq[tok][pc * VE], q + src);
+  }
+  for (int e = tid; e < nt * VP; e += kThreads) {
+    const int tok = e / VP, pc = e % VP;
+    cp_async16(&wv[tok][pc * VE], v + (size_t(w0 + tok) * Hl + h) * dv + j0 + pc * VE);
+  }
+  if (tid < nt) {
+    cp_async4(&wa[tid], alpha + size_t(w0 + tid) * Hl + h);
+    cp_async4(&wb[tid], beta + size_t(w0 + tid) * Hl + h);
+  }
+  cp_async_wait_all();
+}
+
 // grid (dv / 32, Hl, R); thread (warp w, lane = 8 * rg + jq) owns rows
 // 32 w + rg + 4 ii (ii < 8) and columns j0 + 4 jq .. + 3 of the slice.
 template <typename T>
@@ -63,11 +114,16 @@ fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__
             float* __restrict__ s_fork, int* status) {
   pdl_begin();
   __shared__ __align__(16) float red[4 * kCols];
-  // a window of the request's fed tokens: k, q (all rows), v (this slice), gates
-  __shared__ __align__(16) float wk[kWin][kDK];
-  __shared__ __align__(16) float wq[kWin][kDK];
-  __shared__ __align__(16) float wv[kWin][kCols];
-  __shared__ float wa[kWin], wb[kWin];
+  // a window of the request's fed tokens as stored: k, q (all rows), v (this
+  // slice), gates
+  __shared__ __align__(16) T wk[kWin][kDK];
+  __shared__ __align__(16) T wq[kWin][kDK];
+  __shared__ __align__(16) T wv[kWin][kCols];
+  __shared__ __align__(16) float wa[kWin], wb[kWin];
+  // the (length, first fed token) of up to kMeta candidates at a time
+  __shared__ int cm[kMeta], cf[kMeta];
+  // the prefix state slice, each thread's own 8 float4 at [ii][tid]
+  __shared__ __align__(16) float4 ssp[8 * kThreads];
   const int r = blockIdx.z, h = blockIdx.y, j0 = blockIdx.x * kCols;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rg = lane >> 3, jq = lane & 7;
@@ -81,90 +137,96 @@ fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__
     return;
   }
 
-  // the prefix state slice: read once, reused by every candidate
-  float4 sp[8];
-  const size_t head = (size_t(r) * Hl + h) * kDK;
+  // the prefix state slice (read once, kept in shared memory for every
+  // candidate) and the first window of fed tokens load at once
+  {
+    float4 sp[8];
+    const size_t head = (size_t(r) * Hl + h) * kDK;
 #pragma unroll
-  for (int ii = 0; ii < 8; ++ii) {
-    const int i = 32 * warp + rg + 4 * ii;
-    sp[ii] = *reinterpret_cast<const float4*>(s_prefix + (head + i) * dv + col);
+    for (int ii = 0; ii < 8; ++ii) {
+      const int i = 32 * warp + rg + 4 * ii;
+      sp[ii] = *reinterpret_cast<const float4*>(s_prefix + (head + i) * dv + col);
+    }
+#pragma unroll
+    for (int ii = 0; ii < 8; ++ii) ssp[ii * kThreads + tid] = sp[ii];
   }
+  int w0 = f_begin, w1 = min(f_begin + kWin, f_end);  // fed tokens [w0, w1) are staged
+  if (w1 > w0)
+    stage_window(q, k, v, alpha, beta, Hl, dv, h, j0, w0, w1 - w0, tid, wk, wq, wv, wa, wb);
   const float rs = rsqrtf(float(kDK));
-  int w0 = f_begin, w1 = f_begin;  // fed tokens [w0, w1) are staged
 
-  for (int c = c0; c < c1; ++c) {
-    const int m = tgt_offset[c + 1] - tgt_offset[c];
-    const int f0 = cand_row_offset[c] - r - 1;  // fed-token index of y_{c,1}
-    if (m < 1 || f0 < f_begin || f0 + m - 1 > f_end) {
-      if (tid == 0) flag(status, JET_ERR_DEVICE);
-      continue;
+  for (int cb = c0; cb < c1; cb += kMeta) {
+    const int nb = min(kMeta, c1 - cb);
+    __syncthreads();  // the previous batch's lengths are no longer read
+    for (int e = tid; e < nb; e += kThreads) {
+      cm[e] = tgt_offset[cb + e + 1] - tgt_offset[cb + e];
+      cf[e] = cand_row_offset[cb + e] - r - 1;  // fed-token index of y_{c,1}
     }
-    float4 S[8];
+    __syncthreads();
+    for (int e = 0; e < nb; ++e) {
+      const int c = cb + e;
+      const int m = cm[e], f0 = cf[e];
+      if (m < 1 || f0 < f_begin || f0 + m - 1 > f_end) {
+        if (tid == 0) flag(status, JET_ERR_DEVICE);
+        continue;
+      }
+      float4 S[8];
 #pragma unroll
-    for (int ii = 0; ii < 8; ++ii) S[ii] = sp[ii];  // restore the prefix state
-    for (int t = 0; t < m - 1; ++t) {
-      const int f = f0 + t;
-      if (f >= w1) {
-        // stage the next window of fed tokens with coalesced loads
-        __syncthreads();
-        w0 = f;
-        w1 = min(f + kWin, f_end);
-        const int nt = w1 - w0;
-        for (int e = tid; e < nt * kDK; e += kThreads) {
-          const size_t src = (size_t(w0 + e / kDK) * Hl + h) * kDK + e % kDK;
-          wk[e / kDK][e % kDK] = to_f32(k[src]);
-          wq[e / kDK][e % kDK] = to_f32(q[src]);
+      for (int ii = 0; ii < 8; ++ii) S[ii] = ssp[ii * kThreads + tid];  // the prefix state
+      for (int t = 0; t < m - 1; ++t) {
+        const int f = f0 + t;
+        if (f < w0 || f >= w1) {
+          // stage the window of fed tokens starting at f
+          __syncthreads();
+          w0 = f;
+          w1 = min(f + kWin, f_end);
+          stage_window(q, k, v, alpha, beta, Hl, dv, h, j0, w0, w1 - w0, tid, wk, wq, wv, wa, wb);
+          __syncthreads();
         }
-        for (int e = tid; e < nt * kCols; e += kThreads)
-          wv[e / kCols][e % kCols] = to_f32(v[(size_t(w0 + e / kCols) * Hl + h) * dv + j0 + e % kCols]);
-        for (int e = tid; e < nt; e += kThreads) {
-          wa[e] = alpha[size_t(w0 + e) * Hl + h];
-          wb[e] = beta[size_t(w0 + e) * Hl + h];
+        const int wt = f - w0;
+        float kk[8], qq[8];
+#pragma unroll
+        for (int ii = 0; ii < 8; ++ii) {
+          const int i = 32 * warp + rg + 4 * ii;
+          kk[ii] = to_f32(wk[wt][i]);
+          qq[ii] = to_f32(wq[wt][i]);
         }
-        __syncthreads();
-      }
-      const int wt = f - w0;
-      float kk[8], qq[8];
+        const float a = wa[wt], b = wb[wt];
+        const float4 vv = make_float4(to_f32(wv[wt][4 * jq]), to_f32(wv[wt][4 * jq + 1]),
+                                      to_f32(wv[wt][4 * jq + 2]), to_f32(wv[wt][4 * jq + 3]));
+        // u = k^T S for this column quad
+        float4 u = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-      for (int ii = 0; ii < 8; ++ii) {
-        const int i = 32 * warp + rg + 4 * ii;
-        kk[ii] = wk[wt][i];
-        qq[ii] = wq[wt][i];
-      }
-      const float a = wa[wt], b = wb[wt];
-      const float4 vv = *reinterpret_cast<const float4*>(&wv[wt][4 * jq]);
-      // u = k^T S for this column quad
-      float4 u = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int ii = 0; ii < 8; ++ii) u = f4_fma(kk[ii], S[ii], u);
+        u = rows_sum(u, red, warp, lane);
+        // S = alpha S + beta k (v - alpha u)
+        const float4 w = make_float4(b * (vv.x - a * u.x), b * (vv.y - a * u.y),
+                                     b * (vv.z - a * u.z), b * (vv.w - a * u.w));
+        float4 op = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-      for (int ii = 0; ii < 8; ++ii) u = f4_fma(kk[ii], S[ii], u);
-      u = rows_sum(u, red, warp, lane);
-      // S = alpha S + beta k (v - alpha u)
-      const float4 w = make_float4(b * (vv.x - a * u.x), b * (vv.y - a * u.y),
-                                   b * (vv.z - a * u.z), b * (vv.w - a * u.w));
-      float4 op = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-      for (int ii = 0; ii < 8; ++ii) {
-        float4 s = S[ii];
-        s = make_float4(fmaf(kk[ii], w.x, a * s.x), fmaf(kk[ii], w.y, a * s.y),
-                        fmaf(kk[ii], w.z, a * s.z), fmaf(kk[ii], w.w, a * s.w));
-        S[ii] = s;
-        op = f4_fma(qq[ii], s, op);
+        for (int ii = 0; ii < 8; ++ii) {
+          float4 s = S[ii];
+          s = make_float4(fmaf(kk[ii], w.x, a * s.x), fmaf(kk[ii], w.y, a * s.y),
+                          fmaf(kk[ii], w.z, a * s.z), fmaf(kk[ii], w.w, a * s.w));
+          S[ii] = s;
+          op = f4_fma(qq[ii], s, op);
+        }
+        op = rows_sum(op, red, warp, lane);
+        if (warp == 0 && rg == 0) {
+          T* dst = o + (size_t(f) * Hl + h) * dv + col;
+          dst[0] = from_f32<T>(op.x * rs);
+          dst[1] = from_f32<T>(op.y * rs);
+          dst[2] = from_f32<T>(op.z * rs);
+          dst[3] = from_f32<T>(op.w * rs);
+        }
       }
-      op = rows_sum(op, red, warp, lane);
-      if (warp == 0 && rg == 0) {
-        T* dst = o + (size_t(f) * Hl + h) * dv + col;
-        dst[0] = from_f32<T>(op.x * rs);
-        dst[1] = from_f32<T>(op.y * rs);
-        dst[2] = from_f32<T>(op.z * rs);
-        dst[3] = from_f32<T>(op.w * rs);
-      }
-    }
-    if (s_fork) {
-      const size_t fhead = (size_t(c) * Hl + h) * kDK;
+      if (s_fork) {
+        const size_t fhead = (size_t(c) * Hl + h) * kDK;
 #pragma unroll
-      for (int ii = 0; ii < 8; ++ii) {
-        const int i = 32 * warp + rg + 4 * ii;
-        *reinterpret_cast<float4*>(s_fork + (fhead + i) * dv + col) = S[ii];
+        for (int ii = 0; ii < 8; ++ii) {
+          const int i = 32 * warp + rg + 4 * ii;
+          *reinterpret_cast<float4*>(s_fork + (fhead + i) * dv + col) = S[ii];
+        }
       }
     }
   }

@@ -76,6 +76,21 @@ def test_attention_cases(cuda, case):
     check_attention(lay, p, got["o"], list(range(p.N)), tol)
 
 
+def test_attention_longest_first_list_with_splits(cuda):
+    # Enough long prefixes that the planned chunk reaches 16 key tiles (1,088
+    # keys here: half of one SM's share of all tiles), so the persistent kernel
+    # takes its items from the longest-first work list, while every request
+    # still splits into several near-equal chunks (up to 15 for the longest).
+    pl = [8000] * 39 + [16000]
+    p = _custom("tiny", pl, [2] * 40, [1, 2] * 40, seed=50, Hq=8, Hkv=1, d=128, dtype="bf16")
+    got, _ = run_problem(cuda, p)
+    lay = oracle_layout(p)
+    rows = []
+    for r in (0, 17, 38, 39):
+        rows.extend(range(int(lay["row_offset"][r]), int(lay["row_offset"][r + 1])))
+    check_attention(lay, p, got["o"], rows, TOL_ATTN_BF16)
+
+
 # ---------------------------------------------------------------------------
 # LM head: ragged vocabulary and rows, targets at the vocabulary edges
 # ---------------------------------------------------------------------------
@@ -121,13 +136,25 @@ def test_all_vocabulary_targets_sum_to_one(cuda):
 # recurrent-state fork
 # ---------------------------------------------------------------------------
 @pytest.mark.parametrize("keep", [True, False])
-def test_fork_small(cuda, keep):
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_fork_small(cuda, keep, dtype):
     p = _custom("ordinal_hybrid", [3, 4, 2], [10, 3, 1], [1, 2, 3, 1, 1, 3, 2, 2, 1, 3, 4, 1, 6, 1],
-                seed=40, V=4096, D=256, Hl=3, dv=64)
+                seed=40, V=4096, D=256, Hl=3, dv=64, dtype=dtype)
     got, _ = run_problem(cuda, p, keep_fork=keep)
     lay = oracle_layout(p)
     check_fork(lay, p, got, list(range(p.R)))
     check_scores(lay, p, got, list(range(p.R)))
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_fork_long_candidates(cuda, dtype):
+    # candidates of up to 40 tokens: the 32-token window of fed tokens is
+    # staged again inside a candidate and across candidates
+    p = _custom("ordinal_hybrid", [5, 9], [4, 3], [20, 40, 1, 33, 7, 12, 2], seed=41, V=4096,
+                D=256, Hl=2, dv=96, dtype=dtype)
+    got, _ = run_problem(cuda, p)
+    lay = oracle_layout(p)
+    check_fork(lay, p, got, list(range(p.R)))
 
 
 # ---------------------------------------------------------------------------
