@@ -202,22 +202,25 @@ def _call(ms: float, nbytes: int, peaks) -> dict:
 
 def _attend_launches(problem, w) -> int:
     """Kernels jet_prefix_attend launches for this batch: the float32 path is
-    prefix + merge; the bf16 path is the tensor-core kernel plus a chunk
-    combine when any prefix spans more than one chunk (the library's plan:
-    about 608 CTAs, chunks of at least 256 keys)."""
+    prefix + merge; the bf16 path is the work-list kernel (or the counter
+    reset), the persistent tensor-core kernel and a chunk combine when the
+    plan splits the longest prefix (the library's plan: near-equal chunks of
+    at least 640 keys and no finer than half of one SM's share of the key
+    tiles over 152 SMs)."""
     if w.dtype != "bf16":
         return 2
     g = w.Hq // w.Hkv
     R, N = problem.R, problem.N
     max_prefix = int(problem.prefix_len.max())
+    total_prefix = int(problem.prefix_len.sum())
     avg_vecs = (N * g + R - 1) // R
     qv = max(1, 128 // g) * g  # whole rows of g heads per query block
     groups = R * w.Hkv * max(1, (avg_vecs + qv - 1) // qv)
-    splits = min(max(1, (608 + groups - 1) // groups), max(1, (max_prefix + 63) // 64))
-    chunk = (max_prefix + splits - 1) // splits
-    chunk = max(256, (chunk + 63) // 64 * 64)
+    share = groups * (total_prefix / R / 64.0 + 0.5) / 152
+    chunk = max(640, int(share / 2.0 + 0.999) * 64)
+    chunk = min(chunk, max(1, (max_prefix + 63) // 64) * 64)
     splits = (max_prefix + chunk - 1) // chunk
-    return 1 + (1 if splits > 1 else 0)
+    return 2 + (1 if splits > 1 else 0)
 
 
 def aggregate(total_ms: float, e2e_ms: float, R: int, steps: int, world: int, device=None):
