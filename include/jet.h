@@ -244,6 +244,46 @@ jet_status jet_score_candidates(const jet_layout* lay, const jet_dims* dims, con
                                 void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * Low-precision LM head. The paper runs its models with 8-bit (Q8_0) and
+ * 4-bit (Q4_K_M) weights (Appendix A); here a matrix row is stored as OCP FP8
+ * E4M3 codes (1 sign, 4 exponent bits with bias 7, 3 mantissa bits; largest
+ * finite value 448, no infinities) plus one float32 scale s, with
+ * x[k] ~= s * decode(q[k]).
+ *
+ * jet_quantize_rows_e4m3 - quantise the bf16 matrix x [rows, D] row by row:
+ * amax = max_k |x[k]| (float32), s = amax / 448, q[k] = e4m3(x[k] * (448 /
+ * amax)) rounded to nearest even and saturated at +-448; a row of zeros gets
+ * s = 0 and zero codes. q [rows, D] uint8, scale [rows] float32 (device,
+ * caller-owned). Errors: JET_ERR_ARG (rows < 0, null pointer), JET_ERR_SHAPE
+ * (D not a positive multiple of 16), JET_ERR_ALIGN. Used once for w_lm (model
+ * state); jet_score_candidates_e4m3 applies it to the hidden states itself.
+ */
+jet_status jet_quantize_rows_e4m3(const void* x, int32_t rows, int32_t D, uint8_t* q, float* scale,
+                                  void* stream);
+
+/* Workspace bytes of jet_prefix_attend and jet_score_candidates_e4m3 (the
+ * larger of the two). 0 on invalid arguments. */
+size_t jet_workspace_bytes_e4m3(const jet_sizes* n, const jet_dims* dims);
+
+/*
+ * jet_score_candidates_e4m3 - jet_score_candidates with an e4m3 LM head:
+ *   hidden      [N, D] bf16     quantised per row (token) into the workspace
+ *   w_q         [V, D] uint8    e4m3 codes of w_lm (jet_quantize_rows_e4m3)
+ *   w_scale     [V] float32     their per-row scales
+ *   tok_logprob, cand_score     as for jet_score_candidates
+ * The logit is z[n, v] = s_h[n] s_w[v] sum_k decode(h_q[n, k]) decode(w_q[v, k]),
+ * accumulated in float32 on the tensor cores (tcgen05 kind::f8f6f4); the
+ * log-softmax, gather and candidate sums are those of jet_score_candidates.
+ * dims.dtype must be JET_DTYPE_BF16 (else JET_ERR_UNSUPPORTED) and dims.D a
+ * multiple of 16 (else JET_ERR_SHAPE). ws/ws_bytes: scratch of at least
+ * jet_workspace_bytes_e4m3().
+ */
+jet_status jet_score_candidates_e4m3(const jet_layout* lay, const jet_dims* dims,
+                                     const void* hidden, const uint8_t* w_q, const float* w_scale,
+                                     float* tok_logprob, float* cand_score, void* ws,
+                                     size_t ws_bytes, void* stream);
+
+/*
  * jet_score_candidates_noalloc - jet_score_candidates without caller-owned
  * scratch memory. The paper has no counterpart to this entry point: it exists
  * for callers that cannot call cudaMalloc, such as a host application that

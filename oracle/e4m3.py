@@ -81,16 +81,21 @@ def e4m3_encode(y) -> np.ndarray:
     return codes.astype(np.uint8)
 
 
-def quantize_rows(x):
-    """(codes [rows, D] uint8, scale [rows] float32) of a float32 matrix."""
-    x = np.asarray(x, dtype=np.float32)
-    amax = np.max(np.abs(x), axis=1).astype(np.float32)
-    nz = amax > 0
-    inv = np.where(nz, np.float32(E4M3_MAX) / np.where(nz, amax, np.float32(1)),
-                   np.float32(0)).astype(np.float32)
-    y = (x * inv[:, None]).astype(np.float32)
-    codes = e4m3_encode(y)
-    scale = (amax / np.float32(E4M3_MAX)).astype(np.float32)
+def quantize_rows(x, block: int = 2048):
+    """(codes [rows, D] uint8, scale [rows] float32) of a float32 matrix; rows
+    are independent, so they are taken `block` at a time to bound memory."""
+    x = np.asarray(x)
+    codes = np.empty(x.shape, dtype=np.uint8)
+    scale = np.empty(x.shape[0], dtype=np.float32)
+    for r0 in range(0, x.shape[0], block):
+        xb = np.asarray(x[r0:r0 + block], dtype=np.float32)
+        amax = np.max(np.abs(xb), axis=1).astype(np.float32)
+        nz = amax > 0
+        inv = np.where(nz, np.float32(E4M3_MAX) / np.where(nz, amax, np.float32(1)),
+                       np.float32(0)).astype(np.float32)
+        y = (xb * inv[:, None]).astype(np.float32)
+        codes[r0:r0 + block] = e4m3_encode(y)
+        scale[r0:r0 + block] = (amax / np.float32(E4M3_MAX)).astype(np.float32)
     return codes, scale
 
 
@@ -99,9 +104,21 @@ def dequantize_rows(codes, scale) -> np.ndarray:
     return np.asarray(scale, dtype=np.float64)[:, None] * e4m3_decode(codes)
 
 
+class DequantizedRows:
+    """Read-only view of s[r] * decode(codes[r, :]) that dequantises the rows a
+    slice asks for (the full weight matrix would take 8 bytes per element)."""
+
+    def __init__(self, codes, scale):
+        self.codes, self.scale = codes, scale
+        self.shape = codes.shape
+
+    def __getitem__(self, rows):
+        return dequantize_rows(self.codes[rows], self.scale[rows])
+
+
 def token_logprobs_e4m3(lay, H, w_codes, w_scale, targets=None):
     """l_{c,t} (Eq. 1, Eq. 2) of the quantised LM head: the hidden states are
     quantised per token here, the weights come quantised per vocabulary row."""
     h_codes, h_scale = quantize_rows(H)
     return token_logprobs(lay, dequantize_rows(h_codes, h_scale),
-                          dequantize_rows(w_codes, w_scale), targets)
+                          DequantizedRows(w_codes, w_scale), targets)

@@ -102,6 +102,31 @@ jet_status check_fork_dims(const jet_dims* d) {
   return JET_OK;
 }
 
+jet_status check_e4m3_dims(const jet_dims* d) {
+  if (!d) return JET_ERR_ARG;
+  if (d->dtype != JET_DTYPE_BF16) return JET_ERR_UNSUPPORTED;
+  if (d->D < 16 || d->D % 16 != 0) return JET_ERR_SHAPE;
+  if (d->max_sms < 0) return JET_ERR_ARG;
+  return JET_OK;
+}
+
+// scratch of the e4m3 score path: the bf16 path's plan, then the hidden
+// states' codes [N, D] and scales [N]
+struct E4m3Plan {
+  jet::ScorePlan score;
+  size_t hq_off, hs_off, bytes;
+};
+
+E4m3Plan e4m3_plan(const jet_sizes& n, int D) {
+  auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
+  E4m3Plan p{};
+  p.score = jet::score_plan(n);
+  p.hq_off = up(p.score.bytes);
+  p.hs_off = p.hq_off + up(size_t(n.N) * size_t(D));
+  p.bytes = p.hs_off + up(size_t(n.N) * sizeof(float));
+  return p;
+}
+
 jet_status cuda_status(cudaError_t e) { return e == cudaSuccess ? JET_OK : JET_ERR_CUDA; }
 
 #define JET_TRY(expr)            \
@@ -206,6 +231,55 @@ extern "C" jet_status jet_score_candidates(const jet_layout* lay, const jet_dims
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   JET_TRY(cuda_status(jet::launch_lmhead(*lay, *dims, plan, hidden, w_lm, ws, status, st)));
   return cuda_status(jet::launch_score_finish(*lay, plan, ws, tok_logprob, cand_score, status, st));
+}
+
+extern "C" jet_status jet_quantize_rows_e4m3(const void* x, int32_t rows, int32_t D, uint8_t* q,
+                                             float* scale, void* stream) {
+  if (rows < 0) return JET_ERR_ARG;
+  if (D < 16 || D % 16 != 0) return JET_ERR_SHAPE;
+  if (rows == 0) return JET_OK;
+  JET_TRY(check_ptr(x, rows));
+  JET_TRY(check_ptr(q, rows));
+  JET_TRY(check_ptr(scale, rows));
+  return cuda_status(jet::launch_quantize_e4m3(x, rows, D, q, scale,
+                                               static_cast<cudaStream_t>(stream)));
+}
+
+extern "C" size_t jet_workspace_bytes_e4m3(const jet_sizes* n, const jet_dims* d) {
+  if (!n || !d || n->R < 0 || n->N < 0 || n->V < 1 || d->D < 16) return 0;
+  size_t a = 0;
+  if (d->Hq > 0 && d->Hkv > 0 && d->Hq % d->Hkv == 0 && d->d > 0) a = jet::attn_plan(*n, *d).bytes;
+  const size_t b = e4m3_plan(*n, d->D).bytes;
+  return a > b ? a : b;
+}
+
+extern "C" jet_status jet_score_candidates_e4m3(const jet_layout* lay, const jet_dims* dims,
+                                                const void* hidden, const uint8_t* w_q,
+                                                const float* w_scale, float* tok_logprob,
+                                                float* cand_score, void* ws, size_t ws_bytes,
+                                                void* stream) {
+  JET_TRY(check_layout(lay));
+  JET_TRY(check_e4m3_dims(dims));
+  const jet_sizes& n = lay->n;
+  if (n.R == 0) return JET_OK;
+  const E4m3Plan plan = e4m3_plan(n, dims->D);
+  if (plan.score.vtiles > 65535) return JET_ERR_CAPACITY;
+  JET_TRY(check_ptr(hidden, n.N));
+  JET_TRY(check_ptr(w_q, n.V));
+  JET_TRY(check_ptr(w_scale, n.V));
+  JET_TRY(check_ptr(tok_logprob, n.T));
+  JET_TRY(check_ptr(cand_score, n.C));
+  if (!ws || ws_bytes < plan.bytes) return JET_ERR_WORKSPACE;
+  if (!aligned16(ws)) return JET_ERR_ALIGN;
+  int* status = jet::device_status_ptr();
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint8_t* h_q = static_cast<uint8_t*>(ws) + plan.hq_off;
+  float* h_scale = reinterpret_cast<float*>(static_cast<char*>(ws) + plan.hs_off);
+  JET_TRY(cuda_status(jet::launch_quantize_e4m3(hidden, n.N, dims->D, h_q, h_scale, st)));
+  JET_TRY(cuda_status(jet::launch_lmhead_e4m3(*lay, *dims, plan.score, h_q, h_scale, w_q, w_scale,
+                                              ws, status, st)));
+  return cuda_status(
+      jet::launch_score_finish(*lay, plan.score, ws, tok_logprob, cand_score, status, st));
 }
 
 extern "C" jet_status jet_decide(const jet_layout* lay, int32_t mode, const float* cand_score,

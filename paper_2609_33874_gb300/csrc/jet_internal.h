@@ -81,6 +81,13 @@ cudaError_t launch_lmhead_simt(const jet_layout& lay, const jet_dims& d, const S
 cudaError_t launch_lmhead_tc(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
                              const void* hidden, const void* w_lm, void* ws, int* status,
                              cudaStream_t st);
+// e4m3 codes [N, D] / [V, D] with float32 scales per token / vocabulary row
+cudaError_t launch_lmhead_e4m3(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
+                               const uint8_t* h_q, const float* h_scale, const uint8_t* w_q,
+                               const float* w_scale, void* ws, int* status, cudaStream_t st);
+// per-row e4m3 quantisation of a bf16 matrix [rows, D] (D multiple of 16)
+cudaError_t launch_quantize_e4m3(const void* x, int rows, int D, uint8_t* q, float* scale,
+                                 cudaStream_t st);
 cudaError_t launch_lmhead(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
                           const void* hidden, const void* w_lm, void* ws, int* status,
                           cudaStream_t st);

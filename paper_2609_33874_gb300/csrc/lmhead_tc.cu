@@ -21,6 +21,12 @@
 //               partial per (token, vocabulary tile); target logits are read
 //               straight from TMEM.
 // Partials use base 2: m = max z log2(e), s = sum 2^(z log2(e) - m).
+//
+// The e4m3 instantiation (low-precision LM head; Appendix A: the paper's
+// models run with 8-bit and 4-bit weights) keeps the same byte geometry - a
+// 128-byte K slice is 128 e4m3 elements - issues tcgen05.mma kind::f8f6f4
+// (K = 32 per instruction) and applies the per-row weight scale and per-token
+// hidden scale to each logit in the epilogue: z = s_w[v] s_h[n] acc.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -37,7 +43,8 @@ namespace {
 using namespace sm100;
 
 constexpr int kBM = kVocabTile;     // 128 vocabulary rows per tile (MMA M, TMEM lanes)
-constexpr int kBK = 64;             // hidden elements per stage: 128 bytes of bf16
+constexpr int kBK = 64;             // bf16 hidden elements per stage: 128 bytes
+constexpr int kBKBytes = 128;       // bytes of one K slice of a row, either element type
 constexpr int kThreads = 192;
 constexpr int kMaxNt = 256;
 constexpr uint64_t kWaitNs = 2000000000ull;  // budget of one wait
@@ -45,7 +52,7 @@ constexpr uint64_t kDrainNs = 200000000ull;  // budget of the drain after an abo
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kNegBig = -1.0e30f;          // logit of a vocabulary row beyond V
 constexpr int kSmemLimit = 232448;           // opt-in shared memory per block
-constexpr int kFixedSmem = 4 * kMaxNt * 8 + 128 * 16 + 64 * 8 + 64;
+constexpr int kFixedSmem = 4 * kMaxNt * 8 + 128 * 16 + 64 * 8 + 64 + kMaxNt * 4;
 
 struct TcArgs {
   const int32_t* target_ids;
@@ -54,6 +61,8 @@ struct TcArgs {
   const int32_t* row_tgt_index;
   float2* part;
   float* z_tgt;
+  const float* w_scale;  // e4m3: [V] per vocabulary row
+  const float* h_scale;  // e4m3: [N] per token
   int* status;
   int N, T, V, D;
   int Nt, n_tt, units, nkb, stages, vtiles;
@@ -85,9 +94,28 @@ __device__ __forceinline__ void butterfly(float* m, float* s, int lane) {
   }
 }
 
+// D (+)= A B^T, A and B e4m3 codes described in shared memory (K = 32)
+__device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Instruction descriptor of kind::f8f6f4: A and B e4m3 (format 0, K-major),
+// f32 accumulator, shape M x N.
+constexpr uint32_t idesc_e4m3_f32(int M, int N) {
+  return (1u << 4) | (uint32_t(N >> 3) << 17) | (uint32_t(M >> 4) << 24);
+}
+
+template <bool F8>
 __global__ void __launch_bounds__(kThreads, 1)
 lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmH,
                  const TcArgs a) {
+  constexpr int kBKe = F8 ? kBKBytes : kBK;  // elements of one K slice
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -95,7 +123,8 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
   const uint32_t stage_bytes = a_bytes + b_bytes;
   float2* red = reinterpret_cast<float2*>(smem + size_t(a.stages) * stage_bytes);  // [4][256]
   int4* hits = reinterpret_cast<int4*>(red + 4 * kMaxNt);                          // [128]
-  uint64_t* full = reinterpret_cast<uint64_t*>(hits + 128);
+  float* hs = reinterpret_cast<float*>(hits + 128);                                // [256]
+  uint64_t* full = reinterpret_cast<uint64_t*>(hs + kMaxNt);
   uint64_t* empty = full + a.stages;
   uint64_t* tfull = empty + a.stages;
   uint64_t* tempty = tfull + 2;
@@ -152,8 +181,8 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
           }
           uint8_t* sa = smem + size_t(s) * stage_bytes;
           mbar_arrive_expect_tx(full + s, stage_bytes);
-          tma_load_2d(sa, &tmW, full + s, kb * kBK, v0, pol_w);
-          tma_load_2d(sa + a_bytes, &tmH, full + s, kb * kBK, t0, pol_h);
+          tma_load_2d(sa, &tmW, full + s, kb * kBKe, v0, pol_w);
+          tma_load_2d(sa + a_bytes, &tmH, full + s, kb * kBKe, t0, pol_h);
           issued |= 1u << s;
           issued_par = (issued_par & ~(1u << s)) | (ph << s);
           if (++s == a.stages) {
@@ -173,7 +202,7 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      const uint32_t idesc = idesc_bf16_f32(kBM, a.Nt);
+      const uint32_t idesc = F8 ? idesc_e4m3_f32(kBM, a.Nt) : idesc_bf16_f32(kBM, a.Nt);
       int s = 0, local = 0;
       uint32_t ph = 0;
       bool ok = true;
@@ -193,10 +222,16 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
           }
           tc_fence_after();
           const uint32_t sa = smem_u32(smem + size_t(s) * stage_bytes), sb = sa + a_bytes;
+          // 32 bytes of K per instruction: 16 bf16 or 32 e4m3 elements
 #pragma unroll
-          for (int k = 0; k < kBK / 16; ++k)
-            mma_f16(d_tmem, desc_k_sw128(sa + 32 * k), desc_k_sw128(sb + 32 * k), idesc,
-                    (kb | k) != 0);
+          for (int k = 0; k < kBKBytes / 32; ++k) {
+            if (F8)
+              mma_e4m3(d_tmem, desc_k_sw128(sa + 32 * k), desc_k_sw128(sb + 32 * k), idesc,
+                       (kb | k) != 0);
+            else
+              mma_f16(d_tmem, desc_k_sw128(sa + 32 * k), desc_k_sw128(sb + 32 * k), idesc,
+                      (kb | k) != 0);
+          }
           mma_commit(empty + s);  // frees the stage once these MMAs have read it
           if (++s == a.stages) {
             s = 0;
@@ -232,6 +267,14 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
       const uint32_t tcol = tmem_base + buf * buf_cols;
       const uint32_t tl = tcol + (uint32_t(32 * q) << 16);
       const int ncols = min(a.Nt, a.N - t0);
+      const bool row_valid = v0 + vrow < a.V;
+      // e4m3: this row's weight scale, and the unit's token scales in shared memory
+      float wsc = 1.f;
+      if (F8) {
+        wsc = row_valid ? a.w_scale[v0 + vrow] : 0.f;
+        for (int c = et; c < ncols; c += 128) hs[c] = a.h_scale[t0 + c];
+        named_bar_sync(1, 128);
+      }
 
       // target gather: rows [t0, t0 + ncols) whose target lies in this tile
       const int j_begin = a.row_tgt_offset[t0], j_end = a.row_tgt_offset[t0 + ncols];
@@ -259,18 +302,21 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
           if (hv.y == q) {
             const float z = tmem_ld_1col(tl + uint32_t(hv.w));
             tmem_wait_ld();
-            if (lane == hv.z) a.z_tgt[hv.x] = z;
+            if (lane == hv.z) a.z_tgt[hv.x] = F8 ? z * wsc * hs[hv.w] : z;
           }
         }
         named_bar_sync(1, 128);
       }
 
       // (max, sum 2^x) per token column over this warp's 32 vocabulary rows
-      const bool row_valid = v0 + vrow < a.V;
       for (int c0 = 0; c0 < ncols; c0 += 32) {
         float v[32];
         tmem_ld_32cols(tl + uint32_t(c0), v);
         tmem_wait_ld();
+        if (F8) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] *= wsc * hs[c0 + i];
+        }
         float m[16], s[16];
         {
           const bool up = (lane & 16) != 0;
@@ -330,17 +376,19 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// row-major [rows, D] bf16 matrix, box of 64 columns x box_rows rows, 128-byte swizzle
-bool encode_kmajor(CUtensorMap* map, const void* base, int rows, int D, int box_rows) {
+// row-major [rows, D] matrix of bf16 (esize 2) or e4m3 codes (esize 1), box of
+// one 128-byte K slice x box_rows rows, 128-byte swizzle
+bool encode_kmajor(CUtensorMap* map, const void* base, int rows, int D, int box_rows, int esize) {
   auto fn = encode_fn();
   if (!fn) return false;
   const cuuint64_t dims[2] = {cuuint64_t(D), cuuint64_t(rows)};
-  const cuuint64_t strides[1] = {cuuint64_t(D) * 2};
-  const cuuint32_t box[2] = {cuuint32_t(kBK), cuuint32_t(box_rows)};
+  const cuuint64_t strides[1] = {cuuint64_t(D) * esize};
+  const cuuint32_t box[2] = {cuuint32_t(kBKBytes / esize), cuuint32_t(box_rows)};
   const cuuint32_t estr[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
-            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  return fn(map, esize == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8, 2,
+            const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 int sm_count() {
@@ -352,13 +400,19 @@ int sm_count() {
 
 }  // namespace
 
-cudaError_t launch_lmhead_tc(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
-                             const void* hidden, const void* w_lm, void* ws, int* status,
-                             cudaStream_t st) {
+namespace {
+
+// one launch of the LM head on bf16 operands (F8 false) or e4m3 codes with
+// per-row weight scales and per-token hidden scales (F8 true)
+template <bool F8>
+cudaError_t launch_head(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
+                        const void* hidden, const float* h_scale, const void* w_lm,
+                        const float* w_scale, void* ws, int* status, cudaStream_t st) {
   const jet_sizes& n = lay.n;
   int n_tt = (n.N + kMaxNt - 1) / kMaxNt;
   const int Nt = ((n.N + n_tt - 1) / n_tt + 15) / 16 * 16;
   n_tt = (n.N + Nt - 1) / Nt;
+  const int esize = F8 ? 1 : 2;
   TcArgs a{};
   a.target_ids = lay.target_ids;
   a.tgt_row = lay.tgt_row;
@@ -367,6 +421,8 @@ cudaError_t launch_lmhead_tc(const jet_layout& lay, const jet_dims& d, const Sco
   char* base = static_cast<char*>(ws);
   a.part = reinterpret_cast<float2*>(base + plan.part_off);
   a.z_tgt = reinterpret_cast<float*>(base + plan.ztgt_off);
+  a.w_scale = w_scale;
+  a.h_scale = h_scale;
   a.status = status;
   a.N = n.N;
   a.T = n.T;
@@ -376,22 +432,37 @@ cudaError_t launch_lmhead_tc(const jet_layout& lay, const jet_dims& d, const Sco
   a.n_tt = n_tt;
   a.units = plan.vtiles * n_tt;
   a.vtiles = plan.vtiles;
-  a.nkb = (d.D + kBK - 1) / kBK;
+  a.nkb = (d.D * esize + kBKBytes - 1) / kBKBytes;
   a.tmem_cols = Nt <= 128 ? 256 : 512;
-  const int stage_bytes = kBM * 128 + Nt * 128;
+  const int stage_bytes = kBM * kBKBytes + Nt * kBKBytes;
   a.stages = std::min(8, (kSmemLimit - 1024 - kFixedSmem) / stage_bytes);
   const size_t smem = 1024 + size_t(a.stages) * stage_bytes + kFixedSmem;
 
   CUtensorMap tmW, tmH;
-  if (!encode_kmajor(&tmW, w_lm, n.V, d.D, kBM) || !encode_kmajor(&tmH, hidden, n.N, d.D, Nt))
+  if (!encode_kmajor(&tmW, w_lm, n.V, d.D, kBM, esize) ||
+      !encode_kmajor(&tmH, hidden, n.N, d.D, Nt, esize))
     return cudaErrorInvalidValue;
-  cudaError_t e = cudaFuncSetAttribute(lmhead_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       int(smem));
+  cudaError_t e = cudaFuncSetAttribute(lmhead_tc_kernel<F8>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
   if (e != cudaSuccess) return e;
   int sms = sm_count();
   if (d.max_sms > 0) sms = std::min(sms, d.max_sms);
   const int grid = std::max(1, std::min(a.units, sms));
-  return launch_pdl(lmhead_tc_kernel, dim3(grid), dim3(kThreads), smem, st, tmW, tmH, a);
+  return launch_pdl(lmhead_tc_kernel<F8>, dim3(grid), dim3(kThreads), smem, st, tmW, tmH, a);
+}
+
+}  // namespace
+
+cudaError_t launch_lmhead_tc(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
+                             const void* hidden, const void* w_lm, void* ws, int* status,
+                             cudaStream_t st) {
+  return launch_head<false>(lay, d, plan, hidden, nullptr, w_lm, nullptr, ws, status, st);
+}
+
+cudaError_t launch_lmhead_e4m3(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
+                               const uint8_t* h_q, const float* h_scale, const uint8_t* w_q,
+                               const float* w_scale, void* ws, int* status, cudaStream_t st) {
+  return launch_head<true>(lay, d, plan, h_q, h_scale, w_q, w_scale, ws, status, st);
 }
 
 }  // namespace jet

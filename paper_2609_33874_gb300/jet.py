@@ -83,6 +83,10 @@ def _load() -> ctypes.CDLL:
                                      P, P, P, P, P, SZ, P]),
         "jet_score_candidates_noalloc": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
                                              P, P, P, P, P]),
+        "jet_quantize_rows_e4m3": (I, [P, I, I, P, P, P]),
+        "jet_workspace_bytes_e4m3": (SZ, [ctypes.POINTER(jet_sizes), ctypes.POINTER(jet_dims)]),
+        "jet_score_candidates_e4m3": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
+                                          P, P, P, P, P, P, SZ, P]),
         "jet_decide": (I, [ctypes.POINTER(jet_layout), I, P, P, P, P, P]),
         "jet_device_status": (I, [P, ctypes.POINTER(ctypes.c_int32)]),
     }
@@ -96,8 +100,9 @@ def _load() -> ctypes.CDLL:
 _lib = _load()
 DECLARED = ("jet_abi_version", "jet_status_string", "jet_layout_plan", "jet_layout_words",
             "jet_layout_build", "jet_layout_bind", "jet_workspace_bytes", "jet_prefix_attend",
-            "jet_fork_state", "jet_score_candidates", "jet_score_candidates_noalloc", "jet_decide",
-            "jet_device_status")
+            "jet_fork_state", "jet_score_candidates", "jet_score_candidates_noalloc",
+            "jet_quantize_rows_e4m3", "jet_workspace_bytes_e4m3", "jet_score_candidates_e4m3",
+            "jet_decide", "jet_device_status")
 
 
 def library() -> ctypes.CDLL:
@@ -246,6 +251,28 @@ def jet_score_candidates_noalloc(layout, dims: jet_dims, hidden, w_lm, tok_logpr
                                              _addr(hidden), _addr(w_lm), _addr(tok_logprob),
                                              _addr(cand_score), _stream(stream)),
            "jet_score_candidates_noalloc")
+
+
+def jet_quantize_rows_e4m3(x, q, scale, stream=None) -> None:
+    """Per-row e4m3 codes q [rows, D] uint8 and scales [rows] float32 of the
+    bf16 matrix x [rows, D] (see include/jet.h)."""
+    rows, D = (int(x.shape[0]), int(x.shape[1])) if x.dim() == 2 else (0, 0)
+    _check(_lib.jet_quantize_rows_e4m3(_addr(x), rows, D, _addr(q), _addr(scale),
+                                       _stream(stream)), "jet_quantize_rows_e4m3")
+
+
+def jet_workspace_bytes_e4m3(sizes: jet_sizes, dims: jet_dims) -> int:
+    return int(_lib.jet_workspace_bytes_e4m3(ctypes.byref(sizes), ctypes.byref(dims)))
+
+
+def jet_score_candidates_e4m3(layout, dims: jet_dims, hidden, w_q, w_scale, tok_logprob,
+                              cand_score, ws, ws_bytes: Optional[int] = None, stream=None) -> None:
+    ws_bytes = ws.numel() * ws.element_size() if ws_bytes is None else ws_bytes
+    _check(_lib.jet_score_candidates_e4m3(ctypes.byref(_lay(layout)), ctypes.byref(dims),
+                                          _addr(hidden), _addr(w_q), _addr(w_scale),
+                                          _addr(tok_logprob), _addr(cand_score), _addr(ws),
+                                          int(ws_bytes), _stream(stream)),
+           "jet_score_candidates_e4m3")
 
 
 def jet_decide(layout, mode: int, cand_score, q, choice, value, stream=None) -> None:

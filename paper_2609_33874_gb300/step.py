@@ -27,6 +27,16 @@ RESULTS = ("tok_logprob", "cand_score", "q_cand", "choice", "value")
 _OVERLAP_MIN_BYTES = 1 << 20
 
 
+def quantize_lm_head(w_lm: torch.Tensor, stream=None):
+    """e4m3 codes [V, D] and per-row float32 scales [V] of the bf16 LM-head
+    weights (jet_quantize_rows_e4m3), for a step built with lm="e4m3"."""
+    V, D = w_lm.shape
+    w_q = torch.empty(V, D, dtype=torch.uint8, device=w_lm.device)
+    w_scale = torch.empty(V, dtype=torch.float32, device=w_lm.device)
+    jet.jet_quantize_rows_e4m3(w_lm, w_q, w_scale, stream=stream)
+    return w_q, w_scale
+
+
 class ScoringStep:
     """Device state of one batch shape.
 
@@ -34,12 +44,16 @@ class ScoringStep:
     ``mode`` one of ``jet.DECIDE_*``. ``hybrid`` adds the linear-attention
     fork; ``keep_fork_state`` also writes every candidate's final recurrent
     state. ``chain`` feeds the attention output to the LM head (requires
-    Hq * d == D).
+    Hq * d == D). ``lm`` selects the LM head: "bf16" (w_lm is the bf16 weight
+    matrix) or "e4m3" (w_lm is the pair returned by :func:`quantize_lm_head`).
     """
 
     def __init__(self, layout: "jet.HostLayout", dims: "jet.jet_dims", mode: int,
                  device="cuda", hybrid: bool = False, keep_fork_state: bool = False,
-                 chain: bool = False):
+                 chain: bool = False, lm: str = "bf16"):
+        if lm not in ("bf16", "e4m3"):
+            raise ValueError("lm must be 'bf16' or 'e4m3'")
+        self.lm = lm
         self.dev = torch.device(device)
         self.host_layout = layout
         self.layout = layout.to_device(self.dev)
@@ -57,7 +71,7 @@ class ScoringStep:
         self.q_cand = z(n.C)
         self.choice = z(n.R, dtype=torch.int32)
         self.value = z(n.R)
-        ws = jet.jet_workspace_bytes(n, dims)
+        ws = (jet.jet_workspace_bytes_e4m3 if lm == "e4m3" else jet.jet_workspace_bytes)(n, dims)
         self.ws = z((ws + 15) // 16 * 4)  # float32 words, 16-byte multiple
         if hybrid:
             self.lo = z(self.F, dims.Hl, dims.dv, dtype=dt)
@@ -82,10 +96,20 @@ class ScoringStep:
             jet.jet_fork_state(lay, d, x["s_prefix"], x["lq"], x["lk"], x["lv"], x["alpha"],
                                x["beta"], self.lo, self.s_fork, stream=stream)
         hidden = self.o.view(self.N, d.Hq * d.d) if self.chain else x["hidden"]
-        jet.jet_score_candidates(lay, d, hidden, w_lm, self.tok_logprob, self.cand_score, self.ws,
-                                 stream=stream)
+        self.score(hidden, w_lm, stream=stream, layout=lay)
         jet.jet_decide(lay, self.mode, self.cand_score, self.q_cand, self.choice, self.value,
                        stream=stream)
+
+    def score(self, hidden: torch.Tensor, w_lm, stream=None, layout=None) -> None:
+        """The LM-head call of the step (bf16 or e4m3, as the step was built)."""
+        lay = self.layout if layout is None else layout
+        if self.lm == "e4m3":
+            w_q, w_scale = w_lm
+            jet.jet_score_candidates_e4m3(lay, self.dims, hidden, w_q, w_scale, self.tok_logprob,
+                                          self.cand_score, self.ws, stream=stream)
+        else:
+            jet.jet_score_candidates(lay, self.dims, hidden, w_lm, self.tok_logprob,
+                                     self.cand_score, self.ws, stream=stream)
 
     def input_names(self):
         names = list(ATTN_INPUTS) + ([] if self.chain else ["hidden"])

@@ -184,6 +184,32 @@ def test_fork_validation(jet):
     assert lib.jet_fork_state(ctypes.byref(lay.struct), ctypes.byref(dims), *nul) == 1
 
 
+def test_e4m3_validation(jet):
+    lay, dims = _setup(jet)
+    lib = jet.library()
+    ws = jet.jet_workspace_bytes_e4m3(lay.sizes, dims)
+    assert ws > jet.jet_workspace_bytes(lay.sizes, jet.make_dims(jet.DTYPE_BF16, D=64)) - 1
+    # quantiser: shape, rows, null and alignment
+    assert lib.jet_quantize_rows_e4m3(FAKE, 4, 24, FAKE, FAKE, None) == 2   # D % 16 != 0
+    assert lib.jet_quantize_rows_e4m3(FAKE, -1, 64, FAKE, FAKE, None) == 1
+    assert lib.jet_quantize_rows_e4m3(None, 4, 64, FAKE, FAKE, None) == 1
+    assert lib.jet_quantize_rows_e4m3(FAKE, 4, 64, MIS, FAKE, None) == 4
+    assert lib.jet_quantize_rows_e4m3(FAKE, 0, 64, None, None, None) == 0  # nothing to do
+    # scoring: the e4m3 head takes bf16 hidden states and D % 16 == 0
+    f32 = jet.make_dims(jet.DTYPE_F32, D=64)
+    args = (FAKE, FAKE, FAKE, FAKE, FAKE, FAKE)
+    assert lib.jet_score_candidates_e4m3(ctypes.byref(lay.struct), ctypes.byref(f32), *args,
+                                         ws, None) == 7
+    bad = jet.make_dims(jet.DTYPE_BF16, D=72)
+    assert lib.jet_score_candidates_e4m3(ctypes.byref(lay.struct), ctypes.byref(bad), *args,
+                                         ws, None) == 2
+    assert lib.jet_score_candidates_e4m3(ctypes.byref(lay.struct), ctypes.byref(dims), *args,
+                                         64, None) == 5
+    mis = (FAKE, MIS, FAKE, FAKE, FAKE, FAKE)  # w_q
+    assert lib.jet_score_candidates_e4m3(ctypes.byref(lay.struct), ctypes.byref(dims), *mis,
+                                         ws, None) == 4
+
+
 def test_empty_batch_is_a_no_op(jet):
     lay = jet.jet_layout_build([], [], [], [], 16)
     assert lay.sizes.R == 0 and lay.sizes.N == 0
