@@ -35,6 +35,9 @@ What each function computes, and where the paper defines it:
   Eq. 5 with the decision rules of Sec. 3.3 (argmax with ties to the lowest
   index, binary q(true) with C = {false, true}, ordinal expected zero-based
   index).
+* :func:`evaluate` - gold negative log-likelihood with the probabilities of
+  labels that carry the gold answer text summed (Sec. 3.3), and agreement of
+  the choice with the gold answer (Sec. 5.1).
 """
 from __future__ import annotations
 
@@ -44,7 +47,7 @@ from typing import Dict
 import numpy as np
 
 __all__ = ["build_layout", "cascade_attention", "fork_state", "token_logprobs",
-           "candidate_scores", "decide", "score_step"]
+           "candidate_scores", "decide", "evaluate", "score_step"]
 
 ARGMAX, BINARY, ORDINAL = 0, 1, 2
 
@@ -317,6 +320,31 @@ def decide(lay, s, mode: int):
         else:
             value[r] = qr[best]
     return q, choice, value
+
+
+# ----------------------------------------------------------------------------
+# evaluation: gold negative log-likelihood and agreement (Sec. 3.3, Sec. 5.1)
+# ----------------------------------------------------------------------------
+def evaluate(lay, s, choice, gold):
+    """Per request, with q from Eq. 4 and gold[c] true for every candidate
+    whose label carries the gold answer text: nll = -log sum_{gold c} q(c)
+    (equivalent labels' probabilities are summed, Sec. 3.3; infinite when no
+    candidate is gold), correct = gold[choice] (any label with the gold text
+    is accepted; for binary requests the choice is the argmax of {false,
+    true}, i.e. q(true) > 1/2, Sec. 5.1)."""
+    R = lay["R"]
+    nll = np.zeros(R, np.float64)
+    correct = np.zeros(R, np.int32)
+    for r in range(R):
+        c0, c1 = int(lay["cand_offset"][r]), int(lay["cand_offset"][r + 1])
+        sr = np.asarray(s[c0:c1], np.float64)
+        e = np.exp(sr - sr.max())
+        qr = e / e.sum()
+        g = np.asarray(gold[c0:c1], bool)
+        pg = qr[g].sum()
+        nll[r] = -math.log(pg) if pg > 0 else math.inf
+        correct[r] = int(g[int(choice[r])])
+    return nll, correct
 
 
 def score_step(lay, H, W, mode: int):

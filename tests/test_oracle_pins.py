@@ -458,3 +458,48 @@ def test_fork_equals_fresh_recurrence_and_is_isolated():
     for i, c in enumerate(order):
         assert np.array_equal(s_r[i], s_fork[c])
     np.testing.assert_array_equal(o_r, o[perm])
+
+
+# ---------------------------------------------------------------------------
+# evaluation helpers: gold NLL over equivalent labels, agreement
+# ---------------------------------------------------------------------------
+def _eval_layout(n_cand):
+    cand_len = [1] * int(sum(n_cand))
+    return O.build_layout([4] * len(n_cand), n_cand, cand_len, list(range(len(cand_len))), 64)
+
+
+def test_evaluate_closed_forms():
+    lay = _eval_layout([2, 2, 3, 2, 4])
+    s = np.array([0.0, 0.0,            # equal scores, one gold: nll = log 2
+                  -1.0, -3.0,          # both gold: nll = 0
+                  1.0, 2.0, 3.0,       # gold = the two lowest: -log((e+e^2)/(e+e^2+e^3))
+                  5.0, 5.0,            # no gold: infinite
+                  -2.0, 0.5, 0.5, -9.0])  # gold = two tied maxima, choice = first of them
+    gold = np.array([0, 1, 1, 1, 1, 1, 0, 0, 0, 0, 1, 1, 0], bool)
+    q, choice, _ = O.decide(lay, s, O.ARGMAX)
+    nll, correct = O.evaluate(lay, s, choice, gold)
+    assert abs(nll[0] - math.log(2)) < 1e-15 and abs(nll[1]) < 1e-15
+    e = np.exp([1.0, 2.0, 3.0])
+    assert abs(nll[2] + math.log((e[0] + e[1]) / e.sum())) < 1e-14
+    assert nll[3] == math.inf
+    assert abs(nll[4] + math.log(q[10] + q[11])) < 1e-14
+    # choice: ties to the lowest index; accepted when that label is gold
+    np.testing.assert_array_equal(choice, [0, 0, 2, 0, 1])
+    np.testing.assert_array_equal(correct, [0, 1, 0, 0, 1])
+
+
+def test_evaluate_singleton_gold_is_minus_log_q_and_shift_invariant():
+    rng = np.random.default_rng(9)
+    lay = _eval_layout([5, 3, 7])
+    s = rng.normal(0, 4, lay["C"])
+    gold = np.zeros(lay["C"], bool)
+    gold[[2, 6, 12]] = True
+    q, choice, _ = O.decide(lay, s, O.ARGMAX)
+    nll, _ = O.evaluate(lay, s, choice, gold)
+    np.testing.assert_allclose(nll, -np.log(q[[2, 6, 12]]), rtol=1e-13)
+    nll2, _ = O.evaluate(lay, s + 123.0, choice, gold)
+    np.testing.assert_allclose(nll2, nll, rtol=1e-12)
+    # gold = every candidate: probability one
+    nll3, correct3 = O.evaluate(lay, s, choice, np.ones(lay["C"], bool))
+    np.testing.assert_allclose(nll3, 0.0, atol=1e-14)
+    assert correct3.all()
