@@ -345,6 +345,25 @@ def run_gpu(args):
     call_ms = {name: statistics.mean(ev[k].elapsed_time(ev[k + 1]) for ev in call_ev)
                for k, name in enumerate(("attend", "fork", "score", "decide"))}
 
+    # --- evaluation helper (after the step, outside it): gold NLL + agreement,
+    # with every request's first candidate taken as the gold label
+    gold = torch.zeros(step.C, dtype=torch.uint8, device=dev)
+    gold[torch.as_tensor(hl.array("cand_offset")[:-1], dtype=torch.long, device=dev)] = 1
+    nll = torch.empty(step.R, dtype=torch.float32, device=dev)
+    correct = torch.empty(step.R, dtype=torch.int32, device=dev)
+    ev_a, ev_b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n_eval = 20
+    with torch.cuda.stream(stream):
+        jet.jet_evaluate(step.layout, step.cand_score, step.choice, gold, nll, correct,
+                         stream=stream)
+        ev_a.record(stream)
+        for _ in range(n_eval):
+            jet.jet_evaluate(step.layout, step.cand_score, step.choice, gold, nll, correct,
+                             stream=stream)
+        ev_b.record(stream)
+    torch.cuda.synchronize(dev)
+    call_ms["evaluate"] = ev_a.elapsed_time(ev_b) / n_eval
+
     # --- end to end: pinned host inputs, copies inside the timed region ---------
     host = {k: x[k].cpu().pin_memory() for k in names}
     words = torch.from_numpy(hl.words).pin_memory()
@@ -415,7 +434,10 @@ def run_gpu(args):
     calls = dict(attend=_call(call_ms["attend"], attn_bytes, peaks),
                  score=dict(ms=round(call_ms["score"], 4), bound=roof["bound"],
                             frac=roof["frac"]),
-                 decide=dict(ms=round(call_ms["decide"], 4)))
+                 decide=dict(ms=round(call_ms["decide"], 4)),
+                 evaluate=dict(ms=round(call_ms["evaluate"], 4),
+                               note="outside the step: gold NLL over equivalent labels and "
+                                    "agreement, back to back"))
     if w.Hl:
         fork_bytes = (R * w.Hl * w.dk * w.dv * 4 + len(problem.cand_len) * w.Hl * w.dk * w.dv * 4
                       + F * w.Hl * (2 * w.dk + 2 * w.dv) * es + F * w.Hl * 8)

@@ -244,6 +244,23 @@ jet_status jet_score_candidates(const jet_layout* lay, const jet_dims* dims, con
                                 void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * jet_evaluate - evaluation against a gold answer (Sec. 3.3, Sec. 5.1).
+ *   cand_score [C] float32  s(c|x) (jet_score_candidates)
+ *   choice     [R] int32    the chosen candidate of each request (jet_decide)
+ *   gold       [C] uint8    nonzero for every candidate whose label carries
+ *                           the gold answer text (several labels may)
+ *   nll        [R] float32  -log sum_{gold c} q(c), q from Eq. 4: the
+ *                           probabilities of equivalent labels are summed;
+ *                           +infinity when no candidate of the request is gold
+ *   correct    [R] int32    1 when the chosen label carries the gold text
+ * For binary requests the choice is the argmax of {false, true}, i.e. q(true)
+ * thresholded at 1/2 with a tie going to false. Batch accuracy and mean NLL
+ * are the caller's sums over requests.
+ */
+jet_status jet_evaluate(const jet_layout* lay, const float* cand_score, const int32_t* choice,
+                        const uint8_t* gold, float* nll, int32_t* correct, void* stream);
+
+/*
  * Low-precision LM head. The paper runs its models with 8-bit (Q8_0) and
  * 4-bit (Q4_K_M) weights (Appendix A); here a matrix row is stored as OCP FP8
  * E4M3 codes (1 sign, 4 exponent bits with bias 7, 3 mantissa bits; largest

@@ -332,17 +332,21 @@ def evaluate(lay, s, choice, gold):
     candidate is gold), correct = gold[choice] (any label with the gold text
     is accepted; for binary requests the choice is the argmax of {false,
     true}, i.e. q(true) > 1/2, Sec. 5.1)."""
+    def logsumexp(x):
+        m = x.max()
+        return m + math.log(np.exp(x - m).sum())
+
     R = lay["R"]
     nll = np.zeros(R, np.float64)
     correct = np.zeros(R, np.int32)
     for r in range(R):
         c0, c1 = int(lay["cand_offset"][r]), int(lay["cand_offset"][r + 1])
         sr = np.asarray(s[c0:c1], np.float64)
-        e = np.exp(sr - sr.max())
-        qr = e / e.sum()
         g = np.asarray(gold[c0:c1], bool)
-        pg = qr[g].sum()
-        nll[r] = -math.log(pg) if pg > 0 else math.inf
+        # -log sum_{gold} q(c) with q = e^(s_c) / sum_d e^(s_d) (Eq. 4), written
+        # as the difference of two log-sum-exps so that it stays exact where
+        # q itself would underflow
+        nll[r] = logsumexp(sr) - logsumexp(sr[g]) if g.any() else math.inf
         correct[r] = int(g[int(choice[r])])
     return nll, correct
 

@@ -299,6 +299,22 @@ extern "C" jet_status jet_decide(const jet_layout* lay, int32_t mode, const floa
                                         static_cast<cudaStream_t>(stream)));
 }
 
+extern "C" jet_status jet_evaluate(const jet_layout* lay, const float* cand_score,
+                                   const int32_t* choice, const uint8_t* gold, float* nll,
+                                   int32_t* correct, void* stream) {
+  JET_TRY(check_layout(lay));
+  const jet_sizes& n = lay->n;
+  if (n.R == 0) return JET_OK;
+  JET_TRY(check_ptr(cand_score, n.C));
+  JET_TRY(check_ptr(choice, n.R));
+  JET_TRY(check_ptr(gold, n.C));
+  JET_TRY(check_ptr(nll, n.R));
+  JET_TRY(check_ptr(correct, n.R));
+  return cuda_status(jet::launch_evaluate(*lay, cand_score, choice, gold, nll, correct,
+                                          jet::device_status_ptr(),
+                                          static_cast<cudaStream_t>(stream)));
+}
+
 extern "C" jet_status jet_device_status(void* stream, jet_status* out) {
   if (!out) return JET_ERR_ARG;
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return JET_ERR_CUDA;

@@ -97,6 +97,10 @@ cudaError_t launch_score_finish(const jet_layout& lay, const ScorePlan& plan, vo
                                 float* tok_logprob, float* cand_score, int* status,
                                 cudaStream_t st);
 
+cudaError_t launch_evaluate(const jet_layout& lay, const float* cand_score, const int32_t* choice,
+                            const uint8_t* gold, float* nll, int32_t* correct, int* status,
+                            cudaStream_t st);
+
 cudaError_t launch_decide(const jet_layout& lay, int mode, const float* cand_score, float* q,
                           int32_t* choice, float* value, int* status, cudaStream_t st);
 

@@ -7,6 +7,8 @@
 //   s(c|x)  = sum_t l_{c,t}, summed in t order                (Eq. 3)
 //   q(c)    = exp(s_c - M) / sum_d exp(s_d - M), M = max s     (Eq. 4)
 //   choice  = argmax_c s_c, ties to the lowest index          (Eq. 5, Sec. 3.3)
+//   nll     = -log sum_{c: gold label text} q(c)               (Sec. 3.3, Sec. 5.1)
+//   correct = the chosen label carries the gold answer text    (Sec. 5.1)
 #include "jet_device.cuh"
 #include "jet_internal.h"
 
@@ -123,6 +125,52 @@ decide_kernel(const int32_t* __restrict__ cand_offset, int R, int C, int mode,
   }
 }
 
+// one warp per request: nll = lse(all s) - lse(gold s), each log-sum-exp
+// shifted by its own maximum, so a gold probability far below float32's
+// range still gives a finite value
+__global__ void __launch_bounds__(256)
+evaluate_kernel(const int32_t* __restrict__ cand_offset, int R, int C,
+                const float* __restrict__ s, const int32_t* __restrict__ choice,
+                const uint8_t* __restrict__ gold, float* __restrict__ nll,
+                int32_t* __restrict__ correct, int* status) {
+  pdl_begin();
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (r >= R) return;
+  const int c0 = cand_offset[r], c1 = cand_offset[r + 1];
+  if (c0 < 0 || c1 <= c0 || c1 > C) {
+    if (lane == 0) flag(status, JET_ERR_DEVICE);
+    return;
+  }
+  float M = -INFINITY, Mg = -INFINITY;
+  for (int c = c0 + lane; c < c1; c += 32) {
+    M = fmaxf(M, s[c]);
+    if (gold[c]) Mg = fmaxf(Mg, s[c]);
+  }
+  M = warp_max(M);
+  Mg = warp_max(Mg);
+  float all = 0.f, in_gold = 0.f;
+  for (int c = c0 + lane; c < c1; c += 32) {
+    all += expf(s[c] - M);
+    if (gold[c]) in_gold += expf(s[c] - Mg);
+  }
+  all = warp_sum(all);
+  in_gold = warp_sum(in_gold);
+  if (lane == 0) {
+    // no gold candidate: Mg = -inf and the gold probability is zero
+    // (M - Mg) first: exact for nearby maxima, it keeps the offset of the
+    // scores out of the rounding of the small log terms
+    nll[r] = Mg > -INFINITY ? (M - Mg) + (logf(all) - logf(in_gold)) : INFINITY;
+    const int k = choice[r];
+    if (k < 0 || k >= c1 - c0) {
+      flag(status, JET_ERR_DEVICE);
+      correct[r] = 0;
+    } else {
+      correct[r] = gold[c0 + k] ? 1 : 0;
+    }
+  }
+}
+
 }  // namespace
 
 ScorePlan score_plan(const jet_sizes& n) {
@@ -150,6 +198,14 @@ cudaError_t launch_score_finish(const jet_layout& lay, const ScorePlan& plan, vo
   return launch_pdl(finish_kernel, dim3(unsigned((n.C + 127) / 128)), dim3(128), 0, st,
                     lay.tgt_offset, lay.tgt_row, n.C, n.N, n.T, z_tgt, lse, tok_logprob,
                     cand_score, status);
+}
+
+cudaError_t launch_evaluate(const jet_layout& lay, const float* cand_score, const int32_t* choice,
+                            const uint8_t* gold, float* nll, int32_t* correct, int* status,
+                            cudaStream_t st) {
+  const jet_sizes& n = lay.n;
+  return launch_pdl(evaluate_kernel, dim3(unsigned((n.R + 7) / 8)), dim3(256), 0, st,
+                    lay.cand_offset, n.R, n.C, cand_score, choice, gold, nll, correct, status);
 }
 
 cudaError_t launch_decide(const jet_layout& lay, int mode, const float* cand_score, float* q,

@@ -88,6 +88,7 @@ def _load() -> ctypes.CDLL:
         "jet_score_candidates_e4m3": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
                                           P, P, P, P, P, P, SZ, P]),
         "jet_decide": (I, [ctypes.POINTER(jet_layout), I, P, P, P, P, P]),
+        "jet_evaluate": (I, [ctypes.POINTER(jet_layout), P, P, P, P, P, P]),
         "jet_device_status": (I, [P, ctypes.POINTER(ctypes.c_int32)]),
     }
     for name, (res, args) in sig.items():
@@ -102,7 +103,7 @@ DECLARED = ("jet_abi_version", "jet_status_string", "jet_layout_plan", "jet_layo
             "jet_layout_build", "jet_layout_bind", "jet_workspace_bytes", "jet_prefix_attend",
             "jet_fork_state", "jet_score_candidates", "jet_score_candidates_noalloc",
             "jet_quantize_rows_e4m3", "jet_workspace_bytes_e4m3", "jet_score_candidates_e4m3",
-            "jet_decide", "jet_device_status")
+            "jet_decide", "jet_evaluate", "jet_device_status")
 
 
 def library() -> ctypes.CDLL:
@@ -278,6 +279,13 @@ def jet_score_candidates_e4m3(layout, dims: jet_dims, hidden, w_q, w_scale, tok_
 def jet_decide(layout, mode: int, cand_score, q, choice, value, stream=None) -> None:
     _check(_lib.jet_decide(ctypes.byref(_lay(layout)), int(mode), _addr(cand_score), _addr(q),
                            _addr(choice), _addr(value), _stream(stream)), "jet_decide")
+
+
+def jet_evaluate(layout, cand_score, choice, gold, nll, correct, stream=None) -> None:
+    """Gold NLL over equivalent labels and agreement of the choice (see include/jet.h)."""
+    _check(_lib.jet_evaluate(ctypes.byref(_lay(layout)), _addr(cand_score), _addr(choice),
+                             _addr(gold), _addr(nll), _addr(correct), _stream(stream)),
+           "jet_evaluate")
 
 
 def jet_device_status(stream=None) -> int:

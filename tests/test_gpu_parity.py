@@ -276,3 +276,42 @@ def test_end_to_end_pipelined(cuda, overlap):
                    q=out["q_cand"].numpy(), choice=out["choice"].numpy(),
                    value=out["value"].numpy())
         check_scores(oracle_layout(p), p, got, range(len(p.prefix_len)), w_lm=W)
+
+
+# ---------------------------------------------------------------------------
+# evaluation helpers: gold NLL over equivalent labels, agreement
+# ---------------------------------------------------------------------------
+def test_evaluate_against_oracle(cuda):
+    import torch
+    rng = np.random.default_rng(80)
+    R = 300
+    n_cand = rng.integers(1, 40, size=R)
+    C = int(n_cand.sum())
+    hl = cuda.jet_layout_build([4] * R, n_cand, [1] * C, rng.integers(0, 64, size=C), 64)
+    lay = O.build_layout([4] * R, n_cand, [1] * C, hl.array("target_ids"), 64)
+    # scores with request-wide offsets up to 1e3, repeated values (ties) and
+    # requests without any gold label
+    s = (rng.normal(0, 5, C) + np.repeat(rng.uniform(-1e3, 1e3, R), n_cand)).astype(np.float32)
+    s[rng.random(C) < 0.1] = np.float32(7.0)
+    gold = (rng.random(C) < 0.3).astype(np.uint8)
+    gold[: n_cand[0]] = 0
+    dl = hl.to_device("cuda")
+    d_s = torch.from_numpy(s).cuda()
+    q = torch.empty(C, device="cuda")
+    choice = torch.empty(R, dtype=torch.int32, device="cuda")
+    value = torch.empty(R, device="cuda")
+    cuda.jet_decide(dl, cuda.DECIDE_ARGMAX, d_s, q, choice, value)
+    nll = torch.empty(R, device="cuda")
+    correct = torch.empty(R, dtype=torch.int32, device="cuda")
+    cuda.jet_evaluate(dl, d_s, choice, torch.from_numpy(gold).cuda(), nll, correct)
+    torch.cuda.synchronize()
+    assert cuda.jet_device_status() == 0
+    _, ref_choice, _ = O.decide(lay, s.astype(np.float64), O.ARGMAX)
+    np.testing.assert_array_equal(choice.cpu().numpy(), ref_choice)
+    ref_nll, ref_correct = O.evaluate(lay, s.astype(np.float64), ref_choice, gold.astype(bool))
+    got = nll.cpu().numpy().astype(np.float64)
+    inf = np.isinf(ref_nll)
+    assert inf.any() and np.array_equal(np.isinf(got), inf)
+    np.testing.assert_allclose(got[~inf], ref_nll[~inf], rtol=1e-5, atol=2e-5)
+    assert ref_nll[~inf].max() > 200.0   # gold probabilities below float32's range stay finite
+    np.testing.assert_array_equal(correct.cpu().numpy(), ref_correct)
