@@ -27,6 +27,9 @@ What each function computes, and where the paper defines it:
   prefix state before each candidate"; Sec. 5.6). The recurrence itself is not
   given by the paper; the reading used is the gated delta rule
   S <- alpha (S - beta k (k^T S)) + beta k v^T, read out as o = S^T q / sqrt(dk).
+  ``rule="gla"`` selects the plain gated linear-attention variant
+  S <- alpha S + beta k v^T (no erase term), the other recurrence the hybrid
+  models of the paper's family use.
 * :func:`token_logprobs` - Eq. 1 and Eq. 2: log-softmax over the full
   vocabulary, evaluated at the target token.
 * :func:`candidate_scores` - Eq. 3: s(c|x) = sum_t l_{c,t}, no length
@@ -213,14 +216,26 @@ def gated_delta_step(S, q, k, v, alpha, beta):
     return S, (S.T @ q) / math.sqrt(S.shape[0])
 
 
-def fork_state(lay, s_prefix, lq, lk, lv, alpha, beta):
+def gated_linear_step(S, q, k, v, alpha, beta):
+    """The plain gated linear-attention variant of the step: decay and write,
+    S <- alpha S + beta k v^T, without the delta rule's erase term."""
+    S = alpha * S + beta * np.outer(k, v)
+    return S, (S.T @ q) / math.sqrt(S.shape[0])
+
+
+RULES = {"delta": gated_delta_step, "gla": gated_linear_step}
+
+
+def fork_state(lay, s_prefix, lq, lk, lv, alpha, beta, rule: str = "delta"):
     """Per candidate: restore the unchanged prefix state S_r, then feed the
     candidate's tokens y_{c,1..m_c-1} (Sec. 4.1).
 
     Returns (o[F, Hl, dv], s_fork[C, Hl, dk, dv]) where F = N - R fed tokens in
     row order and s_fork is each candidate's state after its last fed token
-    (a copy of S_r when m_c = 1).
+    (a copy of S_r when m_c = 1). ``rule`` names the recurrence: "delta" (the
+    gated delta rule) or "gla" (plain gated linear attention).
     """
+    step = RULES[rule]
     s_prefix = np.asarray(s_prefix, np.float64)
     R, Hl, dk, dv = s_prefix.shape
     C, N = lay["C"], lay["N"]
@@ -234,7 +249,7 @@ def fork_state(lay, s_prefix, lq, lk, lv, alpha, beta):
                 S = s_prefix[r, h].copy()          # restore the prefix state
                 for t in range(1, m):
                     f = _fed_index(lay, first + t - 1)
-                    S, o[f, h] = gated_delta_step(
+                    S, o[f, h] = step(
                         S, np.asarray(lq[f, h], np.float64), np.asarray(lk[f, h], np.float64),
                         np.asarray(lv[f, h], np.float64), float(alpha[f, h]), float(beta[f, h]))
                 s_fork[c, h] = S

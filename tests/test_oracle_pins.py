@@ -503,3 +503,53 @@ def test_evaluate_singleton_gold_is_minus_log_q_and_shift_invariant():
     nll3, correct3 = O.evaluate(lay, s, choice, np.ones(lay["C"], bool))
     np.testing.assert_allclose(nll3, 0.0, atol=1e-14)
     assert correct3.all()
+
+
+# ---------------------------------------------------------------------------
+# recurrence variant: plain gated linear attention
+# ---------------------------------------------------------------------------
+def test_gla_closed_form_from_zero_state():
+    # S_T = sum_t (prod_{s>t} alpha_s) beta_t k_t v_t^T from S_0 = 0
+    rng = np.random.default_rng(31)
+    dk, dv, Tn = 8, 5, 6
+    k = rng.normal(size=(Tn, dk)); v = rng.normal(size=(Tn, dv)); q = rng.normal(size=(Tn, dk))
+    a = rng.uniform(0.9, 1.0, Tn); b = rng.uniform(0, 1, Tn)
+    S = np.zeros((dk, dv))
+    for t in range(Tn):
+        S, o = O.gated_linear_step(S, q[t], k[t], v[t], a[t], b[t])
+    ref = sum(np.prod(a[t + 1:]) * b[t] * np.outer(k[t], v[t]) for t in range(Tn))
+    np.testing.assert_allclose(S, ref, rtol=1e-13, atol=1e-14)
+    np.testing.assert_allclose(o, ref.T @ q[-1] / math.sqrt(dk), rtol=1e-12)
+
+
+def test_gla_and_delta_agree_only_without_overlap():
+    # the two rules coincide when the key is orthogonal to what the state holds
+    dk, dv = 6, 3
+    S0 = np.zeros((dk, dv)); S0[:3] = np.arange(9.0).reshape(3, 3)
+    k = np.zeros(dk); k[4] = 1.0
+    v = np.array([1.0, -2.0, 0.5]); q = np.ones(dk)
+    d1, _ = O.gated_delta_step(S0, q, k, v, 0.95, 0.7)
+    g1, _ = O.gated_linear_step(S0, q, k, v, 0.95, 0.7)
+    np.testing.assert_allclose(d1, g1, rtol=0, atol=1e-15)
+    k2 = np.zeros(dk); k2[1] = 1.0            # overlaps row 1 of the state
+    d2, _ = O.gated_delta_step(S0, q, k2, v, 0.95, 0.7)
+    g2, _ = O.gated_linear_step(S0, q, k2, v, 0.95, 0.7)
+    # delta erases beta of the old row before writing; gla only adds
+    np.testing.assert_allclose(g2[1] - d2[1], 0.95 * 0.7 * S0[1], rtol=1e-14)
+
+
+def test_fork_rule_selects_the_recurrence():
+    lay = O.build_layout([3, 2], [2, 1], [3, 1, 2], [1, 2, 3, 4, 5, 6], 8)
+    rng = np.random.default_rng(33)
+    R, F, Hl, dk, dv = 2, lay["N"] - 2, 2, 4, 3
+    sp = rng.normal(size=(R, Hl, dk, dv))
+    lq, lk, lv = (rng.normal(size=(F, Hl, n)) for n in (dk, dk, dv))
+    al, be = rng.uniform(0.9, 1, (F, Hl)), rng.uniform(0, 1, (F, Hl))
+    od, sd = O.fork_state(lay, sp, lq, lk, lv, al, be)
+    og, sg = O.fork_state(lay, sp, lq, lk, lv, al, be, rule="gla")
+    assert not np.allclose(sd, sg)
+    # candidate 0 of request 0 feeds fed tokens 0, 1 (m = 3): replay it by hand
+    S = sp[0, 1].copy()
+    for f in (0, 1):
+        S = al[f, 1] * S + be[f, 1] * np.outer(lk[f, 1], lv[f, 1])
+    np.testing.assert_allclose(sg[0, 1], S, rtol=1e-13)
