@@ -28,8 +28,8 @@ What each function computes, and where the paper defines it:
   given by the paper; the reading used is the gated delta rule
   S <- alpha (S - beta k (k^T S)) + beta k v^T, read out as o = S^T q / sqrt(dk).
   ``rule="gla"`` selects the plain gated linear-attention variant
-  S <- alpha S + beta k v^T (no erase term), the other recurrence the hybrid
-  models of the paper's family use.
+  S <- alpha S + beta k v^T (no erase term), a second reading of the
+  unnamed recurrence.
 * :func:`token_logprobs` - Eq. 1 and Eq. 2: log-softmax over the full
   vocabulary, evaluated at the target token.
 * :func:`candidate_scores` - Eq. 3: s(c|x) = sum_t l_{c,t}, no length
