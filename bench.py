@@ -276,7 +276,7 @@ def run_gpu(args):
                               problem.target_ids, w.V)
     e4m3 = args.lm == "e4m3"
     step = ScoringStep(hl, dims, jet.MODES[w.mode], device=dev, hybrid=w.Hl > 0,
-                       keep_fork_state=w.Hl > 0, lm=args.lm)
+                       keep_fork_state=w.Hl > 0, lm=args.lm, rule=args.rule)
     names = step.input_names()
     x = {k: jet_synth.torch_tensor(problem, k, device=dev) for k in names}
     w_lm = jet_synth.torch_tensor(problem, "w_lm", device=dev)
@@ -310,7 +310,7 @@ def run_gpu(args):
             ev[1].record(stream)
         if step.hybrid:
             jet.jet_fork_state(lay, d, x["s_prefix"], x["lq"], x["lk"], x["lv"], x["alpha"],
-                               x["beta"], step.lo, step.s_fork, stream=stream)
+                               x["beta"], step.lo, step.s_fork, stream=stream, rule=step.rule)
         if ev:
             ev[2].record(stream)
         step.score(x["hidden"], w_lm, stream=stream)
@@ -455,6 +455,7 @@ def run_gpu(args):
                     Hl=w.Hl, parallelism=f"replicas{world}" if world > 1 else "single",
                     lm_head="e4m3, one float32 scale per weight row and per token" if e4m3
                     else "bf16",
+                    recurrence=(args.rule if w.Hl else None),
                     l2=f"inputs larger than L2: LM-head weights {w.V * w.D * es / 1e9:.2f} GB "
                        f"streamed every step"),
         clocks=clk,
@@ -517,6 +518,8 @@ def main():
     ap.add_argument("--ref-sample", type=int, default=1,
                     help="requests per step of the reference arm")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--rule", default="delta", choices=["delta", "gla"],
+                    help="recurrence of the linear-attention fork (hybrid workloads)")
     ap.add_argument("--lm", default="bf16", choices=["bf16", "e4m3"],
                     help="LM head precision: bf16 (the workload's), or e4m3 codes with one "
                          "scale per weight row and per token (the paper's 8-bit weights)")

@@ -76,6 +76,10 @@ enum {
 
 enum { JET_DTYPE_F32 = 0, JET_DTYPE_BF16 = 1 };
 
+/* recurrences of the linear-attention fork (the paper names none; see
+ * jet_fork_state_rule) */
+enum { JET_RECUR_DELTA = 0, JET_RECUR_GLA = 1 };
+
 /* decision rules of Sec. 3.3 / Eq. 5 */
 enum { JET_DECIDE_ARGMAX = 0, JET_DECIDE_BINARY = 1, JET_DECIDE_ORDINAL = 2 };
 
@@ -226,6 +230,18 @@ jet_status jet_prefix_attend(const jet_layout* lay, const jet_dims* dims, const 
 jet_status jet_fork_state(const jet_layout* lay, const jet_dims* dims, const float* s_prefix,
                           const void* q, const void* k, const void* v, const float* alpha,
                           const float* beta, void* o, float* s_fork, void* stream);
+
+/*
+ * jet_fork_state_rule - jet_fork_state with the recurrence chosen by `rule`:
+ * JET_RECUR_DELTA, the gated delta rule above (what jet_fork_state runs), or
+ * JET_RECUR_GLA, plain gated linear attention S <- alpha S + beta k v^T (no
+ * erase term), with the same inputs, outputs and read-out. Any other rule:
+ * JET_ERR_ARG.
+ */
+jet_status jet_fork_state_rule(const jet_layout* lay, const jet_dims* dims, int32_t rule,
+                               const float* s_prefix, const void* q, const void* k, const void* v,
+                               const float* alpha, const float* beta, void* o, float* s_fork,
+                               void* stream);
 
 /*
  * jet_score_candidates - LM head, full-vocabulary log-softmax and target

@@ -188,12 +188,14 @@ extern "C" jet_status jet_prefix_attend(const jet_layout* lay, const jet_dims* d
                                                static_cast<cudaStream_t>(stream)));
 }
 
-extern "C" jet_status jet_fork_state(const jet_layout* lay, const jet_dims* dims,
-                                     const float* s_prefix, const void* q, const void* k,
-                                     const void* v, const float* alpha, const float* beta, void* o,
-                                     float* s_fork, void* stream) {
+extern "C" jet_status jet_fork_state_rule(const jet_layout* lay, const jet_dims* dims,
+                                          int32_t rule, const float* s_prefix, const void* q,
+                                          const void* k, const void* v, const float* alpha,
+                                          const float* beta, void* o, float* s_fork,
+                                          void* stream) {
   JET_TRY(check_layout(lay));
   JET_TRY(check_fork_dims(dims));
+  if (rule != JET_RECUR_DELTA && rule != JET_RECUR_GLA) return JET_ERR_ARG;
   const jet_sizes& n = lay->n;
   if (n.R == 0) return JET_OK;
   if (n.R > 65535 || dims->Hl > 65535) return JET_ERR_CAPACITY;
@@ -206,9 +208,17 @@ extern "C" jet_status jet_fork_state(const jet_layout* lay, const jet_dims* dims
   JET_TRY(check_ptr(beta, F));
   JET_TRY(check_ptr(o, F));
   if (s_fork && !aligned16(s_fork)) return JET_ERR_ALIGN;
-  return cuda_status(jet::launch_fork_state(*lay, *dims, s_prefix, q, k, v, alpha, beta, o, s_fork,
-                                            jet::device_status_ptr(),
+  return cuda_status(jet::launch_fork_state(*lay, *dims, rule, s_prefix, q, k, v, alpha, beta, o,
+                                            s_fork, jet::device_status_ptr(),
                                             static_cast<cudaStream_t>(stream)));
+}
+
+extern "C" jet_status jet_fork_state(const jet_layout* lay, const jet_dims* dims,
+                                     const float* s_prefix, const void* q, const void* k,
+                                     const void* v, const float* alpha, const float* beta, void* o,
+                                     float* s_fork, void* stream) {
+  return jet_fork_state_rule(lay, dims, JET_RECUR_DELTA, s_prefix, q, k, v, alpha, beta, o,
+                             s_fork, stream);
 }
 
 extern "C" jet_status jet_score_candidates(const jet_layout* lay, const jet_dims* dims,

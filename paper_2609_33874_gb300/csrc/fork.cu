@@ -12,7 +12,9 @@
 // (the paper does not state its recurrence; this is the reading used).
 // The update is column-separable: column j of S needs only k, v_j and the
 // column's own u_j = k^T S[:, j], so a CTA owns a 32-column slice of one
-// head. The kernel is bound by the writes of the forked states.
+// head. The kernel is bound by the writes of the forked states. The plain
+// gated linear-attention variant S <- alpha S + beta k v^T is the same update
+// with u = 0 (the DELTA = false instantiation skips that reduction).
 #include "jet_device.cuh"
 #include "jet_internal.h"
 
@@ -104,7 +106,7 @@ __device__ __forceinline__ void stage_window(const T* __restrict__ q, const T* _
 
 // grid (dv / 32, Hl, R); thread (warp w, lane = 8 * rg + jq) owns rows
 // 32 w + rg + 4 ii (ii < 8) and columns j0 + 4 jq .. + 3 of the slice.
-template <typename T>
+template <typename T, bool DELTA>
 __global__ void __launch_bounds__(kThreads)
 fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__ cand_row_offset,
             const int32_t* __restrict__ tgt_offset, const int32_t* __restrict__ row_offset,
@@ -194,11 +196,13 @@ fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__
         const float a = wa[wt], b = wb[wt];
         const float4 vv = make_float4(to_f32(wv[wt][4 * jq]), to_f32(wv[wt][4 * jq + 1]),
                                       to_f32(wv[wt][4 * jq + 2]), to_f32(wv[wt][4 * jq + 3]));
-        // u = k^T S for this column quad
+        // u = k^T S for this column quad (the delta rule's erase term)
         float4 u = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (DELTA) {
 #pragma unroll
-        for (int ii = 0; ii < 8; ++ii) u = f4_fma(kk[ii], S[ii], u);
-        u = rows_sum(u, red, warp, lane);
+          for (int ii = 0; ii < 8; ++ii) u = f4_fma(kk[ii], S[ii], u);
+          u = rows_sum(u, red, warp, lane);
+        }
         // S = alpha S + beta k (v - alpha u)
         const float4 w = make_float4(b * (vv.x - a * u.x), b * (vv.y - a * u.y),
                                      b * (vv.z - a * u.z), b * (vv.w - a * u.w));
@@ -234,25 +238,39 @@ fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__
 
 }  // namespace
 
-cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, const float* s_prefix,
-                              const void* q, const void* k, const void* v, const float* alpha,
-                              const float* beta, void* o, float* s_fork, int* status,
-                              cudaStream_t st) {
+namespace {
+
+template <bool DELTA>
+cudaError_t launch_rule(const jet_layout& lay, const jet_dims& d, const float* s_prefix,
+                        const void* q, const void* k, const void* v, const float* alpha,
+                        const float* beta, void* o, float* s_fork, int* status,
+                        cudaStream_t st) {
   const jet_sizes& n = lay.n;
   dim3 grid(unsigned(d.dv / kCols), unsigned(d.Hl), unsigned(n.R));
   const int F = n.N - n.R;
   if (d.dtype == JET_DTYPE_F32) {
-    return launch_pdl(fork_kernel<float>, grid, dim3(kThreads), 0, st, lay.cand_offset,
+    return launch_pdl(fork_kernel<float, DELTA>, grid, dim3(kThreads), 0, st, lay.cand_offset,
                       lay.cand_row_offset, lay.tgt_offset, lay.row_offset, n.R, n.C, F, d.Hl,
                       d.dv, s_prefix, static_cast<const float*>(q), static_cast<const float*>(k),
                       static_cast<const float*>(v), alpha, beta, static_cast<float*>(o), s_fork,
                       status);
   }
-  return launch_pdl(fork_kernel<__nv_bfloat16>, grid, dim3(kThreads), 0, st, lay.cand_offset,
-                    lay.cand_row_offset, lay.tgt_offset, lay.row_offset, n.R, n.C, F, d.Hl, d.dv,
-                    s_prefix, static_cast<const __nv_bfloat16*>(q),
+  return launch_pdl(fork_kernel<__nv_bfloat16, DELTA>, grid, dim3(kThreads), 0, st,
+                    lay.cand_offset, lay.cand_row_offset, lay.tgt_offset, lay.row_offset, n.R,
+                    n.C, F, d.Hl, d.dv, s_prefix, static_cast<const __nv_bfloat16*>(q),
                     static_cast<const __nv_bfloat16*>(k), static_cast<const __nv_bfloat16*>(v),
                     alpha, beta, static_cast<__nv_bfloat16*>(o), s_fork, status);
+}
+
+}  // namespace
+
+cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, int rule,
+                              const float* s_prefix, const void* q, const void* k, const void* v,
+                              const float* alpha, const float* beta, void* o, float* s_fork,
+                              int* status, cudaStream_t st) {
+  if (rule == JET_RECUR_GLA)
+    return launch_rule<false>(lay, d, s_prefix, q, k, v, alpha, beta, o, s_fork, status, st);
+  return launch_rule<true>(lay, d, s_prefix, q, k, v, alpha, beta, o, s_fork, status, st);
 }
 
 }  // namespace jet

@@ -68,10 +68,11 @@ cudaError_t launch_attend_tc(const jet_layout& lay, const jet_dims& d, const Att
                              const void* k_cand, const void* v_cand, void* o, float* o_part,
                              float2* ml_part, int* status, cudaStream_t st);
 
-cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, const float* s_prefix,
-                              const void* q, const void* k, const void* v, const float* alpha,
-                              const float* beta, void* o, float* s_fork, int* status,
-                              cudaStream_t st);
+// rule: JET_RECUR_DELTA or JET_RECUR_GLA
+cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, int rule,
+                              const float* s_prefix, const void* q, const void* k, const void* v,
+                              const float* alpha, const float* beta, void* o, float* s_fork,
+                              int* status, cudaStream_t st);
 
 // logits partials: writes part[N][vtiles] (m, s) in base 2 - m = max_v z log2(e),
 // s = sum_v 2^(z log2(e) - m) over the tile - and z_tgt[T]

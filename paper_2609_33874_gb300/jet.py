@@ -27,6 +27,8 @@ STATUS_NAMES = {0: "JET_OK", 1: "JET_ERR_ARG", 2: "JET_ERR_SHAPE", 3: "JET_ERR_R
 DTYPE_F32, DTYPE_BF16 = 0, 1
 DECIDE_ARGMAX, DECIDE_BINARY, DECIDE_ORDINAL = 0, 1, 2
 MODES = {"argmax": DECIDE_ARGMAX, "binary": DECIDE_BINARY, "ordinal": DECIDE_ORDINAL}
+RECUR_DELTA, RECUR_GLA = 0, 1
+RULES = {"delta": RECUR_DELTA, "gla": RECUR_GLA}
 
 
 class JetError(RuntimeError):
@@ -79,6 +81,8 @@ def _load() -> ctypes.CDLL:
                                   P, P, P, P, P, P, P, SZ, P]),
         "jet_fork_state": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
                                P, P, P, P, P, P, P, P, P]),
+        "jet_fork_state_rule": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims), I,
+                                    P, P, P, P, P, P, P, P, P]),
         "jet_score_candidates": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
                                      P, P, P, P, P, SZ, P]),
         "jet_score_candidates_noalloc": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
@@ -101,7 +105,7 @@ def _load() -> ctypes.CDLL:
 _lib = _load()
 DECLARED = ("jet_abi_version", "jet_status_string", "jet_layout_plan", "jet_layout_words",
             "jet_layout_build", "jet_layout_bind", "jet_workspace_bytes", "jet_prefix_attend",
-            "jet_fork_state", "jet_score_candidates", "jet_score_candidates_noalloc",
+            "jet_fork_state", "jet_fork_state_rule", "jet_score_candidates", "jet_score_candidates_noalloc",
             "jet_quantize_rows_e4m3", "jet_workspace_bytes_e4m3", "jet_score_candidates_e4m3",
             "jet_decide", "jet_evaluate", "jet_device_status")
 
@@ -229,10 +233,19 @@ def jet_prefix_attend(layout, dims: jet_dims, q, k_pre, v_pre, k_cand, v_cand, o
 
 
 def jet_fork_state(layout, dims: jet_dims, s_prefix, q, k, v, alpha, beta, o, s_fork=None,
-                   stream=None) -> None:
-    _check(_lib.jet_fork_state(ctypes.byref(_lay(layout)), ctypes.byref(dims), _addr(s_prefix),
-                               _addr(q), _addr(k), _addr(v), _addr(alpha), _addr(beta), _addr(o),
-                               _addr(s_fork), _stream(stream)), "jet_fork_state")
+                   stream=None, rule: int = None) -> None:
+    """The fork with the gated delta rule, or with the recurrence `rule`
+    (RECUR_DELTA or RECUR_GLA) through jet_fork_state_rule."""
+    if rule is None:
+        _check(_lib.jet_fork_state(ctypes.byref(_lay(layout)), ctypes.byref(dims),
+                                   _addr(s_prefix), _addr(q), _addr(k), _addr(v), _addr(alpha),
+                                   _addr(beta), _addr(o), _addr(s_fork), _stream(stream)),
+               "jet_fork_state")
+        return
+    _check(_lib.jet_fork_state_rule(ctypes.byref(_lay(layout)), ctypes.byref(dims), int(rule),
+                                    _addr(s_prefix), _addr(q), _addr(k), _addr(v), _addr(alpha),
+                                    _addr(beta), _addr(o), _addr(s_fork), _stream(stream)),
+           "jet_fork_state_rule")
 
 
 def jet_score_candidates(layout, dims: jet_dims, hidden, w_lm, tok_logprob, cand_score, ws,

@@ -46,14 +46,17 @@ class ScoringStep:
     state. ``chain`` feeds the attention output to the LM head (requires
     Hq * d == D). ``lm`` selects the LM head: "bf16" (w_lm is the bf16 weight
     matrix) or "e4m3" (w_lm is the pair returned by :func:`quantize_lm_head`).
+    ``rule`` selects the fork's recurrence: "delta" (gated delta rule) or "gla"
+    (plain gated linear attention).
     """
 
     def __init__(self, layout: "jet.HostLayout", dims: "jet.jet_dims", mode: int,
                  device="cuda", hybrid: bool = False, keep_fork_state: bool = False,
-                 chain: bool = False, lm: str = "bf16"):
+                 chain: bool = False, lm: str = "bf16", rule: str = "delta"):
         if lm not in ("bf16", "e4m3"):
             raise ValueError("lm must be 'bf16' or 'e4m3'")
         self.lm = lm
+        self.rule = jet.RULES[rule]
         self.dev = torch.device(device)
         self.host_layout = layout
         self.layout = layout.to_device(self.dev)
@@ -94,7 +97,7 @@ class ScoringStep:
                               self.o, self.ws, stream=stream)
         if self.hybrid:
             jet.jet_fork_state(lay, d, x["s_prefix"], x["lq"], x["lk"], x["lv"], x["alpha"],
-                               x["beta"], self.lo, self.s_fork, stream=stream)
+                               x["beta"], self.lo, self.s_fork, stream=stream, rule=self.rule)
         hidden = self.o.view(self.N, d.Hq * d.d) if self.chain else x["hidden"]
         self.score(hidden, w_lm, stream=stream, layout=lay)
         jet.jet_decide(lay, self.mode, self.cand_score, self.q_cand, self.choice, self.value,

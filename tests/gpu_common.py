@@ -22,22 +22,22 @@ def dims_for(jet, w):
     return jet.make_dims(dtype, Hq=w.Hq, Hkv=w.Hkv, d=w.d, D=w.D, Hl=w.Hl, dk=w.dk, dv=w.dv)
 
 
-def build_step(jet, problem, device="cuda", chain=False, keep_fork=True):
+def build_step(jet, problem, device="cuda", chain=False, keep_fork=True, rule="delta"):
     from paper_2609_33874_gb300.step import ScoringStep
     w = problem.work
     hl = jet.jet_layout_build(problem.prefix_len, problem.n_cand, problem.cand_len,
                               problem.target_ids, w.V)
     step = ScoringStep(hl, dims_for(jet, w), jet.MODES[w.mode], device=device,
-                       hybrid=w.Hl > 0, keep_fork_state=keep_fork, chain=chain)
+                       hybrid=w.Hl > 0, keep_fork_state=keep_fork, chain=chain, rule=rule)
     names = step.input_names()
     x = {k: jet_synth.torch_tensor(problem, k, device=device) for k in names}
     w_lm = jet_synth.torch_tensor(problem, "w_lm", device=device)
     return step, x, w_lm
 
 
-def run_problem(jet, problem, device="cuda", chain=False, keep_fork=True):
+def run_problem(jet, problem, device="cuda", chain=False, keep_fork=True, rule="delta"):
     import torch
-    step, x, w_lm = build_step(jet, problem, device, chain, keep_fork)
+    step, x, w_lm = build_step(jet, problem, device, chain, keep_fork, rule)
     step.run(x, w_lm)
     torch.cuda.synchronize()
     assert jet.jet_device_status() == 0
@@ -110,11 +110,12 @@ def check_attention(lay, problem, got_o, rows, tol):
     return ref
 
 
-def check_fork(lay, problem, got, requests):
+def check_fork(lay, problem, got, requests, rule="delta"):
     sub = [r for r in requests]
     s_prefix = problem.f32("s_prefix")
     ref_o, ref_s = O.fork_state(lay, s_prefix, problem.f32("lq"), problem.f32("lk"),
-                                problem.f32("lv"), problem.f32("alpha"), problem.f32("beta"))
+                                problem.f32("lv"), problem.f32("alpha"), problem.f32("beta"),
+                                rule=rule)
     for r in sub:
         c0, c1 = int(lay["cand_offset"][r]), int(lay["cand_offset"][r + 1])
         if got.get("s_fork") is not None:

@@ -184,6 +184,16 @@ def test_fork_validation(jet):
     assert lib.jet_fork_state(ctypes.byref(lay.struct), ctypes.byref(dims), *nul) == 1
 
 
+def test_fork_rule_validation(jet):
+    lay, dims = _setup(jet)
+    lib = jet.library()
+    args = [FAKE] * 9
+    assert lib.jet_fork_state_rule(ctypes.byref(lay.struct), ctypes.byref(dims), 7, *args) == 1
+    bad = jet.make_dims(jet.DTYPE_BF16, Hl=2, dk=64, dv=64)
+    assert lib.jet_fork_state_rule(ctypes.byref(lay.struct), ctypes.byref(bad), jet.RECUR_GLA,
+                                   *args) == 7
+
+
 def test_e4m3_validation(jet):
     lay, dims = _setup(jet)
     lib = jet.library()

@@ -147,14 +147,22 @@ def test_fork_small(cuda, keep, dtype):
 
 
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
-def test_fork_long_candidates(cuda, dtype):
+@pytest.mark.parametrize("rule", ["delta", "gla"])
+def test_fork_long_candidates(cuda, dtype, rule):
     # candidates of up to 40 tokens: the 32-token window of fed tokens is
-    # staged again inside a candidate and across candidates
+    # staged again inside a candidate and across candidates; both recurrences
     p = _custom("ordinal_hybrid", [5, 9], [4, 3], [20, 40, 1, 33, 7, 12, 2], seed=41, V=4096,
                 D=256, Hl=2, dv=96, dtype=dtype)
-    got, _ = run_problem(cuda, p)
+    got, _ = run_problem(cuda, p, rule=rule)
     lay = oracle_layout(p)
-    check_fork(lay, p, got, list(range(p.R)))
+    check_fork(lay, p, got, list(range(p.R)), rule=rule)
+
+
+def test_fork_gla_full_size(cuda):
+    # the hybrid workload's shape with the gated linear-attention recurrence
+    p = jet_synth.make_problem("ordinal_hybrid")
+    got, _ = run_problem(cuda, p, keep_fork=True, rule="gla")
+    check_fork(oracle_layout(p), p, got, [0, 17, 31], rule="gla")
 
 
 # ---------------------------------------------------------------------------
