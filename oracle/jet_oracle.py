@@ -22,6 +22,8 @@ What each function computes, and where the paper defines it:
   their own earlier candidate tokens (Sec. 4.1, Fig. 1 "KV-cache text
   models"). Readings where the paper is silent: scale 1/sqrt(d), grouped-query
   head h uses key/value head floor(h / (Hq/Hkv)), no positional encoding.
+* :func:`prefill_attention` - causal self-attention over each request's
+  prefix, the prefill whose K/V the scoring step reuses (Sec. 4.1).
 * :func:`fork_state` - every candidate continues an unmodified copy of the
   prefix recurrent state (Sec. 4.1, "Hybrid models ... restoring the unchanged
   prefix state before each candidate"; Sec. 5.6). The recurrence itself is not
@@ -49,8 +51,8 @@ from typing import Dict
 
 import numpy as np
 
-__all__ = ["build_layout", "cascade_attention", "fork_state", "token_logprobs",
-           "candidate_scores", "decide", "evaluate", "score_step"]
+__all__ = ["build_layout", "cascade_attention", "prefill_attention", "fork_state",
+           "token_logprobs", "candidate_scores", "decide", "evaluate", "score_step"]
 
 ARGMAX, BINARY, ORDINAL = 0, 1, 2
 
@@ -201,6 +203,31 @@ def cascade_attention(lay, q, k_pre, v_pre, k_cand, v_cand, Hq: int, Hkv: int, r
                                 np.asarray(k_cand[fed, kh], np.float64).reshape(len(fed), d)])
             Vv = np.concatenate([np.asarray(v_pre[p0:p1, kh], np.float64),
                                  np.asarray(v_cand[fed, kh], np.float64).reshape(len(fed), d)])
+            scores = (K @ qn[h]) * scale
+            w = np.exp(scores - scores.max())
+            out[i, h] = (w / w.sum()) @ Vv
+    return out
+
+
+def prefill_attention(prefix_len, q, k, v, Hq: int, Hkv: int, rows=None):
+    """Causal self-attention over every request's prefix, the prefill that
+    produces the shared prefix (Sec. 4.1): position p of request r attends to
+    the request's keys 0..p. q is [sum P, Hq, d]; k, v are [sum P, Hkv, d].
+    ``rows`` selects prefix rows (default: all). All float64."""
+    prefix_len = np.asarray(prefix_len, np.int64)
+    offset = np.concatenate([[0], np.cumsum(prefix_len)])
+    total, _, d = q.shape
+    rows = list(range(total)) if rows is None else [int(n) for n in rows]
+    g = Hq // Hkv
+    scale = 1.0 / math.sqrt(d)
+    out = np.zeros((len(rows), Hq, d), dtype=np.float64)
+    for i, n in enumerate(rows):
+        r = int(np.searchsorted(offset, n, side="right") - 1)
+        p0 = int(offset[r])
+        qn = np.asarray(q[n], np.float64)
+        for h in range(Hq):
+            K = np.asarray(k[p0:n + 1, h // g], np.float64)
+            Vv = np.asarray(v[p0:n + 1, h // g], np.float64)
             scores = (K @ qn[h]) * scale
             w = np.exp(scores - scores.max())
             out[i, h] = (w / w.sum()) @ Vv

@@ -553,3 +553,49 @@ def test_fork_rule_selects_the_recurrence():
     for f in (0, 1):
         S = al[f, 1] * S + be[f, 1] * np.outer(lk[f, 1], lv[f, 1])
     np.testing.assert_allclose(sg[0, 1], S, rtol=1e-13)
+
+
+# ---------------------------------------------------------------------------
+# prefill: causal attention over each request's prefix
+# ---------------------------------------------------------------------------
+def test_prefill_first_position_and_zero_query():
+    rng = np.random.default_rng(41)
+    P = [5, 3]
+    q = rng.normal(size=(8, 4, 6)); k = rng.normal(size=(8, 2, 6)); v = rng.normal(size=(8, 2, 6))
+    q[6] = 0.0
+    out = O.prefill_attention(P, q, k, v, 4, 2)
+    # position 0 of each request sees only its own key: the output is its value
+    np.testing.assert_allclose(out[0], v[0][[0, 0, 1, 1]], rtol=1e-14)
+    np.testing.assert_allclose(out[5], v[5][[0, 0, 1, 1]], rtol=1e-14)
+    # a zero query averages exactly the visible values (request 1, position 1 = row 6)
+    np.testing.assert_allclose(out[6, 2], v[5:7, 1].mean(axis=0), rtol=1e-14)
+
+
+def test_prefill_last_position_equals_the_shared_row():
+    # the shared row of the scoring step is the last prefix position: the
+    # prefill's output there equals cascade attention of that row
+    rng = np.random.default_rng(42)
+    P = [6, 4]
+    lay = O.build_layout(P, [1, 1], [1, 1], [3, 5], 8)
+    d, Hq, Hkv = 8, 6, 3
+    qp = rng.normal(size=(10, Hq, d)); kp = rng.normal(size=(10, Hkv, d))
+    vp = rng.normal(size=(10, Hkv, d))
+    q_rows = qp[[5, 9]]                      # the shared rows' queries
+    casc = O.cascade_attention(lay, q_rows, kp, vp, np.zeros((0, Hkv, d)), np.zeros((0, Hkv, d)),
+                               Hq, Hkv)
+    pre = O.prefill_attention(P, qp, kp, vp, Hq, Hkv, rows=[5, 9])
+    np.testing.assert_allclose(pre, casc, rtol=1e-13)
+
+
+def test_prefill_is_causal():
+    # changing a later key or value never changes an earlier position
+    rng = np.random.default_rng(43)
+    P = [7]
+    q = rng.normal(size=(7, 2, 4)); k = rng.normal(size=(7, 1, 4)); v = rng.normal(size=(7, 1, 4))
+    a = O.prefill_attention(P, q, k, v, 2, 1)
+    k2, v2 = k.copy(), v.copy()
+    k2[4:] += 3.0
+    v2[4:] -= 1.0
+    b = O.prefill_attention(P, q, k2, v2, 2, 1)
+    np.testing.assert_array_equal(a[:4], b[:4])
+    assert not np.allclose(a[4:], b[4:])
