@@ -474,6 +474,74 @@ def run_gpu(args):
 
 
 # ---------------------------------------------------------------------------
+# the prefill (a "next" row, one GPU): causal attention over the prefixes
+# ---------------------------------------------------------------------------
+def run_prefill(args):
+    """Times jet_prefill_attend on the workload's prefixes (their queries,
+    keys and values resident in HBM) and prints one JSON line: prefix tokens
+    per second, with the tensor roofline of the causal attention."""
+    import torch
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    from paper_2609_33874_gb300 import build as _build
+    _build.build()
+    import jet_synth
+    from paper_2609_33874_gb300 import jet
+    w = jet_synth.WORKLOADS[args.workload]
+    R = args.R or w.R
+    p = jet_synth.make_problem(w, R=R)
+    if w.dtype != "bf16":
+        print(json.dumps(dict(metric="prefix tokens prefilled/sec", unavailable="bf16 only")))
+        return
+    hl = jet.jet_layout_build(p.prefix_len, p.n_cand, p.cand_len, p.target_ids, w.V)
+    lay = hl.to_device(dev)
+    dims = jet.make_dims(jet.DTYPE_BF16, Hq=w.Hq, Hkv=w.Hkv, d=w.d, D=w.D)
+    q, k, v = (jet_synth.torch_tensor(p, n, device=dev) for n in ("q_pre", "k_pre", "v_pre"))
+    p.drop()
+    o = torch.empty(p.total_prefix, w.Hq, w.d, dtype=torch.bfloat16, device=dev)
+    wsb = jet.jet_prefill_workspace_bytes(hl.sizes, dims)
+    ws = torch.empty((wsb + 15) // 16 * 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.Stream(dev)
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            jet.jet_prefill_attend(lay, dims, q, k, v, o, ws, stream=stream)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(args.steps):
+            jet.jet_prefill_attend(lay, dims, q, k, v, o, ws, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    assert jet.jet_device_status(stream) == 0
+    ms = e0.elapsed_time(e1) / args.steps
+    P = p.prefix_len.astype(np.float64)
+    # S = QK^T and O = PV over the causal triangle (keys 0..p of position p)
+    flops = float(np.sum(4.0 * w.Hq * w.d * P * (P + 1) / 2))
+    nbytes = p.total_prefix * (2 * w.Hq + 2 * w.Hkv) * w.d * 2  # Q, O, K, V once
+    peaks = _peaks()
+    tf = flops / (ms / 1e3) / 1e12
+    gbs = nbytes / (ms / 1e3) / 1e9
+    ridge = peaks["bf16"] * 1e12 / (peaks["hbm"] * 1e9)
+    if flops / nbytes >= ridge:
+        roof = dict(bound="tensor", achieved=round(tf, 1), peak=peaks["bf16"], unit="TFLOP/s",
+                    frac=round(tf / peaks["bf16"], 4))
+    else:
+        roof = dict(bound="hbm", achieved=round(gbs, 1), peak=peaks["hbm"], unit="GB/s",
+                    frac=round(gbs / peaks["hbm"], 4))
+    roof.update(kernel="jet_prefill_attend (work list + attend_prefix_tc_kernel, causal)",
+                algorithmic_flops=flops, algorithmic_bytes=nbytes, traffic=None,
+                peak_source=peaks["source"])
+    print(json.dumps(dict(
+        metric="prefix tokens prefilled/sec", value=round(p.total_prefix / (ms / 1e3), 1),
+        unit="tokens/s", n_gpus=1, steps=args.steps, warmup=args.warmup,
+        ms_per_step=round(ms, 4), higher_is_better=True, dtype="bf16", data="synthetic",
+        config=dict(workload=args.workload, R=R, total_prefix=p.total_prefix,
+                    max_prefix=int(P.max()), Hq=w.Hq, Hkv=w.Hkv, d=w.d),
+        roofline=roof, gpu_launches=2 * args.steps)), flush=True)
+
+
+# ---------------------------------------------------------------------------
 # reference arm: the fp64 oracle on the host cores
 # ---------------------------------------------------------------------------
 def run_reference(args):
@@ -523,6 +591,9 @@ def main():
     ap.add_argument("--lm", default="bf16", choices=["bf16", "e4m3"],
                     help="LM head precision: bf16 (the workload's), or e4m3 codes with one "
                          "scale per weight row and per token (the paper's 8-bit weights)")
+    ap.add_argument("--prefill", action="store_true",
+                    help="time the prefill (causal attention over the workload's prefixes) "
+                         "instead of the scoring step (one GPU)")
     ap.add_argument("--sweep", action="store_true",
                     help="one line per batch size R = 1, 2, 4, ... up to the workload's R "
                          "(one GPU; no CPU baseline)")
@@ -530,6 +601,8 @@ def main():
     args.warmup = max(3, args.warmup)  # at least three untimed warm-up steps
     if args.impl == "reference":
         run_reference(args)
+    elif args.prefill:
+        run_prefill(args)
     elif args.sweep:
         import jet_synth
         if _dist()[0] > 1:

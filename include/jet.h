@@ -214,6 +214,24 @@ jet_status jet_prefix_attend(const jet_layout* lay, const jet_dims* dims, const 
                              void* stream);
 
 /*
+ * jet_prefill_attend - the prefill before the scoring step: causal
+ * self-attention over every request's prefix (Sec. 4.1: the shared prefix is
+ * evaluated once and its K/V reused by every candidate; scale 1/sqrt(d), no
+ * positional encoding, grouped-query heads as in jet_prefix_attend).
+ *   q     [total_prefix, Hq, d]    queries of the prefix positions
+ *   k, v  [total_prefix, Hkv, d]   the prefix K/V (what jet_prefix_attend reads)
+ *   o     [total_prefix, Hq, d]    position p of request r attends to r's keys 0..p
+ * bf16 only (else JET_ERR_UNSUPPORTED), d in {64, 128, 256}. Uses the layout's
+ * prefix sizes only. ws/ws_bytes: scratch of at least
+ * jet_prefill_workspace_bytes() (a work list of 16 bytes per block of
+ * 128 / (Hq / Hkv) positions and key/value head).
+ */
+size_t jet_prefill_workspace_bytes(const jet_sizes* n, const jet_dims* dims);
+jet_status jet_prefill_attend(const jet_layout* lay, const jet_dims* dims, const void* q,
+                              const void* k, const void* v, void* o, void* ws, size_t ws_bytes,
+                              void* stream);
+
+/*
  * jet_fork_state - per-candidate fork of a linear-attention recurrent state
  * (Sec. 4.1: each candidate continues from the unchanged prefix state).
  *   s_prefix [R, Hl, dk, dv] float32  state after the prefix (read only)

@@ -144,7 +144,7 @@ def _normal_chunks(seed: int, tag: int, n: int, std: float, bf16: bool) -> np.nd
 # tensor tags (part of the seed of each tensor)
 _TAGS = {"structure": 1, "q": 2, "k_pre": 3, "v_pre": 4, "k_cand": 5, "v_cand": 6,
          "hidden": 7, "w_lm": 8, "s_prefix": 9, "lq": 10, "lk": 11, "lv": 12,
-         "alpha": 13, "beta": 14}
+         "alpha": 13, "beta": 14, "q_pre": 15}
 
 
 @dataclasses.dataclass
@@ -204,6 +204,8 @@ class Problem:
             return self._normal("q", (self.N, w.Hq, w.d))
         if name in ("k_pre", "v_pre"):
             return self._normal(name, (self.total_prefix, w.Hkv, w.d))
+        if name == "q_pre":  # queries of every prefix position (the prefill)
+            return self._normal("q_pre", (self.total_prefix, w.Hq, w.d))
         if name in ("k_cand", "v_cand"):
             return self._normal(name, (self.F, w.Hkv, w.d))
         if name == "hidden":

@@ -188,6 +188,32 @@ extern "C" jet_status jet_prefix_attend(const jet_layout* lay, const jet_dims* d
                                                static_cast<cudaStream_t>(stream)));
 }
 
+extern "C" size_t jet_prefill_workspace_bytes(const jet_sizes* n, const jet_dims* d) {
+  if (!n || !d || n->R < 0) return 0;
+  return jet::prefill_workspace_bytes(*n, *d);
+}
+
+extern "C" jet_status jet_prefill_attend(const jet_layout* lay, const jet_dims* dims,
+                                         const void* q, const void* k, const void* v, void* o,
+                                         void* ws, size_t ws_bytes, void* stream) {
+  JET_TRY(check_layout(lay));
+  JET_TRY(check_attn_dims(dims));
+  if (dims->dtype != JET_DTYPE_BF16) return JET_ERR_UNSUPPORTED;
+  const jet_sizes& n = lay->n;
+  if (n.R == 0) return JET_OK;
+  const size_t need = jet::prefill_workspace_bytes(n, *dims);
+  if (need == 0) return JET_ERR_SHAPE;
+  if ((need - 32) / 16 > size_t(INT32_MAX)) return JET_ERR_CAPACITY;  // items a counter indexes
+  JET_TRY(check_ptr(q, n.total_prefix));
+  JET_TRY(check_ptr(k, n.total_prefix));
+  JET_TRY(check_ptr(v, n.total_prefix));
+  JET_TRY(check_ptr(o, n.total_prefix));
+  if (!ws || ws_bytes < need) return JET_ERR_WORKSPACE;
+  if (!aligned16(ws)) return JET_ERR_ALIGN;
+  return cuda_status(jet::launch_prefill_tc(*lay, *dims, q, k, v, o, ws, jet::device_status_ptr(),
+                                            static_cast<cudaStream_t>(stream)));
+}
+
 extern "C" jet_status jet_fork_state_rule(const jet_layout* lay, const jet_dims* dims,
                                           int32_t rule, const float* s_prefix, const void* q,
                                           const void* k, const void* v, const float* alpha,

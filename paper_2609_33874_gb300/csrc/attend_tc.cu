@@ -81,6 +81,7 @@ struct AttArgs {
   int splits;        // chunks per request (the plan's), for the static order
   long long n_all;   // slots in the static order
   int has_cand;      // the batch has fed candidate tokens (F > 0)
+  int prefill;       // 1: causal self-attention over the prefixes (rows = prefix positions)
   float scale_log2;  // log2(e) / sqrt(d)
 };
 
@@ -182,6 +183,29 @@ __device__ __forceinline__ ItemGeo item_geo(const AttArgs& a, int4 it) {
   e.split = it.w;
   e.ok = false;
   if (e.r < 0 || e.r >= a.R || e.kh < 0 || e.kh >= a.Hkv) return e;
+  if (a.prefill) {
+    // prefill: the rows are the request's prefix positions and a block of
+    // them sees the keys up to its last position (per-row causal mask in the
+    // softmax); one chunk per item, the output written directly
+    e.p0 = a.prefix_offset[e.r];
+    e.P = a.prefix_offset[e.r + 1] - e.p0;
+    if (e.p0 < 0 || e.P < 1 || e.p0 + e.P > a.total_prefix || e.split != 0) return e;
+    e.n0 = e.p0;
+    e.nr = e.P;
+    e.row0 = qb * a.rb;
+    if (e.row0 >= e.nr) return e;
+    e.vbase = e.row0 * a.g;
+    e.nv = min(a.rb, e.nr - e.row0) * a.g;
+    e.splits_r = 1;
+    e.k_begin = 0;
+    e.k_end = min(e.P, e.row0 + a.rb);
+    e.npt = (e.k_end + kBN - 1) / kBN;
+    e.nct = 0;
+    e.f_begin = 0;
+    e.ntiles = e.npt;
+    e.ok = true;
+    return e;
+  }
   e.n0 = a.row_offset[e.r];
   e.nr = a.row_offset[e.r + 1] - e.n0;
   e.p0 = a.prefix_offset[e.r];
@@ -646,7 +670,9 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       const ItemGeo e = ring[slot].e;
       const bool valid = i < e.nv;
       int fa = 1, fb = 0;  // fed-token indices this vector may see (none: shared row)
-      if (valid) {
+      // prefill: the last key this vector's position may see (causal)
+      const int kcap = a.prefill ? (e.vbase + i) / g : (1 << 30);
+      if (valid && !a.prefill) {
         const int gv = e.vbase + i;
         const int n = e.n0 + gv / g;
         const int c = a.row_cand[n];
@@ -683,6 +709,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         int klo = 0, khi;
         if (j < e.npt) {
           khi = min(kBN, e.k_end - (e.k_begin + j * kBN));
+          khi = min(khi, kcap + 1 - (e.k_begin + j * kBN));  // prefill: keys <= own position
         } else {
           const int f0 = e.f_begin + (j - e.npt) * kBN;
           klo = max(0, fa - f0);
@@ -997,9 +1024,89 @@ cudaError_t launch_dh(const jet_layout& lay, const jet_dims& d, const AttnPlan& 
                     static_cast<__nv_bfloat16*>(o), status);
 }
 
+// Prefill: causal self-attention over every request's prefix with the same
+// persistent kernel. Items are (request, kv head, block of 128/g positions):
+// a block reads the keys up to its last position, a row masks the keys past
+// its own; no chunking (the blocks already give one item per 128 / g
+// positions), so the output is written directly. Longest items first.
+template <int DH>
+cudaError_t launch_prefill_dh(const jet_layout& lay, const jet_dims& d, const void* q,
+                              const void* k, const void* v, void* o, void* ws, int* status,
+                              cudaStream_t st) {
+  const jet_sizes& n = lay.n;
+  const int g = d.Hq / d.Hkv;
+  if (g > kBV) return cudaErrorInvalidValue;
+  CUtensorMap tmQ, tmK, tmV;
+  if (!encode_3d(&tmQ, q, n.total_prefix, d.Hq, DH, g, kBV / g) ||
+      !encode_3d(&tmK, k, n.total_prefix, d.Hkv, DH, 1, kBN) ||
+      !encode_3d(&tmV, v, n.total_prefix, d.Hkv, DH, 1, kBN))
+    return cudaErrorInvalidValue;
+  AttArgs a{};
+  a.prefix_offset = lay.prefix_offset;
+  a.row_offset = lay.row_offset;
+  a.req_order = lay.req_order;
+  a.row_cand = lay.row_cand;
+  a.cand_row_offset = lay.cand_row_offset;
+  a.q = static_cast<const __nv_bfloat16*>(q);
+  a.o = static_cast<__nv_bfloat16*>(o);
+  a.status = status;
+  a.R = n.R;
+  a.N = n.total_prefix;
+  a.C = 0;
+  a.total_prefix = n.total_prefix;
+  a.Hq = d.Hq;
+  a.Hkv = d.Hkv;
+  a.chunk = 1 << 30;
+  a.g = g;
+  a.rb = kBV / g;
+  a.has_cand = 0;
+  a.prefill = 1;
+  a.scale_log2 = 1.4426950408889634f / sqrtf(float(DH));
+  const int qgroups = (n.max_prefix + a.rb - 1) / a.rb;
+  uintptr_t ctrl = (reinterpret_cast<uintptr_t>(ws) + 15) & ~uintptr_t(15);
+  a.item_next = reinterpret_cast<int*>(ctrl);
+  a.item_count = a.item_next + 1;
+  a.items = reinterpret_cast<int4*>(ctrl + 16);
+  a.splits = 1;
+  a.n_all = (long long)n.R * d.Hkv * qgroups;
+  a.sorted = 1;
+  cudaError_t e =
+      launch_pdl(attend_items_kernel, dim3(1), dim3(1024), 0, st, a, qgroups, 1);
+  if (e != cudaSuccess) return e;
+  const size_t smem = Geo<DH>::kBytes + 1024;
+  e = cudaFuncSetAttribute(attend_prefix_tc_kernel<DH>,
+                           cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  if (e != cudaSuccess) return e;
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+    return cudaErrorInvalidValue;
+  const int grid = int(std::max<long long>(1, std::min<long long>(sms, a.n_all)));
+  return launch_pdl(attend_prefix_tc_kernel<DH>, dim3(grid), dim3(kThreads), smem, st, tmQ, tmK,
+                    tmV, tmK, tmV, a);
+}
+
 }  // namespace
 
 int attn_tc_block() { return kBV; }
+
+size_t prefill_workspace_bytes(const jet_sizes& n, const jet_dims& d) {
+  if (d.Hkv < 1 || d.Hq < d.Hkv || d.Hq % d.Hkv != 0) return 0;
+  const int g = d.Hq / d.Hkv;
+  if (g > kBV) return 0;
+  const int rb = kBV / g;
+  const long long qgroups = (n.max_prefix + rb - 1) / rb;
+  return 32 + 16 * size_t(n.R) * d.Hkv * qgroups;
+}
+
+cudaError_t launch_prefill_tc(const jet_layout& lay, const jet_dims& d, const void* q,
+                              const void* k, const void* v, void* o, void* ws, int* status,
+                              cudaStream_t st) {
+  if (d.d == 64) return launch_prefill_dh<64>(lay, d, q, k, v, o, ws, status, st);
+  if (d.d == 128) return launch_prefill_dh<128>(lay, d, q, k, v, o, ws, status, st);
+  if (d.d == 256) return launch_prefill_dh<256>(lay, d, q, k, v, o, ws, status, st);
+  return cudaErrorInvalidValue;
+}
 
 cudaError_t launch_attend_tc(const jet_layout& lay, const jet_dims& d, const AttnPlan& plan,
                              const void* q, const void* k_pre, const void* v_pre,

@@ -69,6 +69,13 @@ cudaError_t launch_attend_tc(const jet_layout& lay, const jet_dims& d, const Att
                              float2* ml_part, int* status, cudaStream_t st);
 
 // rule: JET_RECUR_DELTA or JET_RECUR_GLA
+// causal self-attention over every request's prefix (bf16, tensor cores);
+// the workspace holds the work list
+size_t prefill_workspace_bytes(const jet_sizes& n, const jet_dims& d);
+cudaError_t launch_prefill_tc(const jet_layout& lay, const jet_dims& d, const void* q,
+                              const void* k, const void* v, void* o, void* ws, int* status,
+                              cudaStream_t st);
+
 cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, int rule,
                               const float* s_prefix, const void* q, const void* k, const void* v,
                               const float* alpha, const float* beta, void* o, float* s_fork,

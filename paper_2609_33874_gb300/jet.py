@@ -79,6 +79,10 @@ def _load() -> ctypes.CDLL:
         "jet_workspace_bytes": (SZ, [ctypes.POINTER(jet_sizes), ctypes.POINTER(jet_dims)]),
         "jet_prefix_attend": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
                                   P, P, P, P, P, P, P, SZ, P]),
+        "jet_prefill_workspace_bytes": (SZ, [ctypes.POINTER(jet_sizes),
+                                             ctypes.POINTER(jet_dims)]),
+        "jet_prefill_attend": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
+                                   P, P, P, P, P, SZ, P]),
         "jet_fork_state": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
                                P, P, P, P, P, P, P, P, P]),
         "jet_fork_state_rule": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims), I,
@@ -105,6 +109,7 @@ def _load() -> ctypes.CDLL:
 _lib = _load()
 DECLARED = ("jet_abi_version", "jet_status_string", "jet_layout_plan", "jet_layout_words",
             "jet_layout_build", "jet_layout_bind", "jet_workspace_bytes", "jet_prefix_attend",
+            "jet_prefill_workspace_bytes", "jet_prefill_attend",
             "jet_fork_state", "jet_fork_state_rule", "jet_score_candidates", "jet_score_candidates_noalloc",
             "jet_quantize_rows_e4m3", "jet_workspace_bytes_e4m3", "jet_score_candidates_e4m3",
             "jet_decide", "jet_evaluate", "jet_device_status")
@@ -230,6 +235,19 @@ def jet_prefix_attend(layout, dims: jet_dims, q, k_pre, v_pre, k_cand, v_cand, o
                                   _addr(k_pre), _addr(v_pre), _addr(k_cand), _addr(v_cand),
                                   _addr(o), _addr(ws), int(ws_bytes), _stream(stream)),
            "jet_prefix_attend")
+
+
+def jet_prefill_workspace_bytes(sizes: jet_sizes, dims: jet_dims) -> int:
+    return int(_lib.jet_prefill_workspace_bytes(ctypes.byref(sizes), ctypes.byref(dims)))
+
+
+def jet_prefill_attend(layout, dims: jet_dims, q, k, v, o, ws, ws_bytes: Optional[int] = None,
+                       stream=None) -> None:
+    """Causal self-attention over every request's prefix (see include/jet.h)."""
+    ws_bytes = ws.numel() * ws.element_size() if ws_bytes is None else ws_bytes
+    _check(_lib.jet_prefill_attend(ctypes.byref(_lay(layout)), ctypes.byref(dims), _addr(q),
+                                   _addr(k), _addr(v), _addr(o), _addr(ws), int(ws_bytes),
+                                   _stream(stream)), "jet_prefill_attend")
 
 
 def jet_fork_state(layout, dims: jet_dims, s_prefix, q, k, v, alpha, beta, o, s_fork=None,
