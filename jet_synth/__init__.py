@@ -144,7 +144,8 @@ def _normal_chunks(seed: int, tag: int, n: int, std: float, bf16: bool) -> np.nd
 # tensor tags (part of the seed of each tensor)
 _TAGS = {"structure": 1, "q": 2, "k_pre": 3, "v_pre": 4, "k_cand": 5, "v_cand": 6,
          "hidden": 7, "w_lm": 8, "s_prefix": 9, "lq": 10, "lk": 11, "lv": 12,
-         "alpha": 13, "beta": 14, "q_pre": 15}
+         "alpha": 13, "beta": 14, "q_pre": 15, "lq_pre": 16, "lk_pre": 17, "lv_pre": 18,
+         "alpha_pre": 19, "beta_pre": 20}
 
 
 @dataclasses.dataclass
@@ -220,19 +221,23 @@ class Problem:
             n = self.R * w.Hl * w.dk * w.dv
             x = _normal_chunks(self.seed, _TAGS["s_prefix"], n, 1.0 / np.sqrt(w.dk), False)
             val = x.reshape(self.R, w.Hl, w.dk, w.dv)
-        elif name in ("lq", "lv"):
-            dim = w.dk if name == "lq" else w.dv
-            val = self._normal(name, (self.F, w.Hl, dim))
-        elif name == "lk":
-            x = _normal_chunks(self.seed, _TAGS["lk"], self.F * w.Hl * w.dk, 1.0, False)
-            x = x.reshape(self.F, w.Hl, w.dk).astype(np.float64)
+        elif name in ("lq", "lv", "lq_pre", "lv_pre"):
+            # fed candidate tokens (F) or, with the _pre suffix, prefix tokens
+            dim = w.dk if name.startswith("lq") else w.dv
+            rows = self.total_prefix if name.endswith("_pre") else self.F
+            val = self._normal(name, (rows, w.Hl, dim))
+        elif name in ("lk", "lk_pre"):
+            rows = self.total_prefix if name.endswith("_pre") else self.F
+            x = _normal_chunks(self.seed, _TAGS[name], rows * w.Hl * w.dk, 1.0, False)
+            x = x.reshape(rows, w.Hl, w.dk).astype(np.float64)
             x /= np.linalg.norm(x, axis=-1, keepdims=True)  # unit-norm keys
             x = x.astype(np.float32)
             val = f32_to_bf16_bits(x).reshape(x.shape) if self.bf16 else x
-        elif name in ("alpha", "beta"):
-            lo, hi = (0.90, 1.00) if name == "alpha" else (0.0, 1.0)
+        elif name in ("alpha", "beta", "alpha_pre", "beta_pre"):
+            lo, hi = (0.90, 1.00) if name.startswith("alpha") else (0.0, 1.0)
+            rows = self.total_prefix if name.endswith("_pre") else self.F
             g = _rng(self.seed, _TAGS[name])
-            val = g.uniform(lo, hi, size=(self.F, w.Hl)).astype(np.float32)
+            val = g.uniform(lo, hi, size=(rows, w.Hl)).astype(np.float32)
         else:
             raise KeyError(name)
         self._cache[name] = val

@@ -24,6 +24,8 @@ What each function computes, and where the paper defines it:
   head h uses key/value head floor(h / (Hq/Hkv)), no positional encoding.
 * :func:`prefill_attention` - causal self-attention over each request's
   prefix, the prefill whose K/V the scoring step reuses (Sec. 4.1).
+* :func:`prefill_state` - the prefix recurrent state: the prefix tokens fed
+  through the recurrence in order, the state every candidate forks from.
 * :func:`fork_state` - every candidate continues an unmodified copy of the
   prefix recurrent state (Sec. 4.1, "Hybrid models ... restoring the unchanged
   prefix state before each candidate"; Sec. 5.6). The recurrence itself is not
@@ -51,7 +53,7 @@ from typing import Dict
 
 import numpy as np
 
-__all__ = ["build_layout", "cascade_attention", "prefill_attention", "fork_state",
+__all__ = ["build_layout", "cascade_attention", "prefill_attention", "prefill_state", "fork_state",
            "token_logprobs", "candidate_scores", "decide", "evaluate", "score_step"]
 
 ARGMAX, BINARY, ORDINAL = 0, 1, 2
@@ -281,6 +283,33 @@ def fork_state(lay, s_prefix, lq, lk, lv, alpha, beta, rule: str = "delta"):
                         np.asarray(lv[f, h], np.float64), float(alpha[f, h]), float(beta[f, h]))
                 s_fork[c, h] = S
     return o, s_fork
+
+
+def prefill_state(prefix_len, s_init, lq, lk, lv, alpha, beta, rule: str = "delta"):
+    """The prefix recurrent state (the prefill of a linear-attention layer):
+    request r's P_r prefix tokens fed in order through the recurrence from
+    s_init[r] (zeros when s_init is None). Token arrays are [sum P, Hl, .].
+    Returns (o [sum P, Hl, dv], s_out [R, Hl, dk, dv]); s_out is the state
+    jet_fork_state forks from (Sec. 4.1)."""
+    step = RULES[rule]
+    prefix_len = np.asarray(prefix_len, np.int64)
+    R = len(prefix_len)
+    total, Hl, dk = np.asarray(lk).shape
+    dv = np.asarray(lv).shape[2]
+    o = np.zeros((total, Hl, dv), np.float64)
+    s_out = np.zeros((R, Hl, dk, dv), np.float64)
+    p0 = 0
+    for r in range(R):
+        for h in range(Hl):
+            S = np.zeros((dk, dv)) if s_init is None else np.asarray(s_init[r, h], np.float64).copy()
+            for p in range(p0, p0 + int(prefix_len[r])):
+                S, o[p, h] = step(S, np.asarray(lq[p, h], np.float64),
+                                  np.asarray(lk[p, h], np.float64),
+                                  np.asarray(lv[p, h], np.float64),
+                                  float(alpha[p, h]), float(beta[p, h]))
+            s_out[r, h] = S
+        p0 += int(prefix_len[r])
+    return o, s_out
 
 
 # ----------------------------------------------------------------------------

@@ -599,3 +599,45 @@ def test_prefill_is_causal():
     b = O.prefill_attention(P, q, k2, v2, 2, 1)
     np.testing.assert_array_equal(a[:4], b[:4])
     assert not np.allclose(a[4:], b[4:])
+
+
+# ---------------------------------------------------------------------------
+# prefill of the recurrent state
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("rule", ["delta", "gla"])
+def test_prefill_state_then_fork_equals_one_scan(rule):
+    # scanning prefix ++ candidate tokens in one pass equals forking the
+    # candidate from the scanned prefix state (the state the fork reuses)
+    rng = np.random.default_rng(51)
+    Hl, dk, dv = 2, 4, 3
+    P = [4, 3]
+    cand = [[2, 3], [1]]                          # candidate lengths m_c
+    lay = O.build_layout(P, [2, 1], [2, 3, 1], list(range(6)), 8)
+    F = lay["N"] - lay["R"]
+    pk = rng.normal(size=(7, Hl, dk)); pq = rng.normal(size=(7, Hl, dk)); pv = rng.normal(size=(7, Hl, dv))
+    pa, pb = rng.uniform(0.9, 1, (7, Hl)), rng.uniform(0, 1, (7, Hl))
+    fk = rng.normal(size=(F, Hl, dk)); fq = rng.normal(size=(F, Hl, dk)); fv = rng.normal(size=(F, Hl, dv))
+    fa, fb = rng.uniform(0.9, 1, (F, Hl)), rng.uniform(0, 1, (F, Hl))
+    s0 = rng.normal(size=(2, Hl, dk, dv))
+    o_pre, s_pre = O.prefill_state(P, s0, pq, pk, pv, pa, pb, rule)
+    _, s_fork = O.fork_state(lay, s_pre, fq, fk, fv, fa, fb, rule=rule)
+    # candidate 1 of request 0 (m = 3) feeds fed tokens 1, 2: scan prefix 0 + those
+    cat = lambda x, y: np.concatenate([x[0:4], y[1:3]])  # noqa: E731
+    _, s_one = O.prefill_state([6], s0[:1], cat(pq, fq), cat(pk, fk), cat(pv, fv),
+                               cat(pa, fa), cat(pb, fb), rule)
+    np.testing.assert_allclose(s_fork[1], s_one[0], rtol=1e-12, atol=1e-13)
+    # the outputs of the prefix positions are the one-pass scan's first outputs
+    o_one, _ = O.prefill_state([4], s0[:1], pq[:4], pk[:4], pv[:4], pa[:4], pb[:4], rule)
+    np.testing.assert_allclose(o_pre[:4], o_one, rtol=1e-13)
+
+
+def test_prefill_state_zero_init_and_empty_writes():
+    rng = np.random.default_rng(52)
+    Hl, dk, dv = 1, 3, 2
+    k = rng.normal(size=(2, Hl, dk)); q = rng.normal(size=(2, Hl, dk)); v = rng.normal(size=(2, Hl, dv))
+    a = np.full((2, Hl), 0.5); b = np.zeros((2, Hl))       # beta = 0: nothing is written
+    s0 = rng.normal(size=(1, Hl, dk, dv))
+    _, s = O.prefill_state([2], s0, q, k, v, a, b)
+    np.testing.assert_allclose(s, 0.25 * s0, rtol=1e-15)      # two decays of 1/2
+    _, z = O.prefill_state([2], None, q, k, v, a, b)
+    assert np.all(z == 0)
