@@ -476,10 +476,42 @@ def run_gpu(args):
 # ---------------------------------------------------------------------------
 # the prefill (a "next" row, one GPU): causal attention over the prefixes
 # ---------------------------------------------------------------------------
+def _time_stream(fn, stream, warmup, steps):
+    """Average milliseconds of fn() over `steps` launches on `stream` (CUDA
+    events on that stream, after `warmup` untimed calls)."""
+    import torch
+    with torch.cuda.stream(stream):
+        for _ in range(warmup):
+            fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(steps):
+            fn()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / steps
+
+
+def _roof(flops, nbytes, ms, peaks):
+    """The binding roofline of a kernel with the given algorithmic work."""
+    tf = flops / (ms / 1e3) / 1e12
+    gbs = nbytes / (ms / 1e3) / 1e9
+    ridge = peaks["bf16"] * 1e12 / (peaks["hbm"] * 1e9)
+    if flops / nbytes >= ridge:
+        return dict(bound="tensor", achieved=round(tf, 1), peak=peaks["bf16"], unit="TFLOP/s",
+                    frac=round(tf / peaks["bf16"], 4))
+    return dict(bound="hbm", achieved=round(gbs, 1), peak=peaks["hbm"], unit="GB/s",
+                frac=round(gbs / peaks["hbm"], 4))
+
+
 def run_prefill(args):
-    """Times jet_prefill_attend on the workload's prefixes (their queries,
-    keys and values resident in HBM) and prints one JSON line: prefix tokens
-    per second, with the tensor roofline of the causal attention."""
+    """Times the prefill of the workload's prefixes (inputs resident in HBM):
+    jet_prefill_attend (causal self-attention) and, for hybrid workloads,
+    jet_prefill_state (the recurrent-state scan of a linear-attention layer).
+    Prints one JSON line: prefix tokens per second through both, with each
+    part's roofline."""
     import torch
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
@@ -495,50 +527,65 @@ def run_prefill(args):
         return
     hl = jet.jet_layout_build(p.prefix_len, p.n_cand, p.cand_len, p.target_ids, w.V)
     lay = hl.to_device(dev)
+    stream = torch.cuda.Stream(dev)
+    peaks = _peaks()
+    P = p.prefix_len.astype(np.float64)
+    parts = {}
+
     dims = jet.make_dims(jet.DTYPE_BF16, Hq=w.Hq, Hkv=w.Hkv, d=w.d, D=w.D)
     q, k, v = (jet_synth.torch_tensor(p, n, device=dev) for n in ("q_pre", "k_pre", "v_pre"))
-    p.drop()
     o = torch.empty(p.total_prefix, w.Hq, w.d, dtype=torch.bfloat16, device=dev)
     wsb = jet.jet_prefill_workspace_bytes(hl.sizes, dims)
     ws = torch.empty((wsb + 15) // 16 * 4, dtype=torch.float32, device=dev)
-    stream = torch.cuda.Stream(dev)
-    with torch.cuda.stream(stream):
-        for _ in range(args.warmup):
-            jet.jet_prefill_attend(lay, dims, q, k, v, o, ws, stream=stream)
-    torch.cuda.synchronize(dev)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    with torch.cuda.stream(stream):
-        for _ in range(args.steps):
-            jet.jet_prefill_attend(lay, dims, q, k, v, o, ws, stream=stream)
-    e1.record(stream)
-    torch.cuda.synchronize(dev)
+    ms = _time_stream(lambda: jet.jet_prefill_attend(lay, dims, q, k, v, o, ws, stream=stream),
+                      stream, args.warmup, args.steps)
     assert jet.jet_device_status(stream) == 0
-    ms = e0.elapsed_time(e1) / args.steps
-    P = p.prefix_len.astype(np.float64)
+    del q, k, v, o, ws
     # S = QK^T and O = PV over the causal triangle (keys 0..p of position p)
     flops = float(np.sum(4.0 * w.Hq * w.d * P * (P + 1) / 2))
     nbytes = p.total_prefix * (2 * w.Hq + 2 * w.Hkv) * w.d * 2  # Q, O, K, V once
-    peaks = _peaks()
-    tf = flops / (ms / 1e3) / 1e12
-    gbs = nbytes / (ms / 1e3) / 1e9
-    ridge = peaks["bf16"] * 1e12 / (peaks["hbm"] * 1e9)
-    if flops / nbytes >= ridge:
-        roof = dict(bound="tensor", achieved=round(tf, 1), peak=peaks["bf16"], unit="TFLOP/s",
-                    frac=round(tf / peaks["bf16"], 4))
-    else:
-        roof = dict(bound="hbm", achieved=round(gbs, 1), peak=peaks["hbm"], unit="GB/s",
-                    frac=round(gbs / peaks["hbm"], 4))
+    roof = _roof(flops, nbytes, ms, peaks)
     roof.update(kernel="jet_prefill_attend (work list + attend_prefix_tc_kernel, causal)",
                 algorithmic_flops=flops, algorithmic_bytes=nbytes, traffic=None,
                 peak_source=peaks["source"])
+    parts["attend"] = dict(ms=round(ms, 4), roofline=roof, launches=2)
+
+    if w.Hl > 0:
+        ldims = jet.make_dims(jet.DTYPE_BF16, Hl=w.Hl, dk=w.dk, dv=w.dv, D=w.D)
+        t = {n: jet_synth.torch_tensor(p, n, device=dev)
+             for n in ("lq_pre", "lk_pre", "lv_pre", "alpha_pre", "beta_pre", "s_prefix")}
+        lo = torch.empty(p.total_prefix, w.Hl, w.dv, dtype=torch.bfloat16, device=dev)
+        s_out = torch.empty(R, w.Hl, w.dk, w.dv, dtype=torch.float32, device=dev)
+        rule = jet.RULES[args.rule]
+        ms_s = _time_stream(
+            lambda: jet.jet_prefill_state(lay, ldims, t["lq_pre"], t["lk_pre"], t["lv_pre"],
+                                          t["alpha_pre"], t["beta_pre"], lo, s_out,
+                                          s_init=t["s_prefix"], rule=rule, stream=stream),
+            stream, args.warmup, args.steps)
+        assert jet.jet_device_status(stream) == 0
+        # q, k, v and the output once, the gates, and the start and final states
+        sbytes = (p.total_prefix * w.Hl * ((2 * w.dk + 2 * w.dv) * 2 + 8)
+                  + 2 * R * w.Hl * w.dk * w.dv * 4)
+        # per token and head: u = k^T S, the rank-one update, o = S^T q
+        sflops = float(p.total_prefix * w.Hl * w.dk * w.dv * (6 if args.rule == "delta" else 4))
+        sroof = _roof(sflops, sbytes, ms_s, peaks)
+        sroof.update(kernel=f"jet_prefill_state (scan_kernel, {args.rule} rule)",
+                     algorithmic_flops=sflops, algorithmic_bytes=sbytes, traffic=None,
+                     peak_source=peaks["source"])
+        parts["state"] = dict(ms=round(ms_s, 4), roofline=sroof, launches=1)
+        del t, lo, s_out
+    p.drop()
+    total_ms = sum(x["ms"] for x in parts.values())
+    dom = max(parts.values(), key=lambda x: x["ms"])
     print(json.dumps(dict(
-        metric="prefix tokens prefilled/sec", value=round(p.total_prefix / (ms / 1e3), 1),
+        metric="prefix tokens prefilled/sec", value=round(p.total_prefix / (total_ms / 1e3), 1),
         unit="tokens/s", n_gpus=1, steps=args.steps, warmup=args.warmup,
-        ms_per_step=round(ms, 4), higher_is_better=True, dtype="bf16", data="synthetic",
+        ms_per_step=round(total_ms, 4), higher_is_better=True, dtype="bf16", data="synthetic",
         config=dict(workload=args.workload, R=R, total_prefix=p.total_prefix,
-                    max_prefix=int(P.max()), Hq=w.Hq, Hkv=w.Hkv, d=w.d),
-        roofline=roof, gpu_launches=2 * args.steps)), flush=True)
+                    max_prefix=int(P.max()), Hq=w.Hq, Hkv=w.Hkv, d=w.d, Hl=w.Hl,
+                    rule=args.rule if w.Hl > 0 else None),
+        roofline=dom["roofline"], parts=parts,
+        gpu_launches=sum(x["launches"] for x in parts.values()) * args.steps)), flush=True)
 
 
 # ---------------------------------------------------------------------------

@@ -232,6 +232,24 @@ jet_status jet_prefill_attend(const jet_layout* lay, const jet_dims* dims, const
                               void* stream);
 
 /*
+ * jet_prefill_state - the prefill of a linear-attention layer: every request's
+ * P_r prefix tokens fed in order through the recurrence `rule` (JET_RECUR_*,
+ * as for jet_fork_state_rule) starting from s_init.
+ *   s_init  [R, Hl, dk, dv] float32   initial states; NULL means zeros
+ *   q, k    [total_prefix, Hl, dk] dims.dtype; v [total_prefix, Hl, dv]
+ *   alpha, beta [total_prefix, Hl] float32
+ *   o       [total_prefix, Hl, dv] dims.dtype  each prefix token's output
+ *   s_out   [R, Hl, dk, dv] float32   the state after the prefix: the
+ *           s_prefix every candidate forks from (Sec. 4.1)
+ * Tokens run one after another within a request (requests, heads and
+ * 32-column slices of the state run in parallel).
+ */
+jet_status jet_prefill_state(const jet_layout* lay, const jet_dims* dims, int32_t rule,
+                             const float* s_init, const void* q, const void* k, const void* v,
+                             const float* alpha, const float* beta, void* o, float* s_out,
+                             void* stream);
+
+/*
  * jet_fork_state - per-candidate fork of a linear-attention recurrent state
  * (Sec. 4.1: each candidate continues from the unchanged prefix state).
  *   s_prefix [R, Hl, dk, dv] float32  state after the prefix (read only)

@@ -214,6 +214,29 @@ extern "C" jet_status jet_prefill_attend(const jet_layout* lay, const jet_dims* 
                                             static_cast<cudaStream_t>(stream)));
 }
 
+extern "C" jet_status jet_prefill_state(const jet_layout* lay, const jet_dims* dims, int32_t rule,
+                                        const float* s_init, const void* q, const void* k,
+                                        const void* v, const float* alpha, const float* beta,
+                                        void* o, float* s_out, void* stream) {
+  JET_TRY(check_layout(lay));
+  JET_TRY(check_fork_dims(dims));
+  if (rule != JET_RECUR_DELTA && rule != JET_RECUR_GLA) return JET_ERR_ARG;
+  const jet_sizes& n = lay->n;
+  if (n.R == 0) return JET_OK;
+  if (n.R > 65535 || dims->Hl > 65535) return JET_ERR_CAPACITY;
+  if (s_init && !aligned16(s_init)) return JET_ERR_ALIGN;
+  JET_TRY(check_ptr(q, n.total_prefix));
+  JET_TRY(check_ptr(k, n.total_prefix));
+  JET_TRY(check_ptr(v, n.total_prefix));
+  JET_TRY(check_ptr(alpha, n.total_prefix));
+  JET_TRY(check_ptr(beta, n.total_prefix));
+  JET_TRY(check_ptr(o, n.total_prefix));
+  JET_TRY(check_ptr(s_out, n.R));
+  return cuda_status(jet::launch_prefill_state(*lay, *dims, rule, s_init, q, k, v, alpha, beta, o,
+                                               s_out, jet::device_status_ptr(),
+                                               static_cast<cudaStream_t>(stream)));
+}
+
 extern "C" jet_status jet_fork_state_rule(const jet_layout* lay, const jet_dims* dims,
                                           int32_t rule, const float* s_prefix, const void* q,
                                           const void* k, const void* v, const float* alpha,

@@ -68,6 +68,11 @@ cudaError_t launch_attend_tc(const jet_layout& lay, const jet_dims& d, const Att
                              const void* k_cand, const void* v_cand, void* o, float* o_part,
                              float2* ml_part, int* status, cudaStream_t st);
 
+// the prefix scan of the recurrent state (prefill of a linear-attention layer)
+cudaError_t launch_prefill_state(const jet_layout& lay, const jet_dims& d, int rule,
+                                 const float* s_init, const void* q, const void* k, const void* v,
+                                 const float* alpha, const float* beta, void* o, float* s_out,
+                                 int* status, cudaStream_t st);
 // rule: JET_RECUR_DELTA or JET_RECUR_GLA
 // causal self-attention over every request's prefix (bf16, tensor cores);
 // the workspace holds the work list

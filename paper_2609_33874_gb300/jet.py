@@ -83,6 +83,8 @@ def _load() -> ctypes.CDLL:
                                              ctypes.POINTER(jet_dims)]),
         "jet_prefill_attend": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
                                    P, P, P, P, P, SZ, P]),
+        "jet_prefill_state": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims), I,
+                                  P, P, P, P, P, P, P, P, P]),
         "jet_fork_state": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
                                P, P, P, P, P, P, P, P, P]),
         "jet_fork_state_rule": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims), I,
@@ -109,7 +111,7 @@ def _load() -> ctypes.CDLL:
 _lib = _load()
 DECLARED = ("jet_abi_version", "jet_status_string", "jet_layout_plan", "jet_layout_words",
             "jet_layout_build", "jet_layout_bind", "jet_workspace_bytes", "jet_prefix_attend",
-            "jet_prefill_workspace_bytes", "jet_prefill_attend",
+            "jet_prefill_workspace_bytes", "jet_prefill_attend", "jet_prefill_state",
             "jet_fork_state", "jet_fork_state_rule", "jet_score_candidates", "jet_score_candidates_noalloc",
             "jet_quantize_rows_e4m3", "jet_workspace_bytes_e4m3", "jet_score_candidates_e4m3",
             "jet_decide", "jet_evaluate", "jet_device_status")
@@ -248,6 +250,15 @@ def jet_prefill_attend(layout, dims: jet_dims, q, k, v, o, ws, ws_bytes: Optiona
     _check(_lib.jet_prefill_attend(ctypes.byref(_lay(layout)), ctypes.byref(dims), _addr(q),
                                    _addr(k), _addr(v), _addr(o), _addr(ws), int(ws_bytes),
                                    _stream(stream)), "jet_prefill_attend")
+
+
+def jet_prefill_state(layout, dims: jet_dims, q, k, v, alpha, beta, o, s_out, s_init=None,
+                      rule: int = 0, stream=None) -> None:
+    """The prefix scan of the recurrent state (see include/jet.h)."""
+    _check(_lib.jet_prefill_state(ctypes.byref(_lay(layout)), ctypes.byref(dims), int(rule),
+                                  _addr(s_init), _addr(q), _addr(k), _addr(v), _addr(alpha),
+                                  _addr(beta), _addr(o), _addr(s_out), _stream(stream)),
+           "jet_prefill_state")
 
 
 def jet_fork_state(layout, dims: jet_dims, s_prefix, q, k, v, alpha, beta, o, s_fork=None,

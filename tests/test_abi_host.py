@@ -194,6 +194,26 @@ def test_fork_rule_validation(jet):
                                    *args) == 7
 
 
+def test_prefill_state_validation(jet):
+    lay, dims = _setup(jet)
+    lib = jet.library()
+    L, D = ctypes.byref(lay.struct), ctypes.byref(dims)
+    # rule, s_init (nullable), q, k, v, alpha, beta, o, s_out, stream
+    args = [FAKE] * 8 + [None]
+    assert lib.jet_prefill_state(L, D, 5, *args) == 1                      # unknown rule
+    bad = jet.make_dims(jet.DTYPE_BF16, Hl=2, dk=64, dv=64)
+    assert lib.jet_prefill_state(L, ctypes.byref(bad), jet.RECUR_DELTA, *args) == 7
+    nul = list(args)
+    nul[5] = None  # beta
+    assert lib.jet_prefill_state(L, D, jet.RECUR_GLA, *nul) == 1
+    mis = list(args)
+    mis[0] = MIS   # s_init is optional but must be aligned when given
+    assert lib.jet_prefill_state(L, D, jet.RECUR_DELTA, *mis) == 4
+    mis = list(args)
+    mis[7] = MIS   # s_out
+    assert lib.jet_prefill_state(L, D, jet.RECUR_DELTA, *mis) == 4
+
+
 def test_e4m3_validation(jet):
     lay, dims = _setup(jet)
     lib = jet.library()

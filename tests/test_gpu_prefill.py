@@ -1,7 +1,9 @@
 """GPU parity of the prefill - causal self-attention over every request's
 prefix - through the C ABI against the oracle on the same seeded inputs:
 ragged prefixes around the 64-key tile and the query-block size, every head
-dimension, and the full-size dense27b_mc prefixes (sampled rows)."""
+dimension, and the full-size dense27b_mc prefixes (sampled rows); and of the
+prefix scan of a linear-attention layer's recurrent state (both rules, both
+dtypes, prefixes around the 32-token staging window, the full hybrid prefixes)."""
 import dataclasses
 
 import numpy as np
@@ -9,7 +11,7 @@ import pytest
 
 import jet_synth
 import oracle as O
-from gpu_common import TOL_ATTN_BF16
+from gpu_common import TOL_ATTN_BF16, TOL_FORK_REL
 
 pytestmark = pytest.mark.gpu
 
@@ -84,3 +86,69 @@ def test_prefill_full_size_dense27b_mc(cuda):
     p = jet_synth.make_problem("dense27b_mc")
     got = _prefill(cuda, p)
     _check(p, got, _sample_rows(p.prefix_len, np.random.default_rng(7), per=4))
+
+
+# ---------------------------------------------------------------------------
+# prefill of the recurrent state (the prefix scan)
+# ---------------------------------------------------------------------------
+def _scan(cuda, p, rule, with_init):
+    import torch
+    w = p.work
+    hl = cuda.jet_layout_build(p.prefix_len, p.n_cand, p.cand_len, p.target_ids, w.V)
+    dims = cuda.make_dims(cuda.DTYPE_BF16 if p.bf16 else cuda.DTYPE_F32, Hl=w.Hl, dk=w.dk,
+                          dv=w.dv, D=w.D)
+    t = {n: jet_synth.torch_tensor(p, n, device="cuda")
+         for n in ("lq_pre", "lk_pre", "lv_pre", "alpha_pre", "beta_pre")}
+    s_init = jet_synth.torch_tensor(p, "s_prefix", device="cuda") if with_init else None
+    dt = torch.bfloat16 if p.bf16 else torch.float32
+    o = torch.empty(p.total_prefix, w.Hl, w.dv, dtype=dt, device="cuda")
+    s_out = torch.empty(p.R, w.Hl, w.dk, w.dv, dtype=torch.float32, device="cuda")
+    cuda.jet_prefill_state(hl.to_device("cuda"), dims, t["lq_pre"], t["lk_pre"], t["lv_pre"],
+                           t["alpha_pre"], t["beta_pre"], o, s_out, s_init=s_init,
+                           rule=cuda.RULES[rule])
+    torch.cuda.synchronize()
+    assert cuda.jet_device_status() == 0
+    return o.float().cpu().numpy(), s_out.cpu().numpy()
+
+
+def _check_scan_out(got, ref, bf16):
+    # outputs are stored in the workload's dtype: bf16 rounds each to 8
+    # significant bits (relative 2^-9), float32 to 24; the state itself is
+    # float32 throughout
+    atol, rtol = (1e-3, 8e-3) if bf16 else (1e-5, 1e-5)
+    err = np.abs(got - ref) - (atol + rtol * np.abs(ref))
+    assert err.max() <= 0, f"scan output error {np.abs(got - ref).max()}"
+
+
+@pytest.mark.parametrize("rule", ["delta", "gla"])
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_prefill_state(cuda, rule, dtype):
+    # prefixes around the 32-token staging window; with and without a start state
+    w = dataclasses.replace(jet_synth.WORKLOADS["ordinal_hybrid"], Hl=3, dv=64, dtype=dtype)
+    pl = [1, 31, 32, 33, 70]
+    R = len(pl)
+    p = jet_synth.custom_problem(w, pl, [1] * R, [1] * R, [0] * R, seed=95)
+    for with_init in (False, True):
+        got_o, got_s = _scan(cuda, p, rule, with_init)
+        ref_o, ref_s = O.prefill_state(p.prefix_len, p.f32("s_prefix") if with_init else None,
+                                       p.f32("lq_pre"), p.f32("lk_pre"), p.f32("lv_pre"),
+                                       p.f32("alpha_pre"), p.f32("beta_pre"), rule)
+        rel = np.abs(got_s - ref_s).max() / np.abs(ref_s).max()
+        assert rel <= TOL_FORK_REL, f"state error {rel}"
+        _check_scan_out(got_o, ref_o, p.bf16)
+
+
+def test_prefill_state_full_hybrid(cuda):
+    # the hybrid workload's prefixes (32 requests x 512 tokens, 16 heads)
+    p = jet_synth.make_problem("ordinal_hybrid")
+    got_o, got_s = _scan(cuda, p, "delta", True)
+    sub = [0, 13, 31]
+    off = np.concatenate([[0], np.cumsum(p.prefix_len)])
+    rows = np.concatenate([np.arange(off[r], off[r + 1]) for r in sub])
+    sel = lambda n: p.f32(n)[rows]  # noqa: E731
+    ref_o, ref_s = O.prefill_state(p.prefix_len[sub], p.f32("s_prefix")[sub], sel("lq_pre"),
+                                   sel("lk_pre"), sel("lv_pre"), sel("alpha_pre"),
+                                   sel("beta_pre"))
+    rel = np.abs(got_s[sub] - ref_s).max() / np.abs(ref_s).max()
+    assert rel <= TOL_FORK_REL, f"state error {rel}"
+    _check_scan_out(got_o[rows], ref_o, True)
