@@ -568,8 +568,15 @@ def run_prefill(args):
                   + 2 * R * w.Hl * w.dk * w.dv * 4)
         # per token and head: u = k^T S, the rank-one update, o = S^T q
         sflops = float(p.total_prefix * w.Hl * w.dk * w.dv * (6 if args.rule == "delta" else 4))
-        sroof = _roof(sflops, sbytes, ms_s, peaks)
+        # the scan is sequential per (request, head): it is bound by fp32 FMA
+        # issue, 152 SMs x 128 lanes x 2 flop per clock at the maximum SM clock
+        alu_peak = 152 * 128 * 2 * peaks["sm_max_mhz"] * 1e6 / 1e12
+        tf_s = sflops / (ms_s / 1e3) / 1e12
+        sroof = dict(bound="alu", achieved=round(tf_s, 2), peak=round(alu_peak, 1),
+                     unit="TFLOP/s", frac=round(tf_s / alu_peak, 4),
+                     hbm_frac=round(sbytes / (ms_s / 1e3) / 1e9 / peaks["hbm"], 4))
         sroof.update(kernel=f"jet_prefill_state (scan_kernel, {args.rule} rule)",
+                     peak_basis="fp32 FMA: 152 SMs x 128 lanes x 2 flop x max SM clock",
                      algorithmic_flops=sflops, algorithmic_bytes=sbytes, traffic=None,
                      peak_source=peaks["source"])
         parts["state"] = dict(ms=round(ms_s, 4), roofline=sroof, launches=1)

@@ -251,65 +251,6 @@ fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__
   }
 }
 
-// The prefix scan (prefill of the recurrent state): grid (dv / 32, Hl, R); a
-// CTA feeds its request's P prefix tokens, 32 at a time staged in shared
-// memory, through the recurrence from s_init (zeros when null), writes every
-// token's output and the final state.
-template <typename T, bool DELTA>
-__global__ void __launch_bounds__(kThreads)
-scan_kernel(const int32_t* __restrict__ prefix_offset, int R, int total, int Hl, int dv,
-            const float* __restrict__ s_init, const T* __restrict__ q, const T* __restrict__ k,
-            const T* __restrict__ v, const float* __restrict__ alpha,
-            const float* __restrict__ beta, T* __restrict__ o, float* __restrict__ s_out,
-            int* status) {
-  pdl_begin();
-  __shared__ __align__(16) float red[4 * kCols];
-  __shared__ __align__(16) T wk[kWin][kDK];
-  __shared__ __align__(16) T wq[kWin][kDK];
-  __shared__ __align__(16) T wv[kWin][kCols];
-  __shared__ __align__(16) float wa[kWin], wb[kWin];
-  const int r = blockIdx.z, h = blockIdx.y, j0 = blockIdx.x * kCols;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int rg = lane >> 3, jq = lane & 7;
-  const int col = j0 + 4 * jq;
-  if (r >= R) return;
-  const int p0 = prefix_offset[r], p1 = prefix_offset[r + 1];
-  if (p0 < 0 || p1 < p0 || p1 > total) {
-    if (tid == 0) flag(status, JET_ERR_DEVICE);
-    return;
-  }
-  const size_t head = (size_t(r) * Hl + h) * kDK;
-  float4 S[8];
-#pragma unroll
-  for (int ii = 0; ii < 8; ++ii) {
-    const int i = 32 * warp + rg + 4 * ii;
-    S[ii] = s_init ? *reinterpret_cast<const float4*>(s_init + (head + i) * dv + col)
-                   : make_float4(0.f, 0.f, 0.f, 0.f);
-  }
-  const float rs = rsqrtf(float(kDK));
-  for (int w0 = p0; w0 < p1; w0 += kWin) {
-    const int nt = min(kWin, p1 - w0);
-    __syncthreads();  // the previous window is no longer read
-    stage_window(q, k, v, alpha, beta, Hl, dv, h, j0, w0, nt, tid, wk, wq, wv, wa, wb);
-    __syncthreads();
-    for (int t = 0; t < nt; ++t) {
-      const float4 op = token_step<T, DELTA>(S, t, wk, wq, wv, wa, wb, red, warp, lane);
-      if (warp == 0 && rg == 0) {
-        T* dst = o + (size_t(w0 + t) * Hl + h) * dv + col;
-        dst[0] = from_f32<T>(op.x * rs);
-        dst[1] = from_f32<T>(op.y * rs);
-        dst[2] = from_f32<T>(op.z * rs);
-        dst[3] = from_f32<T>(op.w * rs);
-      }
-    }
-  }
-#pragma unroll
-  for (int ii = 0; ii < 8; ++ii) {
-    const int i = 32 * warp + rg + 4 * ii;
-    *reinterpret_cast<float4*>(s_out + (head + i) * dv + col) = S[ii];
-  }
-}
-
 }  // namespace
 
 namespace {
@@ -338,26 +279,6 @@ cudaError_t launch_rule(const jet_layout& lay, const jet_dims& d, const float* s
 
 }  // namespace
 
-cudaError_t launch_prefill_state(const jet_layout& lay, const jet_dims& d, int rule,
-                                 const float* s_init, const void* q, const void* k, const void* v,
-                                 const float* alpha, const float* beta, void* o, float* s_out,
-                                 int* status, cudaStream_t st) {
-  const jet_sizes& n = lay.n;
-  dim3 grid(unsigned(d.dv / kCols), unsigned(d.Hl), unsigned(n.R));
-#define JET_SCAN(T, DELTA)                                                                   \
-  return launch_pdl(scan_kernel<T, DELTA>, grid, dim3(kThreads), 0, st, lay.prefix_offset, n.R, \
-                    n.total_prefix, d.Hl, d.dv, s_init, static_cast<const T*>(q),             \
-                    static_cast<const T*>(k), static_cast<const T*>(v), alpha, beta,          \
-                    static_cast<T*>(o), s_out, status)
-  const bool delta = rule != JET_RECUR_GLA;
-  if (d.dtype == JET_DTYPE_F32) {
-    if (delta) JET_SCAN(float, true);
-    JET_SCAN(float, false);
-  }
-  if (delta) JET_SCAN(__nv_bfloat16, true);
-  JET_SCAN(__nv_bfloat16, false);
-#undef JET_SCAN
-}
 
 cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, int rule,
                               const float* s_prefix, const void* q, const void* k, const void* v,

@@ -152,3 +152,19 @@ def test_prefill_state_full_hybrid(cuda):
     rel = np.abs(got_s[sub] - ref_s).max() / np.abs(ref_s).max()
     assert rel <= TOL_FORK_REL, f"state error {rel}"
     _check_scan_out(got_o[rows], ref_o, True)
+
+
+@pytest.mark.parametrize("dv", [32, 160])
+def test_prefill_state_column_tails(cuda, dv):
+    # dv % 64 == 32: the last 64-column block of each head is half full
+    w = dataclasses.replace(jet_synth.WORKLOADS["ordinal_hybrid"], Hl=2, dv=dv, dtype="bf16")
+    pl = [17, 48, 3]
+    R = len(pl)
+    p = jet_synth.custom_problem(w, pl, [1] * R, [1] * R, [0] * R, seed=96)
+    got_o, got_s = _scan(cuda, p, "delta", True)
+    ref_o, ref_s = O.prefill_state(p.prefix_len, p.f32("s_prefix"), p.f32("lq_pre"),
+                                   p.f32("lk_pre"), p.f32("lv_pre"), p.f32("alpha_pre"),
+                                   p.f32("beta_pre"), "delta")
+    rel = np.abs(got_s - ref_s).max() / np.abs(ref_s).max()
+    assert rel <= TOL_FORK_REL, f"state error {rel}"
+    _check_scan_out(got_o, ref_o, True)
