@@ -274,16 +274,16 @@ def run_gpu(args):
     dims = jet.make_dims(dtype, Hq=w.Hq, Hkv=w.Hkv, d=w.d, D=w.D, Hl=w.Hl, dk=w.dk, dv=w.dv)
     hl = jet.jet_layout_build(problem.prefix_len, problem.n_cand, problem.cand_len,
                               problem.target_ids, w.V)
-    e4m3 = args.lm == "e4m3"
+    low = args.lm != "bf16"   # e4m3 or 4-bit weights, e4m3 hidden states
     step = ScoringStep(hl, dims, jet.MODES[w.mode], device=dev, hybrid=w.Hl > 0,
                        keep_fork_state=w.Hl > 0, lm=args.lm, rule=args.rule)
     names = step.input_names()
     x = {k: jet_synth.torch_tensor(problem, k, device=dev) for k in names}
     w_lm = jet_synth.torch_tensor(problem, "w_lm", device=dev)
-    if e4m3:
+    if low:
         # model state: the weights are quantised once, outside the timed region
-        from paper_2609_33874_gb300.step import quantize_lm_head
-        w_lm = quantize_lm_head(w_lm)
+        from paper_2609_33874_gb300.step import quantize_lm_head, quantize_lm_head_w4
+        w_lm = (quantize_lm_head_w4 if args.lm == "w4" else quantize_lm_head)(w_lm)
         torch.cuda.synchronize(dev)
     stream = torch.cuda.Stream(dev)
 
@@ -395,18 +395,21 @@ def run_gpu(args):
     es = 2 if w.dtype == "bf16" else 4
     vtiles = (w.V + 127) // 128
     lm_bytes = w.V * w.D * es + N * w.D * es + vtiles * N * 8 + T * 4
-    if e4m3:
-        # w_lm codes + row scales, bf16 hidden in, its codes out and back, scales
-        lm_bytes = w.V * w.D + w.V * 4 + N * w.D * 2 + 2 * N * w.D + N * 4 + vtiles * N * 8 + T * 4
+    if low:
+        # w_lm codes (+ block exponents for w4) + row scales, bf16 hidden in, its
+        # codes out and back, scales
+        w_bytes = w.V * w.D if args.lm == "e4m3" else w.V * w.D // 2 + w.V * ((w.D + 31) // 32)
+        lm_bytes = w_bytes + w.V * 4 + N * w.D * 2 + 2 * N * w.D + N * 4 + vtiles * N * 8 + T * 4
     lm_flops = 2.0 * N * w.D * w.V
     score_avg_s = call_ms["score"] / 1e3
-    # e4m3 tensor peak: the measured bf16 peak x the nominal 2x of 8-bit operands
-    tc_peak = peaks["bf16"] * (2 if e4m3 else 1)
+    # e4m3 tensor peak (both low-precision heads multiply e4m3 operands): the
+    # measured bf16 peak x the nominal 2x of 8-bit operands
+    tc_peak = peaks["bf16"] * (2 if low else 1)
     ridge = tc_peak * 1e12 / (peaks["hbm"] * 1e9)
     kernel_file = "paper_2609_33874_gb300/csrc/lmhead_tc.cu" if w.dtype == "bf16" and \
         os.path.exists(os.path.join(ROOT, "paper_2609_33874_gb300/csrc/lmhead_tc.cu")) \
         else "paper_2609_33874_gb300/csrc/lmhead_simt.cu"
-    traffic = _traffic(kernel_file, args.workload + (":e4m3" if e4m3 else ""))
+    traffic = _traffic(kernel_file, args.workload + (":" + args.lm if low else ""))
     if w.dtype != "bf16":
         # float32 FMA: SMs x 128 lanes x 2 flop x the maximum SM clock
         sms = torch.cuda.get_device_properties(dev).multi_processor_count
@@ -422,8 +425,9 @@ def run_gpu(args):
         ach = lm_flops / score_avg_s / 1e12
         roof = dict(bound="tensor", achieved=round(ach, 1), peak=round(tc_peak, 1), unit="TFLOP/s",
                     frac=round(ach / tc_peak, 4), traffic=traffic)
-    roof.update(kernel="jet_score_candidates" + ("_e4m3 (quantise hidden + e4m3 LM head + lse "
-                                                 "merge)" if e4m3 else " (LM head + lse merge)"),
+    roof.update(kernel="jet_score_candidates" + (f"_{args.lm} (quantise hidden + {args.lm} LM head "
+                                                 "+ lse merge)" if low else
+                                                 " (LM head + lse merge)"),
                 algorithmic_bytes=lm_bytes, algorithmic_flops=lm_flops,
                 avg_launch_ms=round(score_avg_s * 1e3, 4), peak_source=peaks["source"])
 
@@ -443,18 +447,21 @@ def run_gpu(args):
                       + F * w.Hl * (2 * w.dk + 2 * w.dv) * es + F * w.Hl * 8)
         calls["fork"] = _call(call_ms["fork"], fork_bytes, peaks)
 
-    launches_per_step = _attend_launches(problem, w) + (1 if w.Hl else 0) + 3 + 1 + (1 if e4m3 else 0)
+    launches_per_step = _attend_launches(problem, w) + (1 if w.Hl else 0) + 3 + 1 + (1 if low else 0)
     result = dict(
         metric=METRIC, value=round(value, 2), unit=UNIT, n_gpus=world, steps=args.steps,
         warmup=args.warmup, ms_per_step=round(ms_per_step, 4), higher_is_better=True,
         scaling="weak", vs_baseline=None,
-        dtype=("bf16 (LM head e4m3)" if e4m3 else "bf16") if w.dtype == "bf16" else "f32",
+        dtype=(f"bf16 (LM head {args.lm})" if low else "bf16") if w.dtype == "bf16" else "f32",
         data="synthetic",
         config=dict(workload=args.workload, R=R, N=N, T=T, C=len(problem.cand_len),
                     total_prefix=problem.total_prefix, Hq=w.Hq, Hkv=w.Hkv, d=w.d, D=w.D, V=w.V,
                     Hl=w.Hl, parallelism=f"replicas{world}" if world > 1 else "single",
-                    lm_head="e4m3, one float32 scale per weight row and per token" if e4m3
-                    else "bf16",
+                    lm_head={"bf16": "bf16",
+                             "e4m3": "e4m3, one float32 scale per weight row and per token",
+                             "w4": "weights e2m1 with a power-of-two exponent per 32-element "
+                                   "block and a float32 scale per row; hidden e4m3 per token"}[
+                                       args.lm],
                     recurrence=(args.rule if w.Hl else None),
                     l2=f"inputs larger than L2: LM-head weights {w.V * w.D * es / 1e9:.2f} GB "
                        f"streamed every step"),
@@ -465,7 +472,7 @@ def run_gpu(args):
         roofline=roof,
         calls=calls,
     )
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and not e4m3:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and not low:
         result["cpu_baseline"] = cpu_baseline(args.workload, R, args.cpu_sample)
     if world > 1:
         torch.distributed.destroy_process_group()
@@ -642,9 +649,10 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--rule", default="delta", choices=["delta", "gla"],
                     help="recurrence of the linear-attention fork (hybrid workloads)")
-    ap.add_argument("--lm", default="bf16", choices=["bf16", "e4m3"],
-                    help="LM head precision: bf16 (the workload's), or e4m3 codes with one "
-                         "scale per weight row and per token (the paper's 8-bit weights)")
+    ap.add_argument("--lm", default="bf16", choices=["bf16", "e4m3", "w4"],
+                    help="LM head precision: bf16 (the workload's), e4m3 codes with one "
+                         "scale per weight row and per token (the paper's 8-bit weights), or "
+                         "w4: 4-bit weights in 32-element blocks (the paper's 4-bit weights)")
     ap.add_argument("--prefill", action="store_true",
                     help="time the prefill (causal attention over the workload's prefixes) "
                          "instead of the scoring step (one GPU)")

@@ -353,6 +353,63 @@ jet_status jet_score_candidates_e4m3(const jet_layout* lay, const jet_dims* dims
                                      size_t ws_bytes, void* stream);
 
 /*
+ * 4-bit LM head (w4; the analogue of the paper's 4-bit weights, Appendix A,
+ * whose codes come in 32-element blocks with their own scales). A row x of
+ * w_lm is stored as OCP FP4 E2M1 codes (1 sign, 2 exponent bits with bias 1,
+ * 1 mantissa bit: magnitudes 0, .5, 1, 1.5, 2, 3, 4, 6), one power-of-two
+ * exponent e in [-5, 0] per 32-element block and one float32 scale s per row,
+ * with x[k] ~= s * 2^e(k / 32) * value(code[k]):
+ *   amax = max |x|, s = amax / 6, inv = 6 / amax (float32, rounded to nearest);
+ *   block b: t = (max |x| over the block) * inv, e = the smallest integer in
+ *   [-5, 0] with t <= 6 * 2^e (0 if none); code = e2m1(x * (inv * 2^-e)),
+ *   nearest with ties to the even code, saturated at +-6. A row of zeros gets
+ *   s = 0, zero codes and e = -5.
+ *
+ * Tiled layout of the codes (the order the LM head streams them): one tile of
+ * 8,704 bytes per (vocabulary tile vt of 128 rows, K slice kb of 128
+ * elements), tile index vt * ceil(D / 128) + kb. Bytes [0, 8192): row r of
+ * the tile (vocabulary row 128 vt + r) has 64 bytes at r * 64; its 16-byte
+ * chunk c (elements 128 kb + 32 c .. + 31) is stored in slot c ^ ((r >> 1) & 3).
+ * A chunk is four little-endian 32-bit words of 8 elements each: nibble k
+ * (bits 4k .. 4k+3) holds the magnitude (3 bits) of element k of the word in
+ * its low bits and, in bit 3, the sign of element 4 + k / 2 (k even) or k / 2
+ * (k odd). Bytes [8192, 8704):
+ * the block exponents, int8, row r's four at 8192 + 4 r + c. Rows past V and
+ * elements past D are zero codes.
+ */
+
+/* Bytes of the tiled 4-bit codes of a [V, D] matrix:
+ * ceil(V / 128) * ceil(D / 128) * 8704; 0 on invalid arguments. */
+size_t jet_w4_bytes(int64_t V, int64_t D);
+
+/*
+ * jet_quantize_w4 - quantise the bf16 matrix w [V, D] (device, row-major) into
+ * w4 (jet_w4_bytes(V, D) bytes, 16-byte aligned) and scale [V] float32.
+ * Errors: JET_ERR_ARG (V < 1 or a null pointer), JET_ERR_SHAPE (D not a
+ * positive multiple of 16), JET_ERR_ALIGN. Done once per model (w_lm is model
+ * state).
+ */
+jet_status jet_quantize_w4(const void* w, int64_t V, int64_t D, uint8_t* w4, float* scale,
+                           void* stream);
+
+/*
+ * jet_score_candidates_w4 - jet_score_candidates with a 4-bit LM head:
+ *   hidden      [N, D] bf16     quantised per row (token) to e4m3 into the
+ *                               workspace, as in jet_score_candidates_e4m3
+ *   w4          tiled codes of w_lm from jet_quantize_w4 with the same V, D
+ *   w_scale     [V] float32     their per-row scales
+ * The logit is z[n, v] = s_h[n] s_w[v] sum_k decode(h_q[n, k]) 2^e value(code),
+ * accumulated in float32 on the tensor cores (each 2^e value(code) is an e4m3
+ * value, widened on chip); log-softmax, gather and sums as in
+ * jet_score_candidates. dims as for jet_score_candidates_e4m3; workspace
+ * jet_workspace_bytes_e4m3().
+ */
+jet_status jet_score_candidates_w4(const jet_layout* lay, const jet_dims* dims,
+                                   const void* hidden, const uint8_t* w4, const float* w_scale,
+                                   float* tok_logprob, float* cand_score, void* ws,
+                                   size_t ws_bytes, void* stream);
+
+/*
  * jet_score_candidates_noalloc - jet_score_candidates without caller-owned
  * scratch memory. The paper has no counterpart to this entry point: it exists
  * for callers that cannot call cudaMalloc, such as a host application that

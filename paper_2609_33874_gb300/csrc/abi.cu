@@ -341,6 +341,54 @@ extern "C" jet_status jet_score_candidates_e4m3(const jet_layout* lay, const jet
       jet::launch_score_finish(*lay, plan.score, ws, tok_logprob, cand_score, status, st));
 }
 
+extern "C" size_t jet_w4_bytes(int64_t V, int64_t D) {
+  if (V < 1 || D < 16 || D % 16 != 0 || V > (int64_t(1) << 31) || D > (int64_t(1) << 31))
+    return 0;
+  return size_t((V + jet::kVocabTile - 1) / jet::kVocabTile) * size_t((D + 127) / 128) *
+         size_t(jet::kW4TileBytes);
+}
+
+extern "C" jet_status jet_quantize_w4(const void* w, int64_t V, int64_t D, uint8_t* w4,
+                                      float* scale, void* stream) {
+  if (V < 1) return JET_ERR_ARG;
+  if (D < 16 || D % 16 != 0) return JET_ERR_SHAPE;
+  if (V > (int64_t(1) << 30) || D > (int64_t(1) << 20)) return JET_ERR_CAPACITY;
+  JET_TRY(check_ptr(w, V));
+  JET_TRY(check_ptr(w4, V));
+  JET_TRY(check_ptr(scale, V));
+  return cuda_status(jet::launch_quantize_w4(w, int(V), int(D), w4, scale,
+                                             static_cast<cudaStream_t>(stream)));
+}
+
+extern "C" jet_status jet_score_candidates_w4(const jet_layout* lay, const jet_dims* dims,
+                                              const void* hidden, const uint8_t* w4,
+                                              const float* w_scale, float* tok_logprob,
+                                              float* cand_score, void* ws, size_t ws_bytes,
+                                              void* stream) {
+  JET_TRY(check_layout(lay));
+  JET_TRY(check_e4m3_dims(dims));
+  const jet_sizes& n = lay->n;
+  if (n.R == 0) return JET_OK;
+  const E4m3Plan plan = e4m3_plan(n, dims->D);
+  if (plan.score.vtiles > 65535) return JET_ERR_CAPACITY;
+  JET_TRY(check_ptr(hidden, n.N));
+  JET_TRY(check_ptr(w4, n.V));
+  JET_TRY(check_ptr(w_scale, n.V));
+  JET_TRY(check_ptr(tok_logprob, n.T));
+  JET_TRY(check_ptr(cand_score, n.C));
+  if (!ws || ws_bytes < plan.bytes) return JET_ERR_WORKSPACE;
+  if (!aligned16(ws)) return JET_ERR_ALIGN;
+  int* status = jet::device_status_ptr();
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint8_t* h_q = static_cast<uint8_t*>(ws) + plan.hq_off;
+  float* h_scale = reinterpret_cast<float*>(static_cast<char*>(ws) + plan.hs_off);
+  JET_TRY(cuda_status(jet::launch_quantize_e4m3(hidden, n.N, dims->D, h_q, h_scale, st)));
+  JET_TRY(cuda_status(jet::launch_lmhead_w4(*lay, *dims, plan.score, h_q, h_scale, w4, w_scale,
+                                            ws, status, st)));
+  return cuda_status(
+      jet::launch_score_finish(*lay, plan.score, ws, tok_logprob, cand_score, status, st));
+}
+
 extern "C" jet_status jet_decide(const jet_layout* lay, int32_t mode, const float* cand_score,
                                  float* q, int32_t* choice, float* value, void* stream) {
   JET_TRY(check_layout(lay));

@@ -485,7 +485,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         q_par = v & 1;
         // K_j and V_j are issued as soon as their slots drain, whichever first
         int jk = 0, jv = 0;
-        uint64_t t_last = global_timer_ns();
+        IdleClock clk;
         while (jv < e.ntiles) {
           bool progressed = false;
           if (jk < e.ntiles) {
@@ -526,10 +526,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
               progressed = true;
             }
           }
-          const uint64_t now = global_timer_ns();
-          if (progressed) {
-            t_last = now;
-          } else if (*abort_flag || now - t_last > kWaitNs) {
+          if (clk.expired(progressed, abort_flag, kWaitNs)) {
             ok = false;
             break;
           }
@@ -575,7 +572,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         // issue S_j = Q K_j^T and O += P_j V_j in whichever order their inputs
         // become ready; S_j always precedes P_j V_j
         int js = 0, jo = 0;
-        uint64_t t_last = global_timer_ns();
+        IdleClock clk;
         while (ok && jo < e.ntiles) {
           bool progressed = false;
           if (js < e.ntiles) {
@@ -618,12 +615,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
               progressed = true;
             }
           }
-          const uint64_t now = global_timer_ns();
-          if (progressed) {
-            t_last = now;
-          } else if (*abort_flag || now - t_last > kWaitNs) {
-            ok = false;
-          }
+          if (clk.expired(progressed, abort_flag, kWaitNs)) ok = false;
         }
         if (!ok) break;
         mbar_arrive(item_empty + slot);

@@ -16,6 +16,10 @@ int* device_status_ptr();
 
 // ---- workspace plans -----------------------------------------------------------
 constexpr int kVocabTile = 128;  // vocabulary entries per LM-head partial
+// 4-bit weights: one tile per (128 vocabulary rows, 128-element K slice):
+// 128 x 64 bytes of packed E2M1 codes, then 128 x 4 block exponents
+constexpr int kW4CodeBytes = kVocabTile * 64;
+constexpr int kW4TileBytes = kW4CodeBytes + kVocabTile * 4;
 
 struct AttnPlan {
   int splits;    // prefix chunks per (request, key/value head)
@@ -98,6 +102,13 @@ cudaError_t launch_lmhead_tc(const jet_layout& lay, const jet_dims& d, const Sco
 cudaError_t launch_lmhead_e4m3(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
                                const uint8_t* h_q, const float* h_scale, const uint8_t* w_q,
                                const float* w_scale, void* ws, int* status, cudaStream_t st);
+// the LM head on tiled 4-bit weights (w4) and e4m3 hidden codes
+cudaError_t launch_lmhead_w4(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
+                             const uint8_t* h_q, const float* h_scale, const uint8_t* w4,
+                             const float* w_scale, void* ws, int* status, cudaStream_t st);
+// 4-bit quantisation of a bf16 matrix [V, D] into the tiled layout, scales [V]
+cudaError_t launch_quantize_w4(const void* x, int V, int D, uint8_t* w4, float* scale,
+                               cudaStream_t st);
 // per-row e4m3 quantisation of a bf16 matrix [rows, D] (D multiple of 16)
 cudaError_t launch_quantize_e4m3(const void* x, int rows, int D, uint8_t* q, float* scale,
                                  cudaStream_t st);

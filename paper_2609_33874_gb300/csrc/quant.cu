@@ -4,6 +4,14 @@
 // amax = max |x| (float32), s = amax / 448, q = e4m3(x * (448 / amax)) rounded
 // to nearest even and saturated at +-448 (448 is the largest e4m3 value). A
 // row of zeros gets s = 0 and zero codes.
+//
+// The 4-bit weights (w4; the paper's largest models use 4-bit weights in
+// scaled 32-element blocks, Appendix A) keep one float32 scale per row and, per
+// 32-element block, a power-of-two exponent e in [-5, 0] over OCP FP4 E2M1
+// codes: s = amax / 6, inv = 6 / amax, t = blockmax * inv, e = the smallest
+// value in [-5, 0] with t <= 6 * 2^e (0 if none), code = e2m1(x * (inv * 2^-e))
+// rounded to nearest even and saturated at +-6. They are written in the
+// tiled layout the LM head streams (see include/jet.h).
 #include <cuda_fp8.h>
 
 #include "jet_device.cuh"
@@ -51,7 +59,106 @@ quantize_e4m3_kernel(const __nv_bfloat16* __restrict__ x, int rows, int D,
   }
 }
 
+// E2M1 code of a float32 value: nearest of 0, .5, 1, 1.5, 2, 3, 4, 6, ties to
+// the even code (each comparison is with the midpoint to the next magnitude,
+// strict where the lower code is the even one), saturating, sign in bit 3
+__device__ __forceinline__ uint32_t e2m1_code(float y) {
+  const float a = fabsf(y);
+  const uint32_t c = uint32_t(a > 0.25f) + uint32_t(a >= 0.75f) + uint32_t(a > 1.25f) +
+                     uint32_t(a >= 1.75f) + uint32_t(a > 2.5f) + uint32_t(a >= 3.5f) +
+                     uint32_t(a > 5.0f);
+  return c | ((__float_as_uint(y) >> 28) & 8u);
+}
+
+// one warp per (padded) vocabulary row; rows past V are written as zeros
+__global__ void __launch_bounds__(32 * kRowsPerBlock)
+quantize_w4_kernel(const __nv_bfloat16* __restrict__ x, int V, int D, int rows_pad, int nkb,
+                   uint8_t* __restrict__ w4, float* __restrict__ scale) {
+  pdl_begin();
+  const int lane = threadIdx.x & 31;
+  const int v = blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
+  if (v >= rows_pad) return;
+  const bool real = v < V;
+  const __nv_bfloat16* xr = x + size_t(real ? v : 0) * D;
+  float amax = 0.f;
+  if (real) {
+    for (int k = lane * 8; k < D; k += 256) {
+      const uint4 q = *reinterpret_cast<const uint4*>(xr + k);
+      const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&q);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float2 f = __bfloat1622float2(h[i]);
+        amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
+      }
+    }
+    amax = warp_max(amax);
+    if (lane == 0) scale[v] = amax > 0.f ? __fdiv_rn(amax, 6.f) : 0.f;
+  }
+  const float inv = amax > 0.f ? __fdiv_rn(6.f, amax) : 0.f;
+  const int r = v & (kVocabTile - 1), vt = v / kVocabTile;
+  const int c = lane >> 3;  // the 32-element block (16-byte chunk) of the slice
+  for (int kb = 0; kb < nkb; ++kb) {
+    const int k = kb * 128 + lane * 4;
+    float f[4] = {0.f, 0.f, 0.f, 0.f};
+    if (real && k < D) {
+      const uint2 q = *reinterpret_cast<const uint2*>(xr + k);
+      const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&q.x));
+      const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&q.y));
+      f[0] = a.x; f[1] = a.y; f[2] = b.x; f[3] = b.y;
+    }
+    float bmax = fmaxf(fmaxf(fabsf(f[0]), fabsf(f[1])), fmaxf(fabsf(f[2]), fabsf(f[3])));
+#pragma unroll
+    for (int o = 1; o < 8; o <<= 1) bmax = fmaxf(bmax, __shfl_xor_sync(0xffffffffu, bmax, o));
+    const float t = __fmul_rn(bmax, inv);
+    int e = 0;
+    float thr = 6.f;  // 6 * 2^ee, exact
+#pragma unroll
+    for (int ee = 0; ee >= -5; --ee, thr *= 0.5f)
+      if (t <= thr) e = ee;
+    const float inv_b = __fmul_rn(inv, __int_as_float((127 - e) << 23));  // inv * 2^-e, exact
+    // magnitudes (3 bits) and signs of this lane's 4 elements; a 32-bit word
+    // of the tile holds 8 elements (this lane and its odd/even partner), and
+    // the sign bit of nibble k belongs to element 4 + k / 2 (k even) or k / 2
+    // (k odd) of the word, so that the LM head's widening finds every sign
+    // one shift away from bit 7 of the output byte
+    uint32_t mag = 0, sgn = 0;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const uint32_t cd = e2m1_code(__fmul_rn(f[i], inv_b));
+      mag |= (cd & 7u) << (4 * i);
+      sgn |= (cd >> 3) << i;
+    }
+    const uint32_t psg = __shfl_xor_sync(0xffffffffu, sgn, 1);
+    const bool odd = lane & 1;
+    // even lane (elements 0..3 of the word): nibble signs p0, o0, p1, o1;
+    // odd lane (elements 4..7): o2, p2, o3, p3 (o = own, p = partner)
+    const uint32_t s4 = odd ? ((sgn >> 2) & 1u) | (((psg >> 2) & 1u) << 1) |
+                                  (((sgn >> 3) & 1u) << 2) | (((psg >> 3) & 1u) << 3)
+                            : (psg & 1u) | ((sgn & 1u) << 1) | (((psg >> 1) & 1u) << 2) |
+                                  (((sgn >> 1) & 1u) << 3);
+    uint32_t code = mag;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) code |= ((s4 >> i) & 1u) << (4 * i + 3);
+    uint8_t* tile = w4 + (size_t(vt) * nkb + kb) * kW4TileBytes;
+    // chunk c of row r sits in slot c ^ ((r >> 1) & 3): the converter's
+    // 16-byte reads of 8 consecutive rows then hit 8 different bank groups
+    *reinterpret_cast<uint16_t*>(tile + r * 64 + 16 * (c ^ ((r >> 1) & 3)) + 2 * (lane & 7)) =
+        uint16_t(code);
+    if ((lane & 7) == 0) tile[kW4CodeBytes + r * 4 + c] = uint8_t(int8_t(e));
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_quantize_w4(const void* x, int V, int D, uint8_t* w4, float* scale,
+                               cudaStream_t st) {
+  if (V <= 0) return cudaSuccess;
+  const int rows_pad = (V + kVocabTile - 1) / kVocabTile * kVocabTile;
+  const int nkb = (D + 127) / 128;
+  return launch_pdl(quantize_w4_kernel, dim3(unsigned(rows_pad / kRowsPerBlock)),
+                    dim3(32 * kRowsPerBlock), 0, st, static_cast<const __nv_bfloat16*>(x), V, D,
+                    rows_pad, nkb, w4, scale);
+}
 
 cudaError_t launch_quantize_e4m3(const void* x, int rows, int D, uint8_t* q, float* scale,
                                  cudaStream_t st) {

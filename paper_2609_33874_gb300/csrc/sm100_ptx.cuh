@@ -72,13 +72,43 @@ __device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t budget_ns,
                                           volatile int* abort) {
   if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = global_timer_ns();
-  while (true) {
+  // reading %globaltimer is slow, so the budget and the abort flag are checked
+  // once every 64 polls, not on every one
+  uint64_t t0 = 0;
+  for (uint32_t spin = 1;; ++spin) {
     if (mbar_try_wait(bar, parity)) return true;
-    if (abort && *abort) return false;
-    if (global_timer_ns() - t0 > budget_ns) return false;
+    if ((spin & 63u) == 0) {
+      if (abort && *abort) return false;
+      const uint64_t now = global_timer_ns();
+      if (t0 == 0) t0 = now;
+      else if (now - t0 > budget_ns) return false;
+    }
   }
 }
+
+// Idle tracking of a polling loop that makes progress on several barriers:
+// `idle` counts polls without progress; the clock is read once every 256 of
+// them (reading %globaltimer is slow). True when the loop has made no
+// progress for `budget_ns` or *abort is set.
+struct IdleClock {
+  uint32_t idle = 0;
+  uint64_t t0 = 0;
+  __device__ __forceinline__ bool expired(bool progressed, volatile int* abort,
+                                          uint64_t budget_ns) {
+    if (progressed) {
+      idle = 0;
+      return false;
+    }
+    if ((++idle & 255u) != 0) return false;
+    if (abort && *abort) return true;
+    const uint64_t now = global_timer_ns();
+    if (idle == 256u) {
+      t0 = now;
+      return false;
+    }
+    return now - t0 > budget_ns;
+  }
+};
 
 // mbar_wait by every lane of a warp, with one verdict for the whole warp
 __device__ __forceinline__ bool warp_mbar_wait(uint64_t* bar, uint32_t parity, uint64_t budget_ns,
@@ -112,6 +142,12 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, u
       " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_u32(dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar)), "l"(policy)
       : "memory");
+}
+
+// order this thread's generic-proxy shared-memory writes before later
+// async-proxy (tensor core, TMA) accesses
+__device__ __forceinline__ void fence_proxy_async_shared() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 __device__ __forceinline__ uint64_t policy_evict_first() {

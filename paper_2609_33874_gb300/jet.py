@@ -97,6 +97,10 @@ def _load() -> ctypes.CDLL:
         "jet_workspace_bytes_e4m3": (SZ, [ctypes.POINTER(jet_sizes), ctypes.POINTER(jet_dims)]),
         "jet_score_candidates_e4m3": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
                                           P, P, P, P, P, P, SZ, P]),
+        "jet_w4_bytes": (SZ, [ctypes.c_int64, ctypes.c_int64]),
+        "jet_quantize_w4": (I, [P, ctypes.c_int64, ctypes.c_int64, P, P, P]),
+        "jet_score_candidates_w4": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
+                                        P, P, P, P, P, P, SZ, P]),
         "jet_decide": (I, [ctypes.POINTER(jet_layout), I, P, P, P, P, P]),
         "jet_evaluate": (I, [ctypes.POINTER(jet_layout), P, P, P, P, P, P]),
         "jet_device_status": (I, [P, ctypes.POINTER(ctypes.c_int32)]),
@@ -114,7 +118,7 @@ DECLARED = ("jet_abi_version", "jet_status_string", "jet_layout_plan", "jet_layo
             "jet_prefill_workspace_bytes", "jet_prefill_attend", "jet_prefill_state",
             "jet_fork_state", "jet_fork_state_rule", "jet_score_candidates", "jet_score_candidates_noalloc",
             "jet_quantize_rows_e4m3", "jet_workspace_bytes_e4m3", "jet_score_candidates_e4m3",
-            "jet_decide", "jet_evaluate", "jet_device_status")
+            "jet_w4_bytes", "jet_quantize_w4", "jet_score_candidates_w4", "jet_decide", "jet_evaluate", "jet_device_status")
 
 
 def library() -> ctypes.CDLL:
@@ -316,6 +320,29 @@ def jet_score_candidates_e4m3(layout, dims: jet_dims, hidden, w_q, w_scale, tok_
                                           _addr(tok_logprob), _addr(cand_score), _addr(ws),
                                           int(ws_bytes), _stream(stream)),
            "jet_score_candidates_e4m3")
+
+
+def jet_w4_bytes(V: int, D: int) -> int:
+    """Bytes of the tiled 4-bit codes of a [V, D] matrix (0 if invalid)."""
+    return int(_lib.jet_w4_bytes(int(V), int(D)))
+
+
+def jet_quantize_w4(w, w4, scale, stream=None) -> None:
+    """Tiled 4-bit codes w4 (jet_w4_bytes(V, D) bytes) and row scales [V]
+    float32 of the bf16 matrix w [V, D] (see include/jet.h)."""
+    V, D = (int(w.shape[0]), int(w.shape[1])) if w.dim() == 2 else (0, 0)
+    _check(_lib.jet_quantize_w4(_addr(w), V, D, _addr(w4), _addr(scale), _stream(stream)),
+           "jet_quantize_w4")
+
+
+def jet_score_candidates_w4(layout, dims: jet_dims, hidden, w4, w_scale, tok_logprob,
+                            cand_score, ws, ws_bytes: Optional[int] = None, stream=None) -> None:
+    ws_bytes = ws.numel() * ws.element_size() if ws_bytes is None else ws_bytes
+    _check(_lib.jet_score_candidates_w4(ctypes.byref(_lay(layout)), ctypes.byref(dims),
+                                        _addr(hidden), _addr(w4), _addr(w_scale),
+                                        _addr(tok_logprob), _addr(cand_score), _addr(ws),
+                                        int(ws_bytes), _stream(stream)),
+           "jet_score_candidates_w4")
 
 
 def jet_decide(layout, mode: int, cand_score, q, choice, value, stream=None) -> None:

@@ -37,6 +37,17 @@ def quantize_lm_head(w_lm: torch.Tensor, stream=None):
     return w_q, w_scale
 
 
+def quantize_lm_head_w4(w_lm: torch.Tensor, stream=None):
+    """Tiled 4-bit codes (uint8, jet_w4_bytes(V, D) bytes) and per-row float32
+    scales [V] of the bf16 LM-head weights (jet_quantize_w4), for a step built
+    with lm="w4"."""
+    V, D = w_lm.shape
+    w4 = torch.empty(jet.jet_w4_bytes(V, D), dtype=torch.uint8, device=w_lm.device)
+    w_scale = torch.empty(V, dtype=torch.float32, device=w_lm.device)
+    jet.jet_quantize_w4(w_lm, w4, w_scale, stream=stream)
+    return w4, w_scale
+
+
 class ScoringStep:
     """Device state of one batch shape.
 
@@ -45,7 +56,8 @@ class ScoringStep:
     fork; ``keep_fork_state`` also writes every candidate's final recurrent
     state. ``chain`` feeds the attention output to the LM head (requires
     Hq * d == D). ``lm`` selects the LM head: "bf16" (w_lm is the bf16 weight
-    matrix) or "e4m3" (w_lm is the pair returned by :func:`quantize_lm_head`).
+    matrix), "e4m3" (w_lm is the pair returned by :func:`quantize_lm_head`) or
+    "w4" (the pair returned by :func:`quantize_lm_head_w4`).
     ``rule`` selects the fork's recurrence: "delta" (gated delta rule) or "gla"
     (plain gated linear attention).
     """
@@ -53,8 +65,8 @@ class ScoringStep:
     def __init__(self, layout: "jet.HostLayout", dims: "jet.jet_dims", mode: int,
                  device="cuda", hybrid: bool = False, keep_fork_state: bool = False,
                  chain: bool = False, lm: str = "bf16", rule: str = "delta"):
-        if lm not in ("bf16", "e4m3"):
-            raise ValueError("lm must be 'bf16' or 'e4m3'")
+        if lm not in ("bf16", "e4m3", "w4"):
+            raise ValueError("lm must be 'bf16', 'e4m3' or 'w4'")
         self.lm = lm
         self.rule = jet.RULES[rule]
         self.dev = torch.device(device)
@@ -74,7 +86,7 @@ class ScoringStep:
         self.q_cand = z(n.C)
         self.choice = z(n.R, dtype=torch.int32)
         self.value = z(n.R)
-        ws = (jet.jet_workspace_bytes_e4m3 if lm == "e4m3" else jet.jet_workspace_bytes)(n, dims)
+        ws = (jet.jet_workspace_bytes if lm == "bf16" else jet.jet_workspace_bytes_e4m3)(n, dims)
         self.ws = z((ws + 15) // 16 * 4)  # float32 words, 16-byte multiple
         if hybrid:
             self.lo = z(self.F, dims.Hl, dims.dv, dtype=dt)
@@ -104,9 +116,13 @@ class ScoringStep:
                        stream=stream)
 
     def score(self, hidden: torch.Tensor, w_lm, stream=None, layout=None) -> None:
-        """The LM-head call of the step (bf16 or e4m3, as the step was built)."""
+        """The LM-head call of the step (bf16, e4m3 or w4, as the step was built)."""
         lay = self.layout if layout is None else layout
-        if self.lm == "e4m3":
+        if self.lm == "w4":
+            w4, w_scale = w_lm
+            jet.jet_score_candidates_w4(lay, self.dims, hidden, w4, w_scale, self.tok_logprob,
+                                        self.cand_score, self.ws, stream=stream)
+        elif self.lm == "e4m3":
             w_q, w_scale = w_lm
             jet.jet_score_candidates_e4m3(lay, self.dims, hidden, w_q, w_scale, self.tok_logprob,
                                           self.cand_score, self.ws, stream=stream)

@@ -214,6 +214,29 @@ def test_prefill_state_validation(jet):
     assert lib.jet_prefill_state(L, D, jet.RECUR_DELTA, *mis) == 4
 
 
+def test_w4_validation(jet):
+    lay, dims = _setup(jet)
+    lib = jet.library()
+    assert jet.jet_w4_bytes(300, 208) == 3 * 2 * 8704
+    assert jet.jet_w4_bytes(128, 128) == 8704
+    assert jet.jet_w4_bytes(0, 128) == 0 and jet.jet_w4_bytes(10, 24) == 0
+    # quantiser: rows, shape, null and alignment
+    assert lib.jet_quantize_w4(FAKE, 0, 64, FAKE, FAKE, None) == 1
+    assert lib.jet_quantize_w4(FAKE, 4, 24, FAKE, FAKE, None) == 2     # D % 16 != 0
+    assert lib.jet_quantize_w4(None, 4, 64, FAKE, FAKE, None) == 1
+    assert lib.jet_quantize_w4(FAKE, 4, 64, MIS, FAKE, None) == 4
+    # scoring: float32 dims have no 4-bit path; workspace and alignment checks
+    L = ctypes.byref(lay.struct)
+    f32 = jet.make_dims(jet.DTYPE_F32, D=64)
+    args = [FAKE] * 6
+    assert lib.jet_score_candidates_w4(L, ctypes.byref(f32), *args, 1 << 30, None) == 7
+    bf = jet.make_dims(jet.DTYPE_BF16, D=64)
+    assert lib.jet_score_candidates_w4(L, ctypes.byref(bf), *args, 16, None) == 5
+    mis = list(args)
+    mis[1] = MIS   # w4
+    assert lib.jet_score_candidates_w4(L, ctypes.byref(bf), *mis, 1 << 30, None) == 4
+
+
 def test_e4m3_validation(jet):
     lay, dims = _setup(jet)
     lib = jet.library()
