@@ -29,7 +29,8 @@ import numpy as np
 
 __all__ = [
     "Workload", "WORKLOADS", "Problem", "make_problem", "bf16_round",
-    "bf16_to_f32", "f32_to_bf16_bits",
+    "bf16_to_f32", "f32_to_bf16_bits", "StackSpec", "STACKS", "stack_shapes", "stack_tensor",
+    "stack_x0",
 ]
 
 _CHUNK = 1 << 22  # elements per independently seeded chunk
@@ -285,6 +286,79 @@ def _draw_lengths(spec: tuple, n: int, g: np.random.Generator) -> np.ndarray:
     raise ValueError(kind)
 
 
+# --------------------------------------------------------------------------
+# hybrid decoder stacks (several layers over the step's query rows)
+# --------------------------------------------------------------------------
+@dataclasses.dataclass(frozen=True)
+class StackSpec:
+    """A stack of decoder layers: ``kinds`` lists "linear" (linear attention,
+    forked per candidate) or "full" (attention over the cached prefix) per
+    layer; ``Dff`` is the MLP width (a multiple of 64)."""
+    kinds: tuple
+    Dff: int
+
+
+STACKS: Dict[str, StackSpec] = {
+    # three linear-attention layers per full-attention layer, as in the
+    # paper's hybrid Qwen models; MLP width 3 x D
+    "hybrid4": StackSpec(("linear", "linear", "linear", "full"), 3 * 4096),
+}
+
+_STACK_NAMES = ("g1", "g2", "w_mix", "w_o", "w_gu", "w_d", "k_pre", "v_pre", "s_prefix")
+
+
+def stack_shapes(work: Workload, spec: StackSpec, kind: str, total_prefix: int, R: int):
+    """Shapes of one layer's tensors. w_mix is [(Hq + 2 Hkv) d, D] for a
+    full layer (q, k, v heads in that order) and [Hl (2 dk + dv) + 2 Hl, D] for
+    a linear layer (q, k, v, then the alpha and beta logits); w_gu holds the
+    MLP gate and up rows interleaved in blocks of 64 (rows 128 t .. + 63 gate
+    features 64 t .., rows 128 t + 64 .. up features 64 t ..)."""
+    w = work
+    out = dict(g1=(w.D,), g2=(w.D,), w_gu=(2 * spec.Dff, w.D), w_d=(w.D, spec.Dff))
+    if kind == "full":
+        out.update(w_mix=((w.Hq + 2 * w.Hkv) * w.d, w.D), w_o=(w.D, w.Hq * w.d),
+                   k_pre=(total_prefix, w.Hkv, w.d), v_pre=(total_prefix, w.Hkv, w.d))
+    else:
+        out.update(w_mix=(w.Hl * (2 * w.dk + w.dv) + 2 * w.Hl, w.D), w_o=(w.D, w.Hl * w.dv),
+                   s_prefix=(R, w.Hl, w.dk, w.dv))
+    return out
+
+
+def stack_tensor(problem: "Problem", spec: StackSpec, layer: int, name: str) -> np.ndarray:
+    """One tensor of layer ``layer`` in device format (bf16 bits; the recurrent
+    state float32). Norm gains are 1 + N(0, 0.1^2); weights N(0, 1/fan_in);
+    prefix keys/values N(0, 1); the prefix state N(0, 1/dk)."""
+    w = problem.work
+    kind = spec.kinds[layer]
+    shape = stack_shapes(w, spec, kind, problem.total_prefix, problem.R)[name]
+    key = ("stack", spec, layer, name)
+    if key in problem._cache:
+        return problem._cache[key]
+    tag = 100 + 16 * layer + _STACK_NAMES.index(name)
+    n = int(np.prod(shape))
+    if name in ("g1", "g2"):
+        x = 1.0 + _normal_chunks(problem.seed, tag, n, 0.1, False)
+        val = f32_to_bf16_bits(x.astype(np.float32))
+    elif name == "s_prefix":
+        val = _normal_chunks(problem.seed, tag, n, 1.0 / np.sqrt(w.dk), False)
+    elif name in ("k_pre", "v_pre"):
+        val = _normal_chunks(problem.seed, tag, n, 1.0, True)
+    else:
+        val = _normal_chunks(problem.seed, tag, n, 1.0 / np.sqrt(shape[1]), True)
+    val = val.reshape(shape)
+    problem._cache[key] = val
+    return val
+
+
+def stack_x0(problem: "Problem") -> np.ndarray:
+    """The embeddings of the step's N query rows, [N, D] bf16 bits, N(0, 1)."""
+    key = ("stack_x0", problem.N, problem.work.D)
+    if key not in problem._cache:
+        problem._cache[key] = _normal_chunks(problem.seed, 99, problem.N * problem.work.D, 1.0,
+                                             True).reshape(problem.N, problem.work.D)
+    return problem._cache[key]
+
+
 def make_problem(work, R: Optional[int] = None, seed: Optional[int] = None) -> Problem:
     """Draw the structure of a batch.
 
@@ -333,3 +407,13 @@ def torch_tensor(problem: Problem, name: str, device=None, pin: bool = False):
     if device is not None:
         t = t.to(device)
     return t
+
+
+def array_to_torch(a: np.ndarray, device=None):
+    """A device-format array (bf16 bits or float32) as a torch tensor."""
+    import torch
+    if a.dtype == np.uint16:
+        t = torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16)
+    else:
+        t = torch.from_numpy(np.ascontiguousarray(a))
+    return t if device is None else t.to(device)
