@@ -602,6 +602,75 @@ def run_prefill(args):
         gpu_launches=sum(x["launches"] for x in parts.values()) * args.steps)), flush=True)
 
 
+def run_stack(args):
+    """Times a hybrid decoder stack over the workload's rows followed by the
+    LM head and the decision (inputs resident in HBM) and prints one JSON
+    line: candidate sets per second through the whole forward, with the
+    stack's projections against their roofline."""
+    import torch
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    from paper_2609_33874_gb300 import build as _build
+    _build.build()
+    import jet_synth
+    from paper_2609_33874_gb300 import jet
+    from paper_2609_33874_gb300.step import DecoderStack, ScoringStep
+    w = jet_synth.WORKLOADS[args.workload]
+    spec = jet_synth.STACKS[args.stack]
+    R = args.R or w.R
+    p = jet_synth.make_problem(w, R=R)
+    hl = jet.jet_layout_build(p.prefix_len, p.n_cand, p.cand_len, p.target_ids, w.V)
+    dims = jet.make_dims(jet.DTYPE_BF16, Hq=w.Hq, Hkv=w.Hkv, d=w.d, D=w.D, Hl=w.Hl, dk=w.dk,
+                         dv=w.dv)
+    layers = []
+    for l, kind in enumerate(spec.kinds):
+        names = ["g1", "g2", "w_mix", "w_o", "w_gu", "w_d"] + (
+            ["k_pre", "v_pre"] if kind == "full" else ["s_prefix"])
+        L = {n: jet_synth.array_to_torch(jet_synth.stack_tensor(p, spec, l, n), dev)
+             for n in names}
+        L["kind"] = kind
+        layers.append(L)
+    stack = DecoderStack(hl, dims, layers, spec.Dff, rule=args.rule, device=dev)
+    step = ScoringStep(hl, dims, jet.MODES[w.mode], device=dev)
+    x0 = jet_synth.array_to_torch(jet_synth.stack_x0(p), dev)
+    w_lm = jet_synth.torch_tensor(p, "w_lm", device=dev)
+    p.drop()
+    stream = torch.cuda.Stream(dev)
+
+    def one():
+        x = stack.forward(x0, stream=stream)
+        step.score(x, w_lm, stream=stream)
+        jet.jet_decide(step.layout, step.mode, step.cand_score, step.q_cand, step.choice,
+                       step.value, stream=stream)
+
+    ms = _time_stream(one, stream, args.warmup, args.steps)
+    ms_stack = _time_stream(lambda: stack.forward(x0, stream=stream), stream, 2, args.steps)
+    assert jet.jet_device_status(stream) == 0
+    N = p.N
+    # the stack's projections: weight bytes once per call, 2 N K O flops each
+    wts = 0
+    for l, kind in enumerate(spec.kinds):
+        sh = jet_synth.stack_shapes(w, spec, kind, p.total_prefix, R)
+        wts += sum(int(np.prod(sh[n])) for n in ("w_mix", "w_o", "w_gu", "w_d"))
+    flops = 2.0 * N * wts
+    nbytes = wts * 2 + len(spec.kinds) * N * w.D * 2 * 8  # weights + the rows' passes
+    peaks = _peaks()
+    roof = _roof(flops, nbytes, ms_stack, peaks)
+    roof.update(kernel="jet_stack_forward (proj_tc_kernel projections, rmsnorm, attention, fork)",
+                algorithmic_flops=flops, algorithmic_bytes=nbytes, traffic=None,
+                peak_source=peaks["source"])
+    print(json.dumps(dict(
+        metric="candidate sets scored/sec (decoder stack + LM head)",
+        value=round(R / (ms / 1e3), 1), unit="sets/s", n_gpus=1, steps=args.steps,
+        warmup=args.warmup, ms_per_step=round(ms, 4), higher_is_better=True, dtype="bf16",
+        data="synthetic",
+        config=dict(workload=args.workload, stack=args.stack, kinds=list(spec.kinds),
+                    Dff=spec.Dff, R=R, N=N, D=w.D, rule=args.rule),
+        roofline=roof, parts=dict(stack_ms=round(ms_stack, 4),
+                                  score_and_decide_ms=round(ms - ms_stack, 4)),
+        gpu_launches=None)), flush=True)
+
+
 # ---------------------------------------------------------------------------
 # reference arm: the fp64 oracle on the host cores
 # ---------------------------------------------------------------------------
@@ -653,6 +722,9 @@ def main():
                     help="LM head precision: bf16 (the workload's), e4m3 codes with one "
                          "scale per weight row and per token (the paper's 8-bit weights), or "
                          "w4: 4-bit weights in 32-element blocks (the paper's 4-bit weights)")
+    ap.add_argument("--stack", default=None,
+                    help="time a hybrid decoder stack (e.g. hybrid4) over the workload's rows, "
+                         "then the LM head and the decision (one GPU)")
     ap.add_argument("--prefill", action="store_true",
                     help="time the prefill (causal attention over the workload's prefixes) "
                          "instead of the scoring step (one GPU)")
@@ -663,6 +735,8 @@ def main():
     args.warmup = max(3, args.warmup)  # at least three untimed warm-up steps
     if args.impl == "reference":
         run_reference(args)
+    elif args.stack:
+        run_stack(args)
     elif args.prefill:
         run_prefill(args)
     elif args.sweep:

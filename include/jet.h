@@ -410,6 +410,72 @@ jet_status jet_score_candidates_w4(const jet_layout* lay, const jet_dims* dims,
                                    size_t ws_bytes, void* stream);
 
 /*
+ * Hybrid decoder stacks (Sec. 4.1: hybrid models keep a recurrent state per
+ * linear-attention layer, restored for every candidate, and reuse the prefix
+ * cache at attention layers). jet_stack_forward runs L pre-norm decoder
+ * layers over the step's N rows - each request's shared row and its
+ * candidates' fed tokens - with a fork of the recurrent state at every
+ * linear-attention layer:
+ *   h  = RMSNorm(x) * g1                          (eps 1e-6)
+ *   full layer:   q, k, v = h w_mix^T; the step's cascade attention over the
+ *                 layer's prefix keys/values plus each candidate's own fed
+ *                 tokens (jet_prefix_attend); the shared row's own key/value
+ *                 is the prefix's last position
+ *   linear layer: q, k, v, a, b = h w_mix^T; k normalised per head;
+ *                 alpha = sigmoid(a), beta = sigmoid(b); the fed tokens run
+ *                 the recurrence from the layer's prefix state
+ *                 (jet_fork_state_rule, stack.rule); a shared row reads the
+ *                 prefix state: o = S_prefix^T q / sqrt(dk)
+ *   x  = x + o w_o^T
+ *   x  = x + (SiLU(RMSNorm(x) * g2 w_gate^T) * (... w_up^T)) w_down^T
+ * Activations are bf16 between operations (f32 inside each); the
+ * projections run on the tensor cores.
+ */
+enum { JET_LAYER_LINEAR = 0, JET_LAYER_FULL = 1 };
+
+typedef struct jet_stack_layer {
+  int32_t kind;        /* JET_LAYER_LINEAR or JET_LAYER_FULL                     */
+  int32_t reserved;
+  const void* g1;      /* [D] bf16 RMSNorm gains before the mixer                */
+  const void* g2;      /* [D] bf16 RMSNorm gains before the MLP                  */
+  const void* w_mix;   /* bf16; full: [(Hq + 2 Hkv) d, D], rows q heads, k heads,
+                          v heads; linear: [Hl (2 dk + dv) + 2 Hl, D], rows q, k,
+                          v heads, then the Hl decay and Hl write-strength logits */
+  const void* w_o;     /* bf16 [D, Hq d] (full) or [D, Hl dv] (linear)           */
+  const void* w_gu;    /* bf16 [2 Dff, D]: rows 128 t .. + 63 are the gate rows of
+                          features 64 t .. + 63, rows 128 t + 64 .. + 127 their
+                          up rows                                                */
+  const void* w_d;     /* bf16 [D, Dff]                                           */
+  const void* k_pre;   /* full: bf16 [sum P, Hkv, d] prefix keys; linear: NULL    */
+  const void* v_pre;   /* full: bf16 [sum P, Hkv, d] prefix values               */
+  const float* s_prefix; /* linear: [R, Hl, dk, dv] prefix states; full: NULL   */
+} jet_stack_layer;
+
+typedef struct jet_stack {
+  int32_t L;           /* layers                                                  */
+  int32_t Dff;         /* MLP width, a positive multiple of 64                    */
+  int32_t rule;        /* JET_RECUR_* of the linear layers                        */
+  int32_t reserved;
+  const jet_stack_layer* layers; /* host array of L layers, read during the call */
+} jet_stack;
+
+/* Workspace bytes of jet_stack_forward for these sizes, dims and MLP width;
+ * 0 on invalid arguments. */
+size_t jet_stack_workspace_bytes(const jet_sizes* n, const jet_dims* dims, int32_t Dff);
+
+/*
+ * jet_stack_forward - x = the stack applied to x0 (both [N, D] bf16, device;
+ * x may equal x0). dims: dtype JET_DTYPE_BF16, D a multiple of 16; with a
+ * full layer Hq, Hkv, d as for jet_prefix_attend; with a linear layer Hl even,
+ * dk = 128, dv a multiple of 32. The result is the hidden state that
+ * jet_score_candidates takes. Errors: as for the calls it makes, plus
+ * JET_ERR_ARG (a null layer pointer, an unknown kind or rule, L < 0),
+ * JET_ERR_SHAPE (Dff), JET_ERR_WORKSPACE.
+ */
+jet_status jet_stack_forward(const jet_layout* lay, const jet_dims* dims, const jet_stack* stack,
+                             const void* x0, void* x, void* ws, size_t ws_bytes, void* stream);
+
+/*
  * jet_score_candidates_noalloc - jet_score_candidates without caller-owned
  * scratch memory. The paper has no counterpart to this entry point: it exists
  * for callers that cannot call cudaMalloc, such as a host application that

@@ -2,10 +2,12 @@
 // stream-ordered launches. No entry point allocates memory, synchronises a
 // stream (except jet_device_status) or launches anything after a failed
 // check.
+#include <algorithm>
 #include <cstdint>
 #include <mutex>
 
 #include "jet.h"
+
 #include "jet_internal.h"
 
 namespace jet {
@@ -387,6 +389,169 @@ extern "C" jet_status jet_score_candidates_w4(const jet_layout* lay, const jet_d
                                             ws, status, st)));
   return cuda_status(
       jet::launch_score_finish(*lay, plan.score, ws, tok_logprob, cand_score, status, st));
+}
+
+namespace {
+
+// scratch of jet_stack_forward (offsets 256-byte aligned)
+struct StackPlan {
+  size_t h, z, q, kc, vc, lqa, lqf, lk, lv, al, be, lo, o, u, attn, part, bytes;
+  jet::AttnPlan attn_plan;
+  bool full_ok, lin_ok;
+};
+
+StackPlan stack_plan(const jet_sizes& n, const jet_dims& d, int Dff) {
+  auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
+  StackPlan p{};
+  const size_t N = size_t(n.N), F = size_t(n.N - n.R), b = 2;
+  p.full_ok = check_attn_dims(&d) == JET_OK;
+  p.lin_ok = check_fork_dims(&d) == JET_OK && d.Hl % 2 == 0;
+  const size_t zf = p.full_ok ? size_t(d.Hq + 2 * d.Hkv) * d.d : 0;
+  const size_t zl = p.lin_ok ? size_t(d.Hl) * (2 * d.dk + d.dv) + 2 * d.Hl : 0;
+  const size_t ow = std::max(p.full_ok ? size_t(d.Hq) * d.d : 0,
+                             p.lin_ok ? size_t(d.Hl) * d.dv : 0);
+  size_t at = 0;
+  auto take = [&](size_t bytes) {
+    const size_t off = at;
+    at += up(bytes);
+    return off;
+  };
+  p.h = take(N * d.D * b);
+  p.z = take(N * std::max(zf, zl) * b);
+  p.o = take(N * ow * b);
+  p.u = take(N * size_t(Dff) * b);
+  // split-K partials of the largest projection that splits
+  size_t part = jet::proj_partial_bytes(n.N, 2 * Dff, d.D);
+  part = std::max(part, jet::proj_partial_bytes(n.N, d.D, Dff));
+  if (zf) {
+    part = std::max(part, jet::proj_partial_bytes(n.N, int(zf), d.D));
+    part = std::max(part, jet::proj_partial_bytes(n.N, d.D, d.Hq * d.d));
+  }
+  if (zl) {
+    part = std::max(part, jet::proj_partial_bytes(n.N, int(zl), d.D));
+    part = std::max(part, jet::proj_partial_bytes(n.N, d.D, d.Hl * d.dv));
+  }
+  p.part = take(part);
+  if (p.full_ok) {
+    p.q = take(N * d.Hq * d.d * b);
+    p.kc = take(F * d.Hkv * d.d * b);
+    p.vc = take(F * d.Hkv * d.d * b);
+    p.attn_plan = jet::attn_plan(n, d);
+    p.attn = take(p.attn_plan.bytes);
+  }
+  if (p.lin_ok) {
+    p.lqa = take(N * d.Hl * d.dk * b);
+    p.lqf = take(F * d.Hl * d.dk * b);
+    p.lk = take(F * d.Hl * d.dk * b);
+    p.lv = take(F * d.Hl * d.dv * b);
+    p.al = take(F * d.Hl * 4);
+    p.be = take(F * d.Hl * 4);
+    p.lo = take(F * d.Hl * d.dv * b);
+  }
+  p.bytes = at;
+  return p;
+}
+
+}  // namespace
+
+extern "C" size_t jet_stack_workspace_bytes(const jet_sizes* n, const jet_dims* d, int32_t Dff) {
+  if (!n || !d || n->R < 0 || n->N < n->R || d->D < 16 || Dff < 64 || Dff % 64 != 0) return 0;
+  return stack_plan(*n, *d, Dff).bytes;
+}
+
+extern "C" jet_status jet_stack_forward(const jet_layout* lay, const jet_dims* dims,
+                                        const jet_stack* stack, const void* x0, void* x,
+                                        void* ws, size_t ws_bytes, void* stream) {
+  JET_TRY(check_layout(lay));
+  if (!dims || !stack) return JET_ERR_ARG;
+  JET_TRY(check_dtype(dims));
+  if (dims->dtype != JET_DTYPE_BF16) return JET_ERR_UNSUPPORTED;
+  if (dims->D < 16 || dims->D % 16 != 0) return JET_ERR_SHAPE;
+  if (stack->L < 0 || (stack->L > 0 && !stack->layers)) return JET_ERR_ARG;
+  if (stack->Dff < 64 || stack->Dff % 64 != 0) return JET_ERR_SHAPE;
+  if (stack->rule != JET_RECUR_DELTA && stack->rule != JET_RECUR_GLA) return JET_ERR_ARG;
+  const jet_sizes& n = lay->n;
+  const long long N = n.N, F = n.N - n.R;
+  const StackPlan plan = stack_plan(n, *dims, stack->Dff);
+  // validate every layer before the first launch
+  for (int l = 0; l < stack->L; ++l) {
+    const jet_stack_layer& Ly = stack->layers[l];
+    if (Ly.kind == JET_LAYER_FULL) {
+      JET_TRY(check_attn_dims(dims));
+      if ((long long)n.R * dims->Hkv > 65535) return JET_ERR_CAPACITY;
+      JET_TRY(check_ptr(Ly.k_pre, n.total_prefix));
+      JET_TRY(check_ptr(Ly.v_pre, n.total_prefix));
+    } else if (Ly.kind == JET_LAYER_LINEAR) {
+      JET_TRY(check_fork_dims(dims));
+      if (dims->Hl % 2 != 0) return JET_ERR_UNSUPPORTED;
+      if (n.R > 65535 || dims->Hl > 65535 || dims->dv > 1024) return JET_ERR_CAPACITY;
+      JET_TRY(check_ptr(Ly.s_prefix, n.R));
+    } else {
+      return JET_ERR_ARG;
+    }
+    JET_TRY(check_ptr(Ly.g1, 1));
+    JET_TRY(check_ptr(Ly.g2, 1));
+    JET_TRY(check_ptr(Ly.w_mix, 1));
+    JET_TRY(check_ptr(Ly.w_o, 1));
+    JET_TRY(check_ptr(Ly.w_gu, 1));
+    JET_TRY(check_ptr(Ly.w_d, 1));
+  }
+  if (n.R == 0) return JET_OK;
+  JET_TRY(check_ptr(x0, N));
+  JET_TRY(check_ptr(x, N));
+  if (!ws || ws_bytes < plan.bytes) return JET_ERR_WORKSPACE;
+  if (!aligned16(ws)) return JET_ERR_ALIGN;
+  if (N > 65535 * 8 || (long long)N * dims->D > INT32_MAX) return JET_ERR_CAPACITY;
+  int* status = jet::device_status_ptr();
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  float* part = reinterpret_cast<float*>(w + plan.part);
+  const int D = dims->D, Dff = stack->Dff;
+  const size_t xbytes = size_t(N) * D * 2;
+  if (x != x0)
+    JET_TRY(cuda_status(cudaMemcpyAsync(x, x0, xbytes, cudaMemcpyDeviceToDevice, st)));
+  for (int l = 0; l < stack->L; ++l) {
+    const jet_stack_layer& Ly = stack->layers[l];
+    const bool full = Ly.kind == JET_LAYER_FULL;
+    JET_TRY(cuda_status(jet::launch_rmsnorm(x, Ly.g1, int(N), D, 1e-6f, w + plan.h, st)));
+    const int zw = full ? (dims->Hq + 2 * dims->Hkv) * dims->d
+                        : dims->Hl * (2 * dims->dk + dims->dv) + 2 * dims->Hl;
+    JET_TRY(cuda_status(jet::launch_proj(jet::kProjStore, w + plan.h, int(N), D, D, Ly.w_mix, zw,
+                                         w + plan.z, zw, nullptr, part, status, st)));
+    int ow;
+    if (full) {
+      const int qw = dims->Hq * dims->d, kw = dims->Hkv * dims->d;
+      JET_TRY(cuda_status(jet::launch_split_qkv(*lay, w + plan.z, qw, kw, w + plan.q, w + plan.kc,
+                                                w + plan.vc, status, st)));
+      JET_TRY(cuda_status(jet::launch_prefix_attend(*lay, *dims, plan.attn_plan, w + plan.q,
+                                                    Ly.k_pre, Ly.v_pre, w + plan.kc,
+                                                    w + plan.vc, w + plan.o, w + plan.attn,
+                                                    status, st)));
+      ow = qw;
+    } else {
+      float* al = reinterpret_cast<float*>(w + plan.al);
+      float* be = reinterpret_cast<float*>(w + plan.be);
+      JET_TRY(cuda_status(jet::launch_gates(*lay, w + plan.z, dims->Hl, dims->dv, w + plan.lqa,
+                                            w + plan.lqf, w + plan.lk, w + plan.lv, al, be,
+                                            status, st)));
+      if (F > 0)
+        JET_TRY(cuda_status(jet::launch_fork_state(*lay, *dims, stack->rule, Ly.s_prefix,
+                                                   w + plan.lqf, w + plan.lk, w + plan.lv, al, be,
+                                                   w + plan.lo, nullptr, status, st)));
+      JET_TRY(cuda_status(jet::launch_readout(*lay, Ly.s_prefix, w + plan.lqa, w + plan.lo,
+                                              dims->Hl, dims->dv, w + plan.o, status, st)));
+      ow = dims->Hl * dims->dv;
+    }
+    JET_TRY(cuda_status(jet::launch_proj(jet::kProjResid, w + plan.o, int(N), ow, ow, Ly.w_o, D,
+                                         x, D, x, part, status, st)));
+    JET_TRY(cuda_status(jet::launch_rmsnorm(x, Ly.g2, int(N), D, 1e-6f, w + plan.h, st)));
+    JET_TRY(cuda_status(jet::launch_proj(jet::kProjSwiGLU, w + plan.h, int(N), D, D, Ly.w_gu,
+                                         2 * Dff, w + plan.u, Dff, nullptr, part, status,
+                                         st)));
+    JET_TRY(cuda_status(jet::launch_proj(jet::kProjResid, w + plan.u, int(N), Dff, Dff, Ly.w_d,
+                                         D, x, D, x, part, status, st)));
+  }
+  return JET_OK;
 }
 
 extern "C" jet_status jet_decide(const jet_layout* lay, int32_t mode, const float* cand_score,

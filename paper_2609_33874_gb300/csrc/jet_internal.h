@@ -102,6 +102,26 @@ cudaError_t launch_lmhead_tc(const jet_layout& lay, const jet_dims& d, const Sco
 cudaError_t launch_lmhead_e4m3(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
                                const uint8_t* h_q, const float* h_scale, const uint8_t* w_q,
                                const float* w_scale, void* ws, int* status, cudaStream_t st);
+// ---- decoder stacks -------------------------------------------------------------
+enum { kProjStore = 0, kProjResid = 1, kProjSwiGLU = 2 };
+// out[N, O] = epilogue(x[N, K] w[O, K]^T) on the tensor cores (bf16, f32 accumulate);
+// ldx / ldo are the row strides of x and out in elements; res (kProjResid) may be
+// out; part: f32 scratch of proj_partial_bytes(N, O, K) bytes for a split K (null:
+// no split)
+cudaError_t launch_proj(int epi, const void* x, int N, int K, int ldx, const void* w, int O,
+                        void* out, int ldo, const void* res, float* part, int* status,
+                        cudaStream_t st);
+size_t proj_partial_bytes(int N, int O, int K);
+cudaError_t launch_rmsnorm(const void* x, const void* g, int N, int D, float eps, void* h,
+                           cudaStream_t st);
+cudaError_t launch_split_qkv(const jet_layout& lay, const void* z, int qw, int kw, void* q,
+                             void* kc, void* vc, int* status, cudaStream_t st);
+cudaError_t launch_gates(const jet_layout& lay, const void* z, int Hl, int dv, void* lq_all,
+                         void* lq, void* lk, void* lv, float* alpha, float* beta, int* status,
+                         cudaStream_t st);
+cudaError_t launch_readout(const jet_layout& lay, const float* s_prefix, const void* lq_all,
+                           const void* lo, int Hl, int dv, void* o, int* status, cudaStream_t st);
+
 // the LM head on tiled 4-bit weights (w4) and e4m3 hidden codes
 cudaError_t launch_lmhead_w4(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
                              const uint8_t* h_q, const float* h_scale, const uint8_t* w4,

@@ -1,0 +1,424 @@
+// Projections of a decoder stack on the 5th-generation tensor cores:
+// out[N, O] = epilogue(X[N, K] W[O, K]^T) with bf16 X and W and f32
+// accumulation, for the mixer, output and MLP projections of every layer.
+//
+// The mainloop is the LM head's: weight rows on the MMA's M side (128 rows per
+// tile = the 128 TMEM lanes), the step's rows on N (a token tile of up to 256),
+// one persistent CTA per SM working through (weight tile, token tile) units.
+//   warp 0      TMA producer: 128 x 64 weight tile + Nt x 64 row tile per
+//               stage, both 128-byte swizzled, into a ring of stages
+//   warp 1      TMEM allocator and MMA issuer: 4 x tcgen05.mma kind::f16 (K =
+//               16) per stage into one of two TMEM accumulators
+//   warps 2..5  epilogue: each warp reads its 32 TMEM lanes (32 output
+//               features) x 32 rows at a time and writes bf16 outputs
+// Epilogues: kStore (out = acc), kResid (out = res + acc, one rounding; res
+// may be out itself: every element is read and written by one thread) and
+// kSwiGLU: the weight rows come interleaved in blocks of 64 (tile rows 0..63
+// gate features 64 t .., rows 64..127 the matching up features), the warps
+// holding the up half pass their values through shared memory, and
+// out[n, 64 t + f] = SiLU(gate) * up.
+// Split K: when the (weight tile, token tile) units are too few to occupy the
+// SMs (few output features, long K), each unit covers a range of K and writes
+// its f32 partial; a reduce kernel sums the partials and applies the epilogue.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <mutex>
+
+#include "jet_device.cuh"
+#include "jet_internal.h"
+#include "sm100_ptx.cuh"
+
+namespace jet {
+namespace {
+
+using namespace sm100;
+
+constexpr int kBM = 128;            // weight rows per tile (MMA M, TMEM lanes)
+constexpr int kBK = 64;             // bf16 elements per stage: 128 bytes
+constexpr int kThreads = 192;
+constexpr int kMaxNt = 256;
+constexpr uint64_t kWaitNs = 2000000000ull;
+constexpr uint64_t kDrainNs = 200000000ull;
+constexpr int kSmemLimit = 232448;
+// up-half exchange (64 lanes x 32 columns f32) + barriers and flags
+constexpr int kFixedSmem = 64 * 32 * 4 + 32 * 8 + 64;
+
+struct ProjArgs {
+  __nv_bfloat16* out;
+  const __nv_bfloat16* res;
+  float* part;          // split K: f32 partials [splits][N][O]
+  int* status;
+  int N, O, K, ldo;     // rows, weight rows, reduction length, output row stride
+  int Nt, n_tt, units, nkb, stages, splits;
+  uint32_t tmem_cols;
+};
+
+// unit u -> (weight tile, K split, token tile); the token tiles of one weight
+// slice are consecutive, so they share it through L2
+struct Unit {
+  int ot, sp, t0, kb0, kb1;
+};
+__device__ __forceinline__ Unit unit_of(const ProjArgs& a, int u) {
+  Unit x;
+  const int tt = u % a.n_tt, rest = u / a.n_tt;
+  x.sp = rest % a.splits;
+  x.ot = rest / a.splits;
+  x.t0 = tt * a.Nt;
+  x.kb0 = int((long long)x.sp * a.nkb / a.splits);
+  x.kb1 = int((long long)(x.sp + 1) * a.nkb / a.splits);
+  return x;
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
+               const ProjArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  const uint32_t a_bytes = kBM * 128, b_bytes = uint32_t(a.Nt) * 128;
+  const uint32_t stage_bytes = a_bytes + b_bytes;
+  float* upx = reinterpret_cast<float*>(smem + size_t(a.stages) * stage_bytes);  // [64][32]
+  uint64_t* full = reinterpret_cast<uint64_t*>(upx + 64 * 32);
+  uint64_t* empty = full + a.stages;
+  uint64_t* tfull = empty + a.stages;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int* epi_abort = abort_flag + 1;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < a.stages; ++s) {
+      mbar_init(full + s, 1);
+      mbar_init(empty + s, 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(tfull + b, 1);
+      mbar_init(tempty + b, 4);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    *epi_abort = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmW);
+    tma_prefetch_desc(&tmX);
+  }
+  pdl_begin();
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, a.tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const uint32_t buf_cols = a.tmem_cols / 2;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      const uint64_t pol_w = policy_evict_first(), pol_x = policy_evict_last();
+      int s = 0;
+      uint32_t ph = 0, issued = 0, issued_par = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
+        const Unit x = unit_of(a, u);
+        const int o0 = x.ot * kBM, t0 = x.t0;
+        for (int kb = x.kb0; kb < x.kb1; ++kb) {
+          if (!mbar_wait(empty + s, ph ^ 1u, kWaitNs, abort_flag)) {
+            ok = false;
+            break;
+          }
+          uint8_t* sa = smem + size_t(s) * stage_bytes;
+          mbar_arrive_expect_tx(full + s, stage_bytes);
+          tma_load_2d(sa, &tmW, full + s, kb * kBK, o0, pol_w);
+          tma_load_2d(sa + a_bytes, &tmX, full + s, kb * kBK, t0, pol_x);
+          issued |= 1u << s;
+          issued_par = (issued_par & ~(1u << s)) | (ph << s);
+          if (++s == a.stages) {
+            s = 0;
+            ph ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        flag(a.status, JET_ERR_TIMEOUT);
+        for (int t = 0; t < a.stages; ++t)
+          if (issued & (1u << t)) mbar_wait(full + t, (issued_par >> t) & 1u, kDrainNs, nullptr);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(kBM, a.Nt);
+      int s = 0, local = 0;
+      uint32_t ph = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x, ++local) {
+        const int buf = local & 1;
+        const uint32_t tph = (local >> 1) & 1;
+        if (!mbar_wait(tempty + buf, tph ^ 1u, kWaitNs, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + buf * buf_cols;
+        const Unit x = unit_of(a, u);
+        for (int kb = x.kb0; kb < x.kb1; ++kb) {
+          if (!mbar_wait(full + s, ph, kWaitNs, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + size_t(s) * stage_bytes), sb = sa + a_bytes;
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            mma_f16(d_tmem, desc_k_sw128(sa + 32 * k), desc_k_sw128(sb + 32 * k), idesc,
+                    (kb - x.kb0) != 0 || k != 0);
+          mma_commit(empty + s);
+          if (++s == a.stages) {
+            s = 0;
+            ph ^= 1u;
+          }
+        }
+        if (!ok) break;
+        mma_commit(tfull + buf);
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        flag(a.status, JET_ERR_TIMEOUT);
+        mma_commit(drain);
+        mbar_wait(drain, 0, kDrainNs, nullptr);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;            // TMEM lane quadrant this warp may access
+    int local = 0;
+    for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++local) {
+      const int buf = local & 1;
+      const uint32_t tph = (local >> 1) & 1;
+      const Unit x = unit_of(a, u);
+      const int ot = x.ot, t0 = x.t0;
+      const bool ok = warp_mbar_wait(tfull + buf, tph, kWaitNs, abort_flag);
+      if (!ok || *abort_flag) *epi_abort = 1;
+      named_bar_sync(1, 128);
+      if (*epi_abort) break;
+      tc_fence_after();
+      const uint32_t tl = tmem_base + buf * buf_cols + (uint32_t(32 * q) << 16);
+      const int ncols = min(a.Nt, a.N - t0);
+      for (int c0 = 0; c0 < ncols; c0 += 32) {
+        float v[32];
+        tmem_ld_32cols(tl + uint32_t(c0), v);
+        tmem_wait_ld();
+        const int nc = min(32, ncols - c0);
+        if (a.splits > 1) {
+          // a K range of a split GEMM: the raw f32 partial
+          const int o = ot * kBM + 32 * q + lane;
+          if (o < a.O) {
+            float* pp = a.part + (size_t(x.sp) * a.N + t0 + c0) * a.O + o;
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (i < nc) pp[size_t(i) * a.O] = v[i];
+          }
+        } else if (EPI == kProjSwiGLU) {
+          // lanes 64..127 hold the up features: hand them to the gate lanes
+          if (q >= 2) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) upx[(32 * (q - 2) + lane) * 32 + ((i + lane) & 31)] = v[i];
+          }
+          named_bar_sync(1, 128);
+          if (q < 2) {
+            const int f = ot * 64 + 32 * q + lane;  // output feature
+            if (f < a.O / 2) {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                if (i < nc) {
+                  const float up = upx[(32 * q + lane) * 32 + ((i + lane) & 31)];
+                  const float g = v[i];
+                  const float y = g / (1.f + __expf(-g)) * up;
+                  a.out[size_t(t0 + c0 + i) * a.ldo + f] = __float2bfloat16_rn(y);
+                }
+              }
+            }
+          }
+          named_bar_sync(1, 128);
+        } else {
+          const int o = ot * kBM + 32 * q + lane;  // output feature
+          if (o < a.O) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              if (i < nc) {
+                const size_t at = size_t(t0 + c0 + i) * a.ldo + o;
+                float y = v[i];
+                if (EPI == kProjResid) y += __bfloat162float(a.res[at]);
+                a.out[at] = __float2bfloat16_rn(y);
+              }
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty + buf);
+    }
+    if (*epi_abort) flag(a.status, JET_ERR_TIMEOUT);
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, a.tmem_cols);
+  }
+}
+
+// the epilogue of a split GEMM: sum the f32 partials, then store / add the
+// residual / SiLU(gate) * up; one thread per output element
+template <int EPI>
+__global__ void proj_reduce_kernel(const float* __restrict__ part, int splits, int N, int O,
+                                   __nv_bfloat16* __restrict__ out, int ldo,
+                                   const __nv_bfloat16* res) {
+  pdl_begin();
+  const int width = EPI == kProjSwiGLU ? O / 2 : O;
+  const long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= (long long)N * width) return;
+  const int n = int(e / width), c = int(e % width);
+  if (EPI == kProjSwiGLU) {
+    const int gr = 128 * (c / 64) + c % 64;  // the gate row of feature c; its up row is 64 on
+    float g = 0.f, up = 0.f;
+    for (int s = 0; s < splits; ++s) {
+      const float* row = part + (size_t(s) * N + n) * O;
+      g += row[gr];
+      up += row[gr + 64];
+    }
+    out[size_t(n) * ldo + c] = __float2bfloat16_rn(g / (1.f + __expf(-g)) * up);
+  } else {
+    float acc = 0.f;
+    for (int s = 0; s < splits; ++s) acc += part[(size_t(s) * N + n) * O + c];
+    if (EPI == kProjResid) acc += __bfloat162float(res[size_t(n) * ldo + c]);
+    out[size_t(n) * ldo + c] = __float2bfloat16_rn(acc);
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult qr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &qr) == cudaSuccess &&
+        qr == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// row-major bf16 [rows, K] with row stride ld elements; box 64 x box_rows,
+// 128-byte swizzle
+bool encode_rows(CUtensorMap* map, const void* base, int rows, int K, int ld, int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[2] = {cuuint64_t(K), cuuint64_t(rows)};
+  const cuuint64_t strides[1] = {cuuint64_t(ld) * 2};
+  const cuuint32_t box[2] = {cuuint32_t(kBK), cuuint32_t(box_rows)};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int sm_count() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  return n;
+}
+
+struct Tiling {
+  int n_tt, Nt, otiles, nkb, splits;
+};
+
+// token tiles of at most 256 rows; K split until the units cover 152 SMs
+// twice, keeping at least 8 K slices per unit. A function of the shapes only,
+// so that the workspace planned for a call matches the launch.
+constexpr int kPlanSMs = 152;
+Tiling tiling(int N, int O, int K, bool split) {
+  Tiling t{};
+  t.n_tt = (N + kMaxNt - 1) / kMaxNt;
+  t.Nt = ((N + t.n_tt - 1) / t.n_tt + 15) / 16 * 16;
+  t.n_tt = (N + t.Nt - 1) / t.Nt;
+  t.otiles = (O + kBM - 1) / kBM;
+  t.nkb = (K + kBK - 1) / kBK;
+  const int units = t.otiles * t.n_tt;
+  t.splits = 1;
+  while (split && units * t.splits < 2 * kPlanSMs && t.nkb / (t.splits + 1) >= 8) ++t.splits;
+  return t;
+}
+
+template <int EPI>
+cudaError_t launch_epi(const void* x, int N, int K, int ldx, const void* w, int O, void* out,
+                       int ldo, const void* res, float* part, int* status, cudaStream_t st) {
+  const Tiling tl = tiling(N, O, K, part != nullptr);
+  const int n_tt = tl.n_tt, Nt = tl.Nt;
+  ProjArgs a{};
+  a.part = part;
+  a.splits = part ? tl.splits : 1;
+  a.out = static_cast<__nv_bfloat16*>(out);
+  a.res = static_cast<const __nv_bfloat16*>(res);
+  a.status = status;
+  a.N = N;
+  a.O = O;
+  a.K = K;
+  a.ldo = ldo;
+  a.Nt = Nt;
+  a.n_tt = n_tt;
+  a.units = tl.otiles * n_tt * a.splits;
+  a.nkb = (K + kBK - 1) / kBK;
+  a.tmem_cols = Nt <= 128 ? 256 : 512;
+  const int stage_bytes = kBM * 128 + Nt * 128;
+  a.stages = std::min(8, (kSmemLimit - 1024 - kFixedSmem) / stage_bytes);
+  const size_t smem = 1024 + size_t(a.stages) * stage_bytes + kFixedSmem;
+  CUtensorMap tmW, tmX;
+  if (!encode_rows(&tmW, w, O, K, K, kBM) || !encode_rows(&tmX, x, N, K, ldx, Nt))
+    return cudaErrorInvalidValue;
+  cudaError_t e = cudaFuncSetAttribute(proj_tc_kernel<EPI>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  if (e != cudaSuccess) return e;
+  const int grid = std::max(1, std::min(a.units, sm_count()));
+  e = launch_pdl(proj_tc_kernel<EPI>, dim3(grid), dim3(kThreads), smem, st, tmW, tmX, a);
+  if (e != cudaSuccess || a.splits == 1) return e;
+  const long long total = (long long)N * (EPI == kProjSwiGLU ? O / 2 : O);
+  return launch_pdl(proj_reduce_kernel<EPI>, dim3(unsigned((total + 255) / 256)), dim3(256), 0, st,
+                    static_cast<const float*>(part), a.splits, N, O,
+                    static_cast<__nv_bfloat16*>(out), ldo,
+                    static_cast<const __nv_bfloat16*>(res));
+}
+
+}  // namespace
+
+size_t proj_partial_bytes(int N, int O, int K) {
+  const Tiling t = tiling(N, O, K, true);
+  return t.splits > 1 ? size_t(t.splits) * N * O * sizeof(float) : 0;
+}
+
+cudaError_t launch_proj(int epi, const void* x, int N, int K, int ldx, const void* w, int O,
+                        void* out, int ldo, const void* res, float* part, int* status,
+                        cudaStream_t st) {
+  if (N <= 0 || O <= 0) return cudaSuccess;
+  if (epi == kProjResid)
+    return launch_epi<kProjResid>(x, N, K, ldx, w, O, out, ldo, res, part, status, st);
+  if (epi == kProjSwiGLU)
+    return launch_epi<kProjSwiGLU>(x, N, K, ldx, w, O, out, ldo, res, part, status, st);
+  return launch_epi<kProjStore>(x, N, K, ldx, w, O, out, ldo, res, part, status, st);
+}
+
+}  // namespace jet

@@ -1,0 +1,235 @@
+// Small kernels of a decoder stack over the scoring step's rows: RMSNorm, the
+// split of a full-attention layer's q/k/v projection into the step's query and
+// candidate key/value buffers, the linear-attention layer's gates (per-head
+// key normalisation, sigmoid decay and write strengths), and the shared rows'
+// read of the prefix recurrent state. The projections themselves run on the
+// tensor cores (proj_tc.cu), the attention and the fork on the step's kernels.
+#include "jet_device.cuh"
+#include "jet_internal.h"
+
+namespace jet {
+namespace {
+
+constexpr int kRowsPerBlock = 8;  // one warp per row
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// h[n] = x[n] / sqrt(mean(x[n]^2) + eps) * g, one warp per row (D % 8 == 0)
+__global__ void __launch_bounds__(32 * kRowsPerBlock)
+rmsnorm_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restrict__ g, int N,
+               int D, float eps, __nv_bfloat16* __restrict__ h) {
+  pdl_begin();
+  const int lane = threadIdx.x & 31;
+  const int n = blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
+  if (n >= N) return;
+  const __nv_bfloat16* xr = x + size_t(n) * D;
+  float ss = 0.f;
+  for (int k = lane * 8; k < D; k += 256) {
+    const uint4 v = *reinterpret_cast<const uint4*>(xr + k);
+    const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(p[i]);
+      ss = fmaf(f.x, f.x, fmaf(f.y, f.y, ss));
+    }
+  }
+  ss = warp_sum(ss);
+  const float inv = 1.f / sqrtf(ss / float(D) + eps);
+  __nv_bfloat16* hr = h + size_t(n) * D;
+  for (int k = lane * 8; k < D; k += 256) {
+    const uint4 v = *reinterpret_cast<const uint4*>(xr + k);
+    const uint4 gv = *reinterpret_cast<const uint4*>(g + k);
+    const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&v);
+    const __nv_bfloat162* pg = reinterpret_cast<const __nv_bfloat162*>(&gv);
+    uint4 out;
+    __nv_bfloat162* po = reinterpret_cast<__nv_bfloat162*>(&out);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(p[i]), gg = __bfloat1622float2(pg[i]);
+      po[i] = __floats2bfloat162_rn(f.x * inv * gg.x, f.y * inv * gg.y);
+    }
+    *reinterpret_cast<uint4*>(hr + k) = out;
+  }
+}
+
+// z [N, (Hq + 2 Hkv) d] -> q [N, Hq d] (every row) and k_cand, v_cand
+// [F, Hkv d] (the fed rows, fed-token index n - req - 1); one block per row,
+// 16-byte pieces
+__global__ void split_qkv_kernel(const __nv_bfloat16* __restrict__ z, const int32_t* row_req,
+                                 const int32_t* row_cand, int N, int R, int qw, int kw,
+                                 __nv_bfloat16* __restrict__ q,
+                                 __nv_bfloat16* __restrict__ kc, __nv_bfloat16* __restrict__ vc,
+                                 int* status) {
+  pdl_begin();
+  const int n = blockIdx.x;
+  if (n >= N) return;
+  const int r = row_req[n];
+  const int zw = qw + 2 * kw;
+  const uint4* zr = reinterpret_cast<const uint4*>(z + size_t(n) * zw);
+  uint4* qr = reinterpret_cast<uint4*>(q + size_t(n) * qw);
+  for (int e = threadIdx.x; e < qw / 8; e += blockDim.x) qr[e] = zr[e];
+  if (r < 0 || r >= R) {
+    if (threadIdx.x == 0) flag(status, JET_ERR_DEVICE);
+    return;
+  }
+  // a shared row's key and value are the prefix's last position
+  if (row_cand[n] < 0) return;
+  const int f = n - r - 1;
+  if (f < 0 || f >= N - R) {
+    if (threadIdx.x == 0) flag(status, JET_ERR_DEVICE);
+    return;
+  }
+  uint4* kr = reinterpret_cast<uint4*>(kc + size_t(f) * kw);
+  uint4* vr = reinterpret_cast<uint4*>(vc + size_t(f) * kw);
+  for (int e = threadIdx.x; e < kw / 8; e += blockDim.x) {
+    kr[e] = zr[qw / 8 + e];
+    vr[e] = zr[(qw + kw) / 8 + e];
+  }
+}
+
+// z [N, Hl (2 dk + dv) + 2 Hl] -> lq_all [N, Hl, dk] (every row) and, for the
+// fed rows, lq, lk (normalised per head), lv, alpha = sigmoid(a),
+// beta = sigmoid(b); one warp per (row, head), dk = 128
+__global__ void __launch_bounds__(256)
+gates_kernel(const __nv_bfloat16* __restrict__ z, const int32_t* row_req,
+             const int32_t* row_cand, int N, int R, int Hl,
+             int dv, __nv_bfloat16* __restrict__ lq_all, __nv_bfloat16* __restrict__ lq,
+             __nv_bfloat16* __restrict__ lk, __nv_bfloat16* __restrict__ lv,
+             float* __restrict__ alpha, float* __restrict__ beta, int* status) {
+  pdl_begin();
+  constexpr int dk = 128;
+  const int lane = threadIdx.x & 31;
+  const int wid = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (wid >= N * Hl) return;
+  const int n = wid / Hl, hh = wid % Hl;
+  const int zw = Hl * (2 * dk + dv) + 2 * Hl;
+  const __nv_bfloat16* zr = z + size_t(n) * zw;
+  // this lane's 4 elements of q and k
+  const uint2 qv = *reinterpret_cast<const uint2*>(zr + hh * dk + 4 * lane);
+  const uint2 kv = *reinterpret_cast<const uint2*>(zr + Hl * dk + hh * dk + 4 * lane);
+  *reinterpret_cast<uint2*>(lq_all + (size_t(n) * Hl + hh) * dk + 4 * lane) = qv;
+  const int r = row_req[n];
+  if (r < 0 || r >= R) {
+    if (lane == 0) flag(status, JET_ERR_DEVICE);
+    return;
+  }
+  if (row_cand[n] < 0) return;  // the shared row only reads the prefix state
+  const int f = n - r - 1;
+  if (f < 0 || f >= N - R) {
+    if (lane == 0) flag(status, JET_ERR_DEVICE);
+    return;
+  }
+  *reinterpret_cast<uint2*>(lq + (size_t(f) * Hl + hh) * dk + 4 * lane) = qv;
+  const float2 k01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kv.x));
+  const float2 k23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kv.y));
+  float ss = k01.x * k01.x + k01.y * k01.y + k23.x * k23.x + k23.y * k23.y;
+  ss = warp_sum(ss);
+  const float inv = ss > 0.f ? 1.f / sqrtf(ss) : 0.f;
+  uint2 kn;
+  *reinterpret_cast<__nv_bfloat162*>(&kn.x) = __floats2bfloat162_rn(k01.x * inv, k01.y * inv);
+  *reinterpret_cast<__nv_bfloat162*>(&kn.y) = __floats2bfloat162_rn(k23.x * inv, k23.y * inv);
+  *reinterpret_cast<uint2*>(lk + (size_t(f) * Hl + hh) * dk + 4 * lane) = kn;
+  const __nv_bfloat16* vsrc = zr + 2 * Hl * dk + hh * dv;
+  __nv_bfloat16* vdst = lv + (size_t(f) * Hl + hh) * dv;
+  for (int j = lane; j < dv; j += 32) vdst[j] = vsrc[j];
+  if (lane == 0) {
+    const float a = __bfloat162float(zr[Hl * (2 * dk + dv) + hh]);
+    const float b = __bfloat162float(zr[Hl * (2 * dk + dv) + Hl + hh]);
+    alpha[size_t(f) * Hl + hh] = 1.f / (1.f + expf(-a));
+    beta[size_t(f) * Hl + hh] = 1.f / (1.f + expf(-b));
+  }
+}
+
+// o [N, Hl dv]: a shared row reads the prefix state (S^T q / sqrt(dk)), a fed
+// row takes the fork's output; grid (N, Hl), dv threads
+__global__ void readout_kernel(const float* __restrict__ s_prefix,
+                               const __nv_bfloat16* __restrict__ lq_all,
+                               const __nv_bfloat16* __restrict__ lo, const int32_t* row_req,
+                               const int32_t* row_cand, int N, int R, int Hl, int dv,
+                               __nv_bfloat16* __restrict__ o,
+                               int* status) {
+  pdl_begin();
+  constexpr int dk = 128;
+  __shared__ float qs[dk];
+  const int n = blockIdx.x, hh = blockIdx.y, j = threadIdx.x;
+  if (n >= N) return;
+  const int r = row_req[n];
+  if (r < 0 || r >= R) {
+    if (j == 0) flag(status, JET_ERR_DEVICE);
+    return;
+  }
+  const int f = n - r - 1;  // the fed-token index of a fed row
+  __nv_bfloat16* dst = o + (size_t(n) * Hl + hh) * dv;
+  if (row_cand[n] >= 0) {
+    if (f < 0 || f >= N - R) {
+      if (j == 0) flag(status, JET_ERR_DEVICE);
+      return;
+    }
+    if (j < dv) dst[j] = lo[(size_t(f) * Hl + hh) * dv + j];
+    return;
+  }
+  for (int i = j; i < dk; i += blockDim.x)
+    qs[i] = __bfloat162float(lq_all[(size_t(n) * Hl + hh) * dk + i]);
+  __syncthreads();
+  if (j < dv) {
+    const float* S = s_prefix + (size_t(r) * Hl + hh) * dk * dv;
+    float acc = 0.f;
+    for (int i = 0; i < dk; ++i) acc = fmaf(S[size_t(i) * dv + j], qs[i], acc);
+    dst[j] = __float2bfloat16_rn(acc * rsqrtf(float(dk)));
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_rmsnorm(const void* x, const void* g, int N, int D, float eps, void* h,
+                           cudaStream_t st) {
+  if (N <= 0) return cudaSuccess;
+  return launch_pdl(rmsnorm_kernel, dim3(unsigned((N + kRowsPerBlock - 1) / kRowsPerBlock)),
+                    dim3(32 * kRowsPerBlock), 0, st, static_cast<const __nv_bfloat16*>(x),
+                    static_cast<const __nv_bfloat16*>(g), N, D, eps,
+                    static_cast<__nv_bfloat16*>(h));
+}
+
+cudaError_t launch_split_qkv(const jet_layout& lay, const void* z, int qw, int kw, void* q,
+                             void* kc, void* vc, int* status, cudaStream_t st) {
+  const jet_sizes& n = lay.n;
+  if (n.N <= 0) return cudaSuccess;
+  return launch_pdl(split_qkv_kernel, dim3(unsigned(n.N)), dim3(128), 0, st,
+                    static_cast<const __nv_bfloat16*>(z), lay.row_req, lay.row_cand, n.N, n.R, qw,
+                    kw,
+                    static_cast<__nv_bfloat16*>(q), static_cast<__nv_bfloat16*>(kc),
+                    static_cast<__nv_bfloat16*>(vc), status);
+}
+
+cudaError_t launch_gates(const jet_layout& lay, const void* z, int Hl, int dv, void* lq_all,
+                         void* lq, void* lk, void* lv, float* alpha, float* beta, int* status,
+                         cudaStream_t st) {
+  const jet_sizes& n = lay.n;
+  if (n.N <= 0) return cudaSuccess;
+  const int warps = n.N * Hl;
+  return launch_pdl(gates_kernel, dim3(unsigned((warps + 7) / 8)), dim3(256), 0, st,
+                    static_cast<const __nv_bfloat16*>(z), lay.row_req, lay.row_cand, n.N, n.R, Hl,
+                    dv,
+                    static_cast<__nv_bfloat16*>(lq_all), static_cast<__nv_bfloat16*>(lq),
+                    static_cast<__nv_bfloat16*>(lk), static_cast<__nv_bfloat16*>(lv), alpha, beta,
+                    status);
+}
+
+cudaError_t launch_readout(const jet_layout& lay, const float* s_prefix, const void* lq_all,
+                           const void* lo, int Hl, int dv, void* o, int* status,
+                           cudaStream_t st) {
+  const jet_sizes& n = lay.n;
+  if (n.N <= 0) return cudaSuccess;
+  const int threads = dv < 128 ? 128 : dv;
+  return launch_pdl(readout_kernel, dim3(unsigned(n.N), unsigned(Hl)), dim3(unsigned(threads)), 0,
+                    st, s_prefix, static_cast<const __nv_bfloat16*>(lq_all),
+                    static_cast<const __nv_bfloat16*>(lo), lay.row_req, lay.row_cand, n.N, n.R, Hl,
+                    dv,
+                    static_cast<__nv_bfloat16*>(o), status);
+}
+
+}  // namespace jet

@@ -101,6 +101,10 @@ def _load() -> ctypes.CDLL:
         "jet_quantize_w4": (I, [P, ctypes.c_int64, ctypes.c_int64, P, P, P]),
         "jet_score_candidates_w4": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
                                         P, P, P, P, P, P, SZ, P]),
+        "jet_stack_workspace_bytes": (SZ, [ctypes.POINTER(jet_sizes), ctypes.POINTER(jet_dims),
+                                           I]),
+        "jet_stack_forward": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
+                                  P, P, P, P, SZ, P]),
         "jet_decide": (I, [ctypes.POINTER(jet_layout), I, P, P, P, P, P]),
         "jet_evaluate": (I, [ctypes.POINTER(jet_layout), P, P, P, P, P, P]),
         "jet_device_status": (I, [P, ctypes.POINTER(ctypes.c_int32)]),
@@ -118,7 +122,8 @@ DECLARED = ("jet_abi_version", "jet_status_string", "jet_layout_plan", "jet_layo
             "jet_prefill_workspace_bytes", "jet_prefill_attend", "jet_prefill_state",
             "jet_fork_state", "jet_fork_state_rule", "jet_score_candidates", "jet_score_candidates_noalloc",
             "jet_quantize_rows_e4m3", "jet_workspace_bytes_e4m3", "jet_score_candidates_e4m3",
-            "jet_w4_bytes", "jet_quantize_w4", "jet_score_candidates_w4", "jet_decide", "jet_evaluate", "jet_device_status")
+            "jet_w4_bytes", "jet_quantize_w4", "jet_score_candidates_w4",
+            "jet_stack_workspace_bytes", "jet_stack_forward", "jet_decide", "jet_evaluate", "jet_device_status")
 
 
 def library() -> ctypes.CDLL:
@@ -216,6 +221,33 @@ def jet_layout_build(prefix_len, n_cand, cand_len, target_ids, V: int) -> HostLa
                                  _ptr32(words), words.size, ctypes.byref(struct)),
            "jet_layout_build")
     return HostLayout(sizes, words, struct)
+
+
+LAYER_LINEAR, LAYER_FULL = 0, 1
+
+
+class jet_stack_layer(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int32), ("reserved", ctypes.c_int32)] + [
+        (n, ctypes.c_void_p) for n in ("g1", "g2", "w_mix", "w_o", "w_gu", "w_d", "k_pre",
+                                       "v_pre", "s_prefix")]
+
+
+class jet_stack(ctypes.Structure):
+    _fields_ = [("L", ctypes.c_int32), ("Dff", ctypes.c_int32), ("rule", ctypes.c_int32),
+                ("reserved", ctypes.c_int32), ("layers", ctypes.POINTER(jet_stack_layer))]
+
+
+def make_stack(layers, Dff: int, rule: int = 0):
+    """A jet_stack over a list of dicts (kind, g1, g2, w_mix, w_o, w_gu, w_d,
+    and k_pre/v_pre or s_prefix as tensors); returns (struct, keep-alive)."""
+    arr = (jet_stack_layer * max(1, len(layers)))()
+    for i, Ly in enumerate(layers):
+        arr[i].kind = int(Ly["kind"])
+        for n in ("g1", "g2", "w_mix", "w_o", "w_gu", "w_d", "k_pre", "v_pre", "s_prefix"):
+            setattr(arr[i], n, _addr(Ly.get(n)))
+    st = jet_stack(len(layers), int(Dff), int(rule), 0,
+                   ctypes.cast(arr, ctypes.POINTER(jet_stack_layer)))
+    return st, arr
 
 
 def make_dims(dtype: int, Hq=0, Hkv=0, d=0, D=0, Hl=0, dk=0, dv=0, max_sms=0) -> jet_dims:
@@ -343,6 +375,20 @@ def jet_score_candidates_w4(layout, dims: jet_dims, hidden, w4, w_scale, tok_log
                                         _addr(tok_logprob), _addr(cand_score), _addr(ws),
                                         int(ws_bytes), _stream(stream)),
            "jet_score_candidates_w4")
+
+
+def jet_stack_workspace_bytes(sizes: jet_sizes, dims: jet_dims, Dff: int) -> int:
+    return int(_lib.jet_stack_workspace_bytes(ctypes.byref(sizes), ctypes.byref(dims), int(Dff)))
+
+
+def jet_stack_forward(layout, dims: jet_dims, stack, x0, x, ws, ws_bytes: Optional[int] = None,
+                      stream=None) -> None:
+    """x = the decoder stack applied to x0 (see include/jet.h); ``stack`` is
+    the struct returned by :func:`make_stack`."""
+    ws_bytes = ws.numel() * ws.element_size() if ws_bytes is None else ws_bytes
+    _check(_lib.jet_stack_forward(ctypes.byref(_lay(layout)), ctypes.byref(dims),
+                                  ctypes.byref(stack), _addr(x0), _addr(x), _addr(ws),
+                                  int(ws_bytes), _stream(stream)), "jet_stack_forward")
 
 
 def jet_decide(layout, mode: int, cand_score, q, choice, value, stream=None) -> None:

@@ -202,3 +202,33 @@ class ScoringStep:
         h2d += sum(host[k].numel() * host[k].element_size() for k in self.input_names())
         d2h = sum(getattr(self, k).numel() * getattr(self, k).element_size() for k in RESULTS)
         return h2d, d2h
+
+
+class DecoderStack:
+    """A hybrid decoder stack's device tensors and workspace for one batch
+    shape. ``layers`` is a list of dicts: kind ("linear" or "full") and the
+    tensors g1, g2, w_mix, w_o, w_gu, w_d and k_pre/v_pre (full) or s_prefix
+    (linear), already on the device."""
+
+    def __init__(self, layout: "jet.HostLayout", dims: "jet.jet_dims", layers, Dff: int,
+                 rule: str = "delta", device="cuda"):
+        self.dev = torch.device(device)
+        self.layout = layout.to_device(self.dev)
+        self.dims = dims
+        self.layers = [dict(L, kind=jet.LAYER_FULL if L["kind"] == "full" else jet.LAYER_LINEAR)
+                       for L in layers]
+        self.stack, self._keep = jet.make_stack(self.layers, Dff, jet.RULES[rule])
+        n = layout.sizes
+        self.N = n.N
+        wsb = jet.jet_stack_workspace_bytes(n, dims, Dff)
+        if wsb == 0:
+            raise ValueError("invalid stack sizes")
+        self.ws = torch.empty((wsb + 15) // 16 * 4, dtype=torch.float32, device=self.dev)
+        self.x = torch.empty(n.N, dims.D, dtype=torch.bfloat16, device=self.dev)
+
+    def forward(self, x0: torch.Tensor, stream=None, layout=None) -> torch.Tensor:
+        """Enqueue the stack on ``stream``; returns the output rows [N, D]."""
+        lay = self.layout if layout is None else layout
+        jet.jet_stack_forward(lay, self.dims, self.stack, x0, self.x, self.ws, stream=stream)
+        return self.x
+

@@ -237,6 +237,38 @@ def test_w4_validation(jet):
     assert lib.jet_score_candidates_w4(L, ctypes.byref(bf), *mis, 1 << 30, None) == 4
 
 
+def test_stack_validation(jet):
+    lay, dims = _setup(jet)   # Hq 8, Hkv 2, d 64, D 64, Hl 2, dk 128, dv 64
+    lib = jet.library()
+    L = ctypes.byref(lay.struct)
+    ws = jet.jet_stack_workspace_bytes(lay.sizes, dims, 128)
+    assert ws > 0 and jet.jet_stack_workspace_bytes(lay.sizes, dims, 100) == 0
+    full = dict(kind="full", **{n: FAKE for n in ("g1", "g2", "w_mix", "w_o", "w_gu", "w_d",
+                                                  "k_pre", "v_pre")})
+    lin = dict(kind="linear", **{n: FAKE for n in ("g1", "g2", "w_mix", "w_o", "w_gu", "w_d",
+                                                   "s_prefix")})
+
+    def call(layers, Dff=128, rule=0, d=dims, ws_bytes=ws):
+        arr = [dict(L2, kind=jet.LAYER_FULL if L2["kind"] == "full" else
+                    (jet.LAYER_LINEAR if L2["kind"] == "linear" else L2["kind"]))
+               for L2 in layers]
+        st, keep = jet.make_stack(arr, Dff, rule)
+        return lib.jet_stack_forward(L, ctypes.byref(d), ctypes.byref(st), FAKE, FAKE, FAKE,
+                                     ws_bytes, None)
+
+    assert call([full, lin], ws_bytes=16) == 5                        # workspace
+    assert call([full, lin], Dff=96) == 2                             # Dff % 64 != 0
+    assert call([full], rule=9) == 1                                  # unknown rule
+    assert call([dict(full, kind=7)]) == 1                            # unknown kind
+    assert call([dict(lin, s_prefix=None)]) == 1                      # null state
+    assert call([dict(full, w_gu=MIS)]) == 4                          # misaligned weight
+    odd = jet.make_dims(jet.DTYPE_BF16, Hq=8, Hkv=2, d=64, D=64, Hl=3, dk=128, dv=64)
+    assert call([lin], d=odd) == 7                                    # Hl odd
+    f32 = jet.make_dims(jet.DTYPE_F32, Hq=8, Hkv=2, d=64, D=64, Hl=2, dk=128, dv=64)
+    assert call([full], d=f32) == 7                                   # bf16 only
+    assert call([]) == 0                                              # no layers: a copy
+
+
 def test_e4m3_validation(jet):
     lay, dims = _setup(jet)
     lib = jet.library()
