@@ -20,6 +20,11 @@
 // Split K: when the (weight tile, token tile) units are too few to occupy the
 // SMs (few output features, long K), each unit covers a range of K and writes
 // its f32 partial; a reduce kernel sums the partials and applies the epilogue.
+// Tile pairs: with at most 128 rows per row tile, a unit covers two weight
+// tiles that share every row tile (two TMEM accumulators, still double
+// buffered), which halves the row-tile bytes a weight byte costs - the row
+// tile is re-read from L2 for every weight tile, and the bytes one SM can take
+// in, not HBM, bound these small-N GEMMs.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -52,7 +57,9 @@ struct ProjArgs {
   int* status;
   int N, O, K, ldo;     // rows, weight rows, reduction length, output row stride
   int Nt, n_tt, units, nkb, stages, splits;
-  uint32_t tmem_cols;
+  int pair;             // weight tiles per unit (1 or 2)
+  int nbuf;             // accumulator sets (2: the epilogue overlaps the next unit)
+  uint32_t tmem_cols, acc_cols;
 };
 
 // unit u -> (weight tile, K split, token tile); the token tiles of one weight
@@ -79,7 +86,7 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   const uint32_t a_bytes = kBM * 128, b_bytes = uint32_t(a.Nt) * 128;
-  const uint32_t stage_bytes = a_bytes + b_bytes;
+  const uint32_t stage_bytes = a.pair * a_bytes + b_bytes;
   float* upx = reinterpret_cast<float*>(smem + size_t(a.stages) * stage_bytes);  // [64][32]
   uint64_t* full = reinterpret_cast<uint64_t*>(upx + 64 * 32);
   uint64_t* empty = full + a.stages;
@@ -118,7 +125,6 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const uint32_t buf_cols = a.tmem_cols / 2;
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -129,7 +135,7 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
       bool ok = true;
       for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
         const Unit x = unit_of(a, u);
-        const int o0 = x.ot * kBM, t0 = x.t0;
+        const int o0 = x.ot * a.pair * kBM, t0 = x.t0;
         for (int kb = x.kb0; kb < x.kb1; ++kb) {
           if (!mbar_wait(empty + s, ph ^ 1u, kWaitNs, abort_flag)) {
             ok = false;
@@ -137,8 +143,9 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
           }
           uint8_t* sa = smem + size_t(s) * stage_bytes;
           mbar_arrive_expect_tx(full + s, stage_bytes);
-          tma_load_2d(sa, &tmW, full + s, kb * kBK, o0, pol_w);
-          tma_load_2d(sa + a_bytes, &tmX, full + s, kb * kBK, t0, pol_x);
+          for (int t = 0; t < a.pair; ++t)
+            tma_load_2d(sa + t * a_bytes, &tmW, full + s, kb * kBK, o0 + t * kBM, pol_w);
+          tma_load_2d(sa + a.pair * a_bytes, &tmX, full + s, kb * kBK, t0, pol_x);
           issued |= 1u << s;
           issued_par = (issued_par & ~(1u << s)) | (ph << s);
           if (++s == a.stages) {
@@ -162,14 +169,14 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
       uint32_t ph = 0;
       bool ok = true;
       for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x, ++local) {
-        const int buf = local & 1;
-        const uint32_t tph = (local >> 1) & 1;
+        const int buf = local % a.nbuf;
+        const uint32_t tph = (local / a.nbuf) & 1;
         if (!mbar_wait(tempty + buf, tph ^ 1u, kWaitNs, abort_flag)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + buf * buf_cols;
+        const uint32_t d_tmem = tmem_base + uint32_t(buf * a.pair) * a.acc_cols;
         const Unit x = unit_of(a, u);
         for (int kb = x.kb0; kb < x.kb1; ++kb) {
           if (!mbar_wait(full + s, ph, kWaitNs, abort_flag)) {
@@ -177,11 +184,14 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
             break;
           }
           tc_fence_after();
-          const uint32_t sa = smem_u32(smem + size_t(s) * stage_bytes), sb = sa + a_bytes;
+          const uint32_t sa = smem_u32(smem + size_t(s) * stage_bytes);
+          const uint32_t sb = sa + a.pair * a_bytes;
+          for (int t = 0; t < a.pair; ++t) {
 #pragma unroll
-          for (int k = 0; k < 4; ++k)
-            mma_f16(d_tmem, desc_k_sw128(sa + 32 * k), desc_k_sw128(sb + 32 * k), idesc,
-                    (kb - x.kb0) != 0 || k != 0);
+            for (int k = 0; k < 4; ++k)
+              mma_f16(d_tmem + t * a.acc_cols, desc_k_sw128(sa + t * a_bytes + 32 * k),
+                      desc_k_sw128(sb + 32 * k), idesc, (kb - x.kb0) != 0 || k != 0);
+          }
           mma_commit(empty + s);
           if (++s == a.stages) {
             s = 0;
@@ -203,17 +213,20 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
     const int q = warp & 3;            // TMEM lane quadrant this warp may access
     int local = 0;
     for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++local) {
-      const int buf = local & 1;
-      const uint32_t tph = (local >> 1) & 1;
+      const int buf = local % a.nbuf;
+      const uint32_t tph = (local / a.nbuf) & 1;
       const Unit x = unit_of(a, u);
-      const int ot = x.ot, t0 = x.t0;
+      const int t0 = x.t0;
       const bool ok = warp_mbar_wait(tfull + buf, tph, kWaitNs, abort_flag);
       if (!ok || *abort_flag) *epi_abort = 1;
       named_bar_sync(1, 128);
       if (*epi_abort) break;
       tc_fence_after();
-      const uint32_t tl = tmem_base + buf * buf_cols + (uint32_t(32 * q) << 16);
       const int ncols = min(a.Nt, a.N - t0);
+      for (int pt = 0; pt < a.pair; ++pt) {
+      const int ot = x.ot * a.pair + pt;  // this accumulator's weight tile
+      const uint32_t tl = tmem_base + uint32_t(buf * a.pair + pt) * a.acc_cols +
+                          (uint32_t(32 * q) << 16);
       for (int c0 = 0; c0 < ncols; c0 += 32) {
         float v[32];
         tmem_ld_32cols(tl + uint32_t(c0), v);
@@ -265,6 +278,7 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
           }
         }
       }
+      }  // the unit's weight tiles
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty + buf);
@@ -344,7 +358,7 @@ int sm_count() {
 }
 
 struct Tiling {
-  int n_tt, Nt, otiles, nkb, splits;
+  int n_tt, Nt, otiles, pair, groups, nkb, splits;
 };
 
 // token tiles of at most 256 rows; K split until the units cover 152 SMs
@@ -357,8 +371,12 @@ Tiling tiling(int N, int O, int K, bool split) {
   t.Nt = ((N + t.n_tt - 1) / t.n_tt + 15) / 16 * 16;
   t.n_tt = (N + t.Nt - 1) / t.Nt;
   t.otiles = (O + kBM - 1) / kBM;
+  // pairs only where both accumulator sets still fit (Nt <= 128): without the
+  // overlap of the epilogue with the next unit a pair was measured slower
+  t.pair = (t.otiles >= 2 && t.Nt <= 128) ? 2 : 1;
+  t.groups = (t.otiles + t.pair - 1) / t.pair;
   t.nkb = (K + kBK - 1) / kBK;
-  const int units = t.otiles * t.n_tt;
+  const int units = t.groups * t.n_tt;
   t.splits = 1;
   while (split && units * t.splits < 2 * kPlanSMs && t.nkb / (t.splits + 1) >= 8) ++t.splits;
   return t;
@@ -381,10 +399,13 @@ cudaError_t launch_epi(const void* x, int N, int K, int ldx, const void* w, int 
   a.ldo = ldo;
   a.Nt = Nt;
   a.n_tt = n_tt;
-  a.units = tl.otiles * n_tt * a.splits;
+  a.pair = tl.pair;
+  a.units = tl.groups * n_tt * a.splits;
   a.nkb = (K + kBK - 1) / kBK;
-  a.tmem_cols = Nt <= 128 ? 256 : 512;
-  const int stage_bytes = kBM * 128 + Nt * 128;
+  a.acc_cols = Nt <= 128 ? 128 : 256;
+  a.nbuf = 2 * a.pair * int(a.acc_cols) <= 512 ? 2 : 1;
+  a.tmem_cols = uint32_t(a.nbuf * a.pair) * a.acc_cols;
+  const int stage_bytes = a.pair * kBM * 128 + Nt * 128;
   a.stages = std::min(8, (kSmemLimit - 1024 - kFixedSmem) / stage_bytes);
   const size_t smem = 1024 + size_t(a.stages) * stage_bytes + kFixedSmem;
   CUtensorMap tmW, tmX;
