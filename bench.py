@@ -223,6 +223,41 @@ def _attend_launches(problem, w) -> int:
     return 2 + (1 if splits > 1 else 0)
 
 
+def _proj_launches(N: int, O: int, K: int) -> int:
+    """Kernels one projection launches: the GEMM, plus the reduce of a split K
+    (the library's rule: row tiles of at most 256, two weight tiles per unit
+    for row tiles of at most 128, K split until the units cover 152 SMs twice
+    with at least 8 K slices each)."""
+    n_tt = (N + 255) // 256
+    Nt = ((N + n_tt - 1) // n_tt + 15) // 16 * 16
+    n_tt = (N + Nt - 1) // Nt
+    otiles = (O + 127) // 128
+    pair = 2 if (otiles >= 2 and Nt <= 128) else 1
+    units = (otiles + pair - 1) // pair * n_tt
+    nkb = (K + 63) // 64
+    splits = 1
+    while units * splits < 2 * 152 and nkb // (splits + 1) >= 8:
+        splits += 1
+    return 1 + (1 if splits > 1 else 0)
+
+
+def _stack_launches(problem, w, spec) -> int:
+    """Kernels one jet_stack_forward launches (the copy of x0 aside)."""
+    N, D, Dff = problem.N, w.D, spec.Dff
+    n = 0
+    for kind in spec.kinds:
+        if kind == "full":
+            zw, ow = (w.Hq + 2 * w.Hkv) * w.d, w.Hq * w.d
+            mixer = 1 + _attend_launches(problem, w)       # split + attention
+        else:
+            zw, ow = w.Hl * (2 * w.dk + w.dv) + 2 * w.Hl, w.Hl * w.dv
+            mixer = 3                                        # gates, fork, readout
+        n += 2 + mixer                                       # two RMSNorms
+        n += _proj_launches(N, zw, D) + _proj_launches(N, D, ow)
+        n += _proj_launches(N, 2 * Dff, D) + _proj_launches(N, D, Dff)
+    return n
+
+
 def aggregate(total_ms: float, e2e_ms: float, R: int, steps: int, world: int, device=None):
     """Whole-job numbers of N independent replicas: the slowest rank's timed
     regions (max over ranks) and the sets all ranks scored per second.
@@ -668,7 +703,7 @@ def run_stack(args):
                     Dff=spec.Dff, R=R, N=N, D=w.D, rule=args.rule),
         roofline=roof, parts=dict(stack_ms=round(ms_stack, 4),
                                   score_and_decide_ms=round(ms - ms_stack, 4)),
-        gpu_launches=None)), flush=True)
+        gpu_launches=(_stack_launches(p, w, spec) + 4) * args.steps)), flush=True)
 
 
 # ---------------------------------------------------------------------------
