@@ -158,3 +158,27 @@ def test_stack_full_size_hybrid4(cuda):
     p = jet_synth.make_problem("ordinal_hybrid")
     got, _ = _gpu_stack(cuda, p, spec, "delta")
     _check_rows(got, _oracle_stack(p, spec, "delta"), len(spec.kinds))
+
+
+def test_stack_edges(cuda):
+    import torch
+    from paper_2609_33874_gb300.step import DecoderStack
+    # every candidate a single token: no fed rows (F = 0), a one-token prefix
+    spec = jet_synth.StackSpec(("linear", "full"), 128)
+    p = jet_synth.custom_problem(SMALL, [1, 5], [2, 3], [1, 1, 1, 1, 1], [3, 4, 5, 6, 7], seed=43)
+    got, st = _gpu_stack(cuda, p, spec, "delta")
+    _check_rows(got, _oracle_stack(p, spec, "delta"), len(spec.kinds))
+    # in place (x = x0) gives the same rows as out of place
+    x0 = jet_synth.array_to_torch(jet_synth.stack_x0(p), "cuda")
+    xin = x0.clone()
+    cuda.jet_stack_forward(st.layout, st.dims, st.stack, xin, xin, st.ws)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(xin.float().cpu().numpy(), got)
+    # no layers: a copy
+    w = p.work
+    hl = cuda.jet_layout_build(p.prefix_len, p.n_cand, p.cand_len, p.target_ids, w.V)
+    empty = DecoderStack(hl, st.dims, [], 128)
+    y = empty.forward(x0)
+    torch.cuda.synchronize()
+    assert cuda.jet_device_status() == 0
+    assert torch.equal(y, x0)
