@@ -10,25 +10,25 @@
 namespace jet {
 namespace {
 
-constexpr int kRowsPerBlock = 8;  // one warp per row
-
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
 }
 
-// h[n] = x[n] / sqrt(mean(x[n]^2) + eps) * g, one warp per row (D % 8 == 0)
-__global__ void __launch_bounds__(32 * kRowsPerBlock)
+// h[n] = x[n] / sqrt(mean(x[n]^2) + eps) * g, one 128-thread block per row
+// (D % 8 == 0): a row of a few KB gets four warps' loads in flight
+constexpr int kNormThreads = 128;
+__global__ void __launch_bounds__(kNormThreads)
 rmsnorm_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restrict__ g, int N,
                int D, float eps, __nv_bfloat16* __restrict__ h) {
   pdl_begin();
-  const int lane = threadIdx.x & 31;
-  const int n = blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
+  __shared__ float part[kNormThreads / 32];
+  const int n = blockIdx.x, tid = threadIdx.x;
   if (n >= N) return;
   const __nv_bfloat16* xr = x + size_t(n) * D;
   float ss = 0.f;
-  for (int k = lane * 8; k < D; k += 256) {
+  for (int k = tid * 8; k < D; k += kNormThreads * 8) {
     const uint4 v = *reinterpret_cast<const uint4*>(xr + k);
     const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&v);
 #pragma unroll
@@ -38,9 +38,14 @@ rmsnorm_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restr
     }
   }
   ss = warp_sum(ss);
+  if ((tid & 31) == 0) part[tid >> 5] = ss;
+  __syncthreads();
+  ss = 0.f;
+#pragma unroll
+  for (int w = 0; w < kNormThreads / 32; ++w) ss += part[w];
   const float inv = 1.f / sqrtf(ss / float(D) + eps);
   __nv_bfloat16* hr = h + size_t(n) * D;
-  for (int k = lane * 8; k < D; k += 256) {
+  for (int k = tid * 8; k < D; k += kNormThreads * 8) {
     const uint4 v = *reinterpret_cast<const uint4*>(xr + k);
     const uint4 gv = *reinterpret_cast<const uint4*>(g + k);
     const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&v);
@@ -188,8 +193,8 @@ __global__ void readout_kernel(const float* __restrict__ s_prefix,
 cudaError_t launch_rmsnorm(const void* x, const void* g, int N, int D, float eps, void* h,
                            cudaStream_t st) {
   if (N <= 0) return cudaSuccess;
-  return launch_pdl(rmsnorm_kernel, dim3(unsigned((N + kRowsPerBlock - 1) / kRowsPerBlock)),
-                    dim3(32 * kRowsPerBlock), 0, st, static_cast<const __nv_bfloat16*>(x),
+  return launch_pdl(rmsnorm_kernel, dim3(unsigned(N)), dim3(kNormThreads), 0, st,
+                    static_cast<const __nv_bfloat16*>(x),
                     static_cast<const __nv_bfloat16*>(g), N, D, eps,
                     static_cast<__nv_bfloat16*>(h));
 }
