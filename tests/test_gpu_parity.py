@@ -149,11 +149,23 @@ def test_fork_small(cuda, keep, dtype):
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 @pytest.mark.parametrize("rule", ["delta", "gla"])
 def test_fork_long_candidates(cuda, dtype, rule):
-    # candidates of up to 40 tokens: the 32-token window of fed tokens is
-    # staged again inside a candidate and across candidates; both recurrences
+    # candidates of up to 40 tokens: a candidate runs through several 16-token
+    # windows of fed tokens (its state carried across them); both recurrences
     p = _custom("ordinal_hybrid", [5, 9], [4, 3], [20, 40, 1, 33, 7, 12, 2], seed=41, V=4096,
                 D=256, Hl=2, dv=96, dtype=dtype)
     got, _ = run_problem(cuda, p, rule=rule)
+    lay = oracle_layout(p)
+    check_fork(lay, p, got, list(range(p.R)), rule=rule)
+
+
+@pytest.mark.parametrize("rule", ["delta", "gla"])
+def test_fork_window_splits(cuda, rule):
+    # short candidates that straddle the 16-token windows of fed tokens at
+    # several offsets, beside one-token candidates and a request with none fed
+    cl = [2] + [3] * 9 + [1, 4, 2, 5, 3, 1, 6, 2] + [1, 1]
+    p = _custom("ordinal_hybrid", [6, 3], [18, 2], cl, seed=42, V=4096, D=256, Hl=2, dv=64,
+                dtype="bf16")
+    got, _ = run_problem(cuda, p, keep_fork=True, rule=rule)
     lay = oracle_layout(p)
     check_fork(lay, p, got, list(range(p.R)), rule=rule)
 
