@@ -1,12 +1,11 @@
-// Device code shared by the two kernels of the linear-attention recurrence
-// (scan.cu: the prefix scan; fork.cu: the per-candidate fork): a CTA keeps a
+// Device code of the register-resident linear-attention recurrence (the
+// prefix scan, scan.cu): a CTA keeps a
 // 128 x 64 slice of the state S in registers (thread = 32 rows x 2 columns,
 // the lanes of a row group adjacent), fed tokens are staged 16 at a time
 // (asynchronous copies into a raw buffer, widened to fp32 at the window
 // boundary, one extra k row for the window's last token), and one sweep over
 // a thread's rows per token applies the update and accumulates the output and
-// the next token's k^T S. Included by one translation unit each, inside an
-// anonymous namespace.
+// the next token's k^T S. Included inside an anonymous namespace.
 #pragma once
 
 
