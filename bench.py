@@ -251,7 +251,7 @@ def _stack_launches(problem, w, spec) -> int:
             mixer = 1 + _attend_launches(problem, w)       # split + attention
         else:
             zw, ow = w.Hl * (2 * w.dk + w.dv) + 2 * w.Hl, w.Hl * w.dv
-            mixer = 3                                        # gates, fork, readout
+            mixer = 2                                        # gates, fork (with the shared rows)
         n += 2 + mixer                                       # two RMSNorms
         n += _proj_launches(N, zw, D) + _proj_launches(N, D, ow)
         n += _proj_launches(N, 2 * Dff, D) + _proj_launches(N, D, Dff)

@@ -395,7 +395,7 @@ namespace {
 
 // scratch of jet_stack_forward (offsets 256-byte aligned)
 struct StackPlan {
-  size_t h, z, q, kc, vc, lqa, lqf, lk, lv, al, be, lo, o, u, attn, part, bytes;
+  size_t h, z, q, kc, vc, lqa, lqf, lk, lv, al, be, o, u, attn, part, bytes;
   jet::AttnPlan attn_plan;
   bool full_ok, lin_ok;
 };
@@ -446,7 +446,6 @@ StackPlan stack_plan(const jet_sizes& n, const jet_dims& d, int Dff) {
     p.lv = take(F * d.Hl * d.dv * b);
     p.al = take(F * d.Hl * 4);
     p.be = take(F * d.Hl * 4);
-    p.lo = take(F * d.Hl * d.dv * b);
   }
   p.bytes = at;
   return p;
@@ -534,12 +533,12 @@ extern "C" jet_status jet_stack_forward(const jet_layout* lay, const jet_dims* d
       JET_TRY(cuda_status(jet::launch_gates(*lay, w + plan.z, dims->Hl, dims->dv, w + plan.lqa,
                                             w + plan.lqf, w + plan.lk, w + plan.lv, al, be,
                                             status, st)));
-      if (F > 0)
-        JET_TRY(cuda_status(jet::launch_fork_state(*lay, *dims, stack->rule, Ly.s_prefix,
-                                                   w + plan.lqf, w + plan.lk, w + plan.lv, al, be,
-                                                   w + plan.lo, nullptr, status, st)));
-      JET_TRY(cuda_status(jet::launch_readout(*lay, Ly.s_prefix, w + plan.lqa, w + plan.lo,
-                                              dims->Hl, dims->dv, w + plan.o, status, st)));
+      // fed rows through the fork, shared rows from the prefix states: all N
+      // rows of the mixer output
+      JET_TRY(cuda_status(jet::launch_fork_state(*lay, *dims, stack->rule, Ly.s_prefix,
+                                                 w + plan.lqf, w + plan.lk, w + plan.lv, al, be,
+                                                 w + plan.o, nullptr, status, st,
+                                                 w + plan.lqa)));
       ow = dims->Hl * dims->dv;
     }
     JET_TRY(cuda_status(jet::launch_proj(jet::kProjResid, w + plan.o, int(N), ow, ow, Ly.w_o, D,

@@ -150,14 +150,18 @@ __device__ __forceinline__ float4 token_step(float4 (&S)[8], int wt, const T (*w
 
 // grid (dv / 32, Hl, R); thread (warp w, lane = 8 * rg + jq) owns rows
 // 32 w + rg + 4 ii (ii < 8) and columns j0 + 4 jq .. + 3 of the slice.
+// q_rows (optional, [N, Hl, dk]): every row's q; the request's shared row then
+// reads the prefix state, o = S_r^T q / sqrt(dk), and o holds all N rows
+// (fed token f at row f + r + 1) instead of the fed tokens alone.
 template <typename T, bool DELTA>
 __global__ void __launch_bounds__(kThreads)
 fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__ cand_row_offset,
             const int32_t* __restrict__ tgt_offset, const int32_t* __restrict__ row_offset,
             int R, int C, int F, int Hl, int dv, const float* __restrict__ s_prefix,
             const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
-            const float* __restrict__ alpha, const float* __restrict__ beta, T* __restrict__ o,
-            float* __restrict__ s_fork, int* status) {
+            const float* __restrict__ alpha, const float* __restrict__ beta,
+            const T* __restrict__ q_rows, T* __restrict__ o, float* __restrict__ s_fork,
+            int* status) {
   pdl_begin();
   __shared__ __align__(16) float red[4 * kCols];
   // a window of the request's fed tokens as stored: k, q (all rows), v (this
@@ -170,6 +174,7 @@ fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__
   __shared__ int cm[kMeta], cf[kMeta];
   // the prefix state slice, each thread's own 8 float4 at [ii][tid]
   __shared__ __align__(16) float4 ssp[8 * kThreads];
+  __shared__ float qsh[kDK];  // the shared row's q (with q_rows)
   const int r = blockIdx.z, h = blockIdx.y, j0 = blockIdx.x * kCols;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rg = lane >> 3, jq = lane & 7;
@@ -185,9 +190,11 @@ fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__
 
   // the prefix state slice (read once, kept in shared memory for every
   // candidate) and the first window of fed tokens load at once
+  const float rs = rsqrtf(float(kDK));
   {
     float4 sp[8];
     const size_t head = (size_t(r) * Hl + h) * kDK;
+    if (q_rows && tid < kDK) qsh[tid] = to_f32(q_rows[(size_t(row_offset[r]) * Hl + h) * kDK + tid]);
 #pragma unroll
     for (int ii = 0; ii < 8; ++ii) {
       const int i = 32 * warp + rg + 4 * ii;
@@ -195,11 +202,27 @@ fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__
     }
 #pragma unroll
     for (int ii = 0; ii < 8; ++ii) ssp[ii * kThreads + tid] = sp[ii];
+    if (q_rows) {
+      // the shared row: o = S_r^T q / sqrt(dk), from the prefix state itself
+      __syncthreads();  // qsh is in
+      float4 op = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int ii = 0; ii < 8; ++ii) op = f4_fma(qsh[32 * warp + rg + 4 * ii], sp[ii], op);
+      op = rows_sum(op, red, warp, lane);
+      if (warp == 0 && rg == 0) {
+        T* dst = o + (size_t(row_offset[r]) * Hl + h) * dv + col;
+        dst[0] = from_f32<T>(op.x * rs);
+        dst[1] = from_f32<T>(op.y * rs);
+        dst[2] = from_f32<T>(op.z * rs);
+        dst[3] = from_f32<T>(op.w * rs);
+      }
+    }
   }
+  // with q_rows, fed token f is written at row f + r + 1
+  const size_t o_shift = q_rows ? size_t(r) + 1 : 0;
   int w0 = f_begin, w1 = min(f_begin + kWin, f_end);  // fed tokens [w0, w1) are staged
   if (w1 > w0)
     stage_window(q, k, v, alpha, beta, Hl, dv, h, j0, w0, w1 - w0, tid, wk, wq, wv, wa, wb);
-  const float rs = rsqrtf(float(kDK));
 
   for (int cb = c0; cb < c1; cb += kMeta) {
     const int nb = min(kMeta, c1 - cb);
@@ -232,7 +255,7 @@ fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__
         const float4 op = token_step<T, DELTA>(S, wt_of(f, w0), wk, wq, wv, wa, wb, red, warp,
                                                lane);
         if (warp == 0 && rg == 0) {
-          T* dst = o + (size_t(f) * Hl + h) * dv + col;
+          T* dst = o + ((size_t(f) + o_shift) * Hl + h) * dv + col;
           dst[0] = from_f32<T>(op.x * rs);
           dst[1] = from_f32<T>(op.y * rs);
           dst[2] = from_f32<T>(op.z * rs);
@@ -258,8 +281,8 @@ namespace {
 template <bool DELTA>
 cudaError_t launch_rule(const jet_layout& lay, const jet_dims& d, const float* s_prefix,
                         const void* q, const void* k, const void* v, const float* alpha,
-                        const float* beta, void* o, float* s_fork, int* status,
-                        cudaStream_t st) {
+                        const float* beta, const void* q_rows, void* o, float* s_fork,
+                        int* status, cudaStream_t st) {
   const jet_sizes& n = lay.n;
   dim3 grid(unsigned(d.dv / kCols), unsigned(d.Hl), unsigned(n.R));
   const int F = n.N - n.R;
@@ -267,14 +290,15 @@ cudaError_t launch_rule(const jet_layout& lay, const jet_dims& d, const float* s
     return launch_pdl(fork_kernel<float, DELTA>, grid, dim3(kThreads), 0, st, lay.cand_offset,
                       lay.cand_row_offset, lay.tgt_offset, lay.row_offset, n.R, n.C, F, d.Hl,
                       d.dv, s_prefix, static_cast<const float*>(q), static_cast<const float*>(k),
-                      static_cast<const float*>(v), alpha, beta, static_cast<float*>(o), s_fork,
-                      status);
+                      static_cast<const float*>(v), alpha, beta,
+                      static_cast<const float*>(q_rows), static_cast<float*>(o), s_fork, status);
   }
   return launch_pdl(fork_kernel<__nv_bfloat16, DELTA>, grid, dim3(kThreads), 0, st,
                     lay.cand_offset, lay.cand_row_offset, lay.tgt_offset, lay.row_offset, n.R,
                     n.C, F, d.Hl, d.dv, s_prefix, static_cast<const __nv_bfloat16*>(q),
                     static_cast<const __nv_bfloat16*>(k), static_cast<const __nv_bfloat16*>(v),
-                    alpha, beta, static_cast<__nv_bfloat16*>(o), s_fork, status);
+                    alpha, beta, static_cast<const __nv_bfloat16*>(q_rows),
+                    static_cast<__nv_bfloat16*>(o), s_fork, status);
 }
 
 }  // namespace
@@ -283,10 +307,11 @@ cudaError_t launch_rule(const jet_layout& lay, const jet_dims& d, const float* s
 cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, int rule,
                               const float* s_prefix, const void* q, const void* k, const void* v,
                               const float* alpha, const float* beta, void* o, float* s_fork,
-                              int* status, cudaStream_t st) {
+                              int* status, cudaStream_t st, const void* q_rows) {
   if (rule == JET_RECUR_GLA)
-    return launch_rule<false>(lay, d, s_prefix, q, k, v, alpha, beta, o, s_fork, status, st);
-  return launch_rule<true>(lay, d, s_prefix, q, k, v, alpha, beta, o, s_fork, status, st);
+    return launch_rule<false>(lay, d, s_prefix, q, k, v, alpha, beta, q_rows, o, s_fork, status,
+                              st);
+  return launch_rule<true>(lay, d, s_prefix, q, k, v, alpha, beta, q_rows, o, s_fork, status, st);
 }
 
 }  // namespace jet

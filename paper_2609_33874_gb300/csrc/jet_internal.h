@@ -85,10 +85,13 @@ cudaError_t launch_prefill_tc(const jet_layout& lay, const jet_dims& d, const vo
                               const void* k, const void* v, void* o, void* ws, int* status,
                               cudaStream_t st);
 
+// q_rows (optional, every row's q [N, Hl, dk]): o then covers all N rows, the
+// shared rows reading the prefix states (o = S_r^T q / sqrt(dk)) and fed token
+// f at row f + r + 1; without it o holds the fed tokens only
 cudaError_t launch_fork_state(const jet_layout& lay, const jet_dims& d, int rule,
                               const float* s_prefix, const void* q, const void* k, const void* v,
                               const float* alpha, const float* beta, void* o, float* s_fork,
-                              int* status, cudaStream_t st);
+                              int* status, cudaStream_t st, const void* q_rows = nullptr);
 
 // logits partials: writes part[N][vtiles] (m, s) in base 2 - m = max_v z log2(e),
 // s = sum_v 2^(z log2(e) - m) over the tile - and z_tgt[T]
@@ -119,8 +122,6 @@ cudaError_t launch_split_qkv(const jet_layout& lay, const void* z, int qw, int k
 cudaError_t launch_gates(const jet_layout& lay, const void* z, int Hl, int dv, void* lq_all,
                          void* lq, void* lk, void* lv, float* alpha, float* beta, int* status,
                          cudaStream_t st);
-cudaError_t launch_readout(const jet_layout& lay, const float* s_prefix, const void* lq_all,
-                           const void* lo, int Hl, int dv, void* o, int* status, cudaStream_t st);
 
 // the LM head on tiled 4-bit weights (w4) and e4m3 hidden codes
 cudaError_t launch_lmhead_w4(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,

@@ -1,9 +1,10 @@
 // Small kernels of a decoder stack over the scoring step's rows: RMSNorm, the
 // split of a full-attention layer's q/k/v projection into the step's query and
 // candidate key/value buffers, the linear-attention layer's gates (per-head
-// key normalisation, sigmoid decay and write strengths), and the shared rows'
-// read of the prefix recurrent state. The projections themselves run on the
-// tensor cores (proj_tc.cu), the attention and the fork on the step's kernels.
+// key normalisation, sigmoid decay and write strengths). The projections
+// themselves run on the tensor cores (proj_tc.cu), the attention and the fork
+// (which also reads the shared rows' outputs off the prefix states) on the
+// step's kernels.
 #include "jet_device.cuh"
 #include "jet_internal.h"
 
@@ -149,45 +150,6 @@ gates_kernel(const __nv_bfloat16* __restrict__ z, const int32_t* row_req,
   }
 }
 
-// o [N, Hl dv]: a shared row reads the prefix state (S^T q / sqrt(dk)), a fed
-// row takes the fork's output; grid (N, Hl), dv threads
-__global__ void readout_kernel(const float* __restrict__ s_prefix,
-                               const __nv_bfloat16* __restrict__ lq_all,
-                               const __nv_bfloat16* __restrict__ lo, const int32_t* row_req,
-                               const int32_t* row_cand, int N, int R, int Hl, int dv,
-                               __nv_bfloat16* __restrict__ o,
-                               int* status) {
-  pdl_begin();
-  constexpr int dk = 128;
-  __shared__ float qs[dk];
-  const int n = blockIdx.x, hh = blockIdx.y, j = threadIdx.x;
-  if (n >= N) return;
-  const int r = row_req[n];
-  if (r < 0 || r >= R) {
-    if (j == 0) flag(status, JET_ERR_DEVICE);
-    return;
-  }
-  const int f = n - r - 1;  // the fed-token index of a fed row
-  __nv_bfloat16* dst = o + (size_t(n) * Hl + hh) * dv;
-  if (row_cand[n] >= 0) {
-    if (f < 0 || f >= N - R) {
-      if (j == 0) flag(status, JET_ERR_DEVICE);
-      return;
-    }
-    if (j < dv) dst[j] = lo[(size_t(f) * Hl + hh) * dv + j];
-    return;
-  }
-  for (int i = j; i < dk; i += blockDim.x)
-    qs[i] = __bfloat162float(lq_all[(size_t(n) * Hl + hh) * dk + i]);
-  __syncthreads();
-  if (j < dv) {
-    const float* S = s_prefix + (size_t(r) * Hl + hh) * dk * dv;
-    float acc = 0.f;
-    for (int i = 0; i < dk; ++i) acc = fmaf(S[size_t(i) * dv + j], qs[i], acc);
-    dst[j] = __float2bfloat16_rn(acc * rsqrtf(float(dk)));
-  }
-}
-
 }  // namespace
 
 cudaError_t launch_rmsnorm(const void* x, const void* g, int N, int D, float eps, void* h,
@@ -222,19 +184,6 @@ cudaError_t launch_gates(const jet_layout& lay, const void* z, int Hl, int dv, v
                     static_cast<__nv_bfloat16*>(lq_all), static_cast<__nv_bfloat16*>(lq),
                     static_cast<__nv_bfloat16*>(lk), static_cast<__nv_bfloat16*>(lv), alpha, beta,
                     status);
-}
-
-cudaError_t launch_readout(const jet_layout& lay, const float* s_prefix, const void* lq_all,
-                           const void* lo, int Hl, int dv, void* o, int* status,
-                           cudaStream_t st) {
-  const jet_sizes& n = lay.n;
-  if (n.N <= 0) return cudaSuccess;
-  const int threads = dv < 128 ? 128 : dv;
-  return launch_pdl(readout_kernel, dim3(unsigned(n.N), unsigned(Hl)), dim3(unsigned(threads)), 0,
-                    st, s_prefix, static_cast<const __nv_bfloat16*>(lq_all),
-                    static_cast<const __nv_bfloat16*>(lo), lay.row_req, lay.row_cand, n.N, n.R, Hl,
-                    dv,
-                    static_cast<__nv_bfloat16*>(o), status);
 }
 
 }  // namespace jet
