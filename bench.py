@@ -244,17 +244,23 @@ def _proj_launches(N: int, O: int, K: int) -> int:
 def _stack_launches(problem, w, spec) -> int:
     """Kernels one jet_stack_forward launches (the copy of x0 aside)."""
     N, D, Dff = problem.N, w.D, spec.Dff
-    n = 0
-    for kind in spec.kinds:
+
+    def resid(K, norm):
+        # a residual projection; the RMSNorm after it shares the reduce of a
+        # split K, else it is a launch of its own
+        k = _proj_launches(N, D, K)
+        return k + (1 if norm and k == 1 else 0)
+
+    n = 1 if spec.kinds else 0                               # the first layer's RMSNorm
+    for l, kind in enumerate(spec.kinds):
         if kind == "full":
             zw, ow = (w.Hq + 2 * w.Hkv) * w.d, w.Hq * w.d
             mixer = 1 + _attend_launches(problem, w)       # split + attention
         else:
             zw, ow = w.Hl * (2 * w.dk + w.dv) + 2 * w.Hl, w.Hl * w.dv
             mixer = 2                                        # gates, fork (with the shared rows)
-        n += 2 + mixer                                       # two RMSNorms
-        n += _proj_launches(N, zw, D) + _proj_launches(N, D, ow)
-        n += _proj_launches(N, 2 * Dff, D) + _proj_launches(N, D, Dff)
+        n += mixer + _proj_launches(N, zw, D) + resid(ow, True)
+        n += _proj_launches(N, 2 * Dff, D) + resid(Dff, l + 1 < len(spec.kinds))
     return n
 
 

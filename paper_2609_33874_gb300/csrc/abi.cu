@@ -470,7 +470,7 @@ extern "C" jet_status jet_stack_forward(const jet_layout* lay, const jet_dims* d
   if (stack->Dff < 64 || stack->Dff % 64 != 0) return JET_ERR_SHAPE;
   if (stack->rule != JET_RECUR_DELTA && stack->rule != JET_RECUR_GLA) return JET_ERR_ARG;
   const jet_sizes& n = lay->n;
-  const long long N = n.N, F = n.N - n.R;
+  const long long N = n.N;
   const StackPlan plan = stack_plan(n, *dims, stack->Dff);
   // validate every layer before the first launch
   for (int l = 0; l < stack->L; ++l) {
@@ -512,7 +512,9 @@ extern "C" jet_status jet_stack_forward(const jet_layout* lay, const jet_dims* d
   for (int l = 0; l < stack->L; ++l) {
     const jet_stack_layer& Ly = stack->layers[l];
     const bool full = Ly.kind == JET_LAYER_FULL;
-    JET_TRY(cuda_status(jet::launch_rmsnorm(x, Ly.g1, int(N), D, 1e-6f, w + plan.h, st)));
+    // h = RMSNorm(x; g1): the previous layer's down projection already wrote it
+    if (l == 0)
+      JET_TRY(cuda_status(jet::launch_rmsnorm(x, Ly.g1, int(N), D, 1e-6f, w + plan.h, st)));
     const int zw = full ? (dims->Hq + 2 * dims->Hkv) * dims->d
                         : dims->Hl * (2 * dims->dk + dims->dv) + 2 * dims->Hl;
     JET_TRY(cuda_status(jet::launch_proj(jet::kProjStore, w + plan.h, int(N), D, D, Ly.w_mix, zw,
@@ -541,14 +543,18 @@ extern "C" jet_status jet_stack_forward(const jet_layout* lay, const jet_dims* d
                                                  w + plan.lqa)));
       ow = dims->Hl * dims->dv;
     }
+    // x += W_o o, then h = RMSNorm(x; g2)
     JET_TRY(cuda_status(jet::launch_proj(jet::kProjResid, w + plan.o, int(N), ow, ow, Ly.w_o, D,
-                                         x, D, x, part, status, st)));
-    JET_TRY(cuda_status(jet::launch_rmsnorm(x, Ly.g2, int(N), D, 1e-6f, w + plan.h, st)));
+                                         x, D, x, part, status, st, Ly.g2, 1e-6f, w + plan.h)));
     JET_TRY(cuda_status(jet::launch_proj(jet::kProjSwiGLU, w + plan.h, int(N), D, D, Ly.w_gu,
                                          2 * Dff, w + plan.u, Dff, nullptr, part, status,
                                          st)));
+    // x += W_d u, then the next layer's h = RMSNorm(x; g1')
+    const bool next = l + 1 < stack->L;
     JET_TRY(cuda_status(jet::launch_proj(jet::kProjResid, w + plan.u, int(N), Dff, Dff, Ly.w_d,
-                                         D, x, D, x, part, status, st)));
+                                         D, x, D, x, part, status, st,
+                                         next ? stack->layers[l + 1].g1 : nullptr, 1e-6f,
+                                         next ? w + plan.h : nullptr)));
   }
   return JET_OK;
 }

@@ -110,10 +110,12 @@ enum { kProjStore = 0, kProjResid = 1, kProjSwiGLU = 2 };
 // out[N, O] = epilogue(x[N, K] w[O, K]^T) on the tensor cores (bf16, f32 accumulate);
 // ldx / ldo are the row strides of x and out in elements; res (kProjResid) may be
 // out; part: f32 scratch of proj_partial_bytes(N, O, K) bytes for a split K (null:
-// no split)
+// no split); kProjResid with norm_h: also h = RMSNorm(out; norm_g, norm_eps),
+// the next layer input, in the same pass where the K split allows
 cudaError_t launch_proj(int epi, const void* x, int N, int K, int ldx, const void* w, int O,
                         void* out, int ldo, const void* res, float* part, int* status,
-                        cudaStream_t st);
+                        cudaStream_t st, const void* norm_g = nullptr, float norm_eps = 0.f,
+                        void* norm_h = nullptr);
 size_t proj_partial_bytes(int N, int O, int K);
 cudaError_t launch_rmsnorm(const void* x, const void* g, int N, int D, float eps, void* h,
                            cudaStream_t st);

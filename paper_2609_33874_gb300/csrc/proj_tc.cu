@@ -322,6 +322,79 @@ __global__ void proj_reduce_kernel(const float* __restrict__ part, int splits, i
   }
 }
 
+// A split residual GEMM's epilogue together with the RMSNorm that follows it
+// in a decoder layer: one 512-thread block per row (a row's partials need many
+// loads in flight; with 128 threads the pass was slower than the two it
+// replaces), x = res + the sum of the partials (one rounding), then
+// h = x / sqrt(mean(x^2) + eps) * g from the rounded row, in the order of the
+// stand-alone RMSNorm kernel (the same results as the two passes). D % 8 == 0;
+// res may be out.
+constexpr int kNormThreads = 512;
+__global__ void __launch_bounds__(kNormThreads)
+proj_reduce_norm_kernel(const float* __restrict__ part, int splits, int N, int D,
+                        __nv_bfloat16* out, const __nv_bfloat16* res,
+                        const __nv_bfloat16* __restrict__ g, float eps,
+                        __nv_bfloat16* __restrict__ h) {
+  pdl_begin();
+  __shared__ float wsum[kNormThreads / 32];
+  const int n = blockIdx.x, tid = threadIdx.x;
+  if (n >= N) return;
+  __nv_bfloat16* xr = out + size_t(n) * D;
+  const __nv_bfloat16* rr = res + size_t(n) * D;
+  float ss = 0.f;
+#pragma unroll 2
+  for (int k = tid * 8; k < D; k += kNormThreads * 8) {
+    float acc[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc[i] = 0.f;
+    // several splits' loads in flight at once: a block per row has few threads
+#pragma unroll 4
+    for (int s = 0; s < splits; ++s) {
+      const float4* pp = reinterpret_cast<const float4*>(part + (size_t(s) * N + n) * D + k);
+      const float4 a0 = pp[0], a1 = pp[1];
+      acc[0] += a0.x; acc[1] += a0.y; acc[2] += a0.z; acc[3] += a0.w;
+      acc[4] += a1.x; acc[5] += a1.y; acc[6] += a1.z; acc[7] += a1.w;
+    }
+    const uint4 rv = *reinterpret_cast<const uint4*>(rr + k);
+    const __nv_bfloat162* pr = reinterpret_cast<const __nv_bfloat162*>(&rv);
+    uint4 xv;
+    __nv_bfloat162* px = reinterpret_cast<__nv_bfloat162*>(&xv);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(pr[i]);
+      px[i] = __floats2bfloat162_rn(acc[2 * i] + f.x, acc[2 * i + 1] + f.y);
+    }
+    *reinterpret_cast<uint4*>(xr + k) = xv;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(px[i]);
+      ss = fmaf(f.x, f.x, fmaf(f.y, f.y, ss));
+    }
+  }
+  ss = warp_sum(ss);
+  if ((tid & 31) == 0) wsum[tid >> 5] = ss;
+  __syncthreads();
+  ss = 0.f;
+#pragma unroll
+  for (int w = 0; w < kNormThreads / 32; ++w) ss += wsum[w];
+  const float inv = 1.f / sqrtf(ss / float(D) + eps);
+  __nv_bfloat16* hr = h + size_t(n) * D;
+  for (int k = tid * 8; k < D; k += kNormThreads * 8) {
+    const uint4 v = *reinterpret_cast<const uint4*>(xr + k);  // this thread's own writes
+    const uint4 gv = *reinterpret_cast<const uint4*>(g + k);
+    const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&v);
+    const __nv_bfloat162* pg = reinterpret_cast<const __nv_bfloat162*>(&gv);
+    uint4 o4;
+    __nv_bfloat162* po = reinterpret_cast<__nv_bfloat162*>(&o4);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(p[i]), gg = __bfloat1622float2(pg[i]);
+      po[i] = __floats2bfloat162_rn(f.x * inv * gg.x, f.y * inv * gg.y);
+    }
+    *reinterpret_cast<uint4*>(hr + k) = o4;
+  }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   static std::once_flag once;
@@ -357,6 +430,17 @@ int sm_count() {
   return n;
 }
 
+// the RMSNorm a residual projection's output feeds (h null: none)
+struct Norm {
+  const void* g;
+  float eps;
+  void* h;
+};
+
+template <int EPI>
+cudaError_t launch_reduce(const ProjArgs& a, float* part, int N, int O, void* out, int ldo,
+                          const void* res, cudaStream_t st);
+
 struct Tiling {
   int n_tt, Nt, otiles, pair, groups, nkb, splits;
 };
@@ -384,7 +468,8 @@ Tiling tiling(int N, int O, int K, bool split) {
 
 template <int EPI>
 cudaError_t launch_epi(const void* x, int N, int K, int ldx, const void* w, int O, void* out,
-                       int ldo, const void* res, float* part, int* status, cudaStream_t st) {
+                       int ldo, const void* res, float* part, int* status, cudaStream_t st,
+                       const Norm& nm) {
   const Tiling tl = tiling(N, O, K, part != nullptr);
   const int n_tt = tl.n_tt, Nt = tl.Nt;
   ProjArgs a{};
@@ -416,7 +501,24 @@ cudaError_t launch_epi(const void* x, int N, int K, int ldx, const void* w, int 
   if (e != cudaSuccess) return e;
   const int grid = std::max(1, std::min(a.units, sm_count()));
   e = launch_pdl(proj_tc_kernel<EPI>, dim3(grid), dim3(kThreads), smem, st, tmW, tmX, a);
-  if (e != cudaSuccess || a.splits == 1) return e;
+  if (e != cudaSuccess) return e;
+  const bool norm = EPI == kProjResid && nm.h != nullptr;
+  if (norm && a.splits > 1 && ldo == O && O % 8 == 0)
+    return launch_pdl(proj_reduce_norm_kernel, dim3(unsigned(N)), dim3(kNormThreads), 0, st,
+                      static_cast<const float*>(part), a.splits, N, O,
+                      static_cast<__nv_bfloat16*>(out), static_cast<const __nv_bfloat16*>(res),
+                      static_cast<const __nv_bfloat16*>(nm.g), nm.eps,
+                      static_cast<__nv_bfloat16*>(nm.h));
+  if (a.splits > 1) {
+    e = launch_reduce<EPI>(a, part, N, O, out, ldo, res, st);
+    if (e != cudaSuccess) return e;
+  }
+  return norm ? launch_rmsnorm(out, nm.g, N, O, nm.eps, nm.h, st) : cudaSuccess;
+}
+
+template <int EPI>
+cudaError_t launch_reduce(const ProjArgs& a, float* part, int N, int O, void* out, int ldo,
+                          const void* res, cudaStream_t st) {
   const long long total = (long long)N * (EPI == kProjSwiGLU ? O / 2 : O);
   return launch_pdl(proj_reduce_kernel<EPI>, dim3(unsigned((total + 255) / 256)), dim3(256), 0, st,
                     static_cast<const float*>(part), a.splits, N, O,
@@ -433,13 +535,14 @@ size_t proj_partial_bytes(int N, int O, int K) {
 
 cudaError_t launch_proj(int epi, const void* x, int N, int K, int ldx, const void* w, int O,
                         void* out, int ldo, const void* res, float* part, int* status,
-                        cudaStream_t st) {
+                        cudaStream_t st, const void* norm_g, float norm_eps, void* norm_h) {
   if (N <= 0 || O <= 0) return cudaSuccess;
+  const Norm nm{norm_g, norm_eps, norm_h};
   if (epi == kProjResid)
-    return launch_epi<kProjResid>(x, N, K, ldx, w, O, out, ldo, res, part, status, st);
+    return launch_epi<kProjResid>(x, N, K, ldx, w, O, out, ldo, res, part, status, st, nm);
   if (epi == kProjSwiGLU)
-    return launch_epi<kProjSwiGLU>(x, N, K, ldx, w, O, out, ldo, res, part, status, st);
-  return launch_epi<kProjStore>(x, N, K, ldx, w, O, out, ldo, res, part, status, st);
+    return launch_epi<kProjSwiGLU>(x, N, K, ldx, w, O, out, ldo, res, part, status, st, nm);
+  return launch_epi<kProjStore>(x, N, K, ldx, w, O, out, ldo, res, part, status, st, nm);
 }
 
 }  // namespace jet

@@ -17,9 +17,10 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
-// h[n] = x[n] / sqrt(mean(x[n]^2) + eps) * g, one 128-thread block per row
-// (D % 8 == 0): a row of a few KB gets four warps' loads in flight
-constexpr int kNormThreads = 128;
+// h[n] = x[n] / sqrt(mean(x[n]^2) + eps) * g, one 512-thread block per row
+// (D % 8 == 0): a row of a few KB gets sixteen warps' loads in flight; the
+// fused residual-and-norm pass of the projections keeps the same order
+constexpr int kNormThreads = 512;
 __global__ void __launch_bounds__(kNormThreads)
 rmsnorm_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restrict__ g, int N,
                int D, float eps, __nv_bfloat16* __restrict__ h) {
