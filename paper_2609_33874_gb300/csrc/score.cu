@@ -15,16 +15,21 @@
 namespace jet {
 namespace {
 
-// one block per row; coalesced reads of the row's partials part[n][0..vtiles)
-__global__ void __launch_bounds__(128)
+// one block per row (blockDim.x a multiple of 32, at most kLseThreads);
+// coalesced reads of the row's partials part[n][0..vtiles). 512 threads: a
+// row's ~1,200 partials are then two or three loads a thread, all in flight
+// at once (with 128 threads the merge was latency-bound: 1.5-2 us more a step)
+constexpr int kLseThreads = 512;
+__global__ void __launch_bounds__(kLseThreads)
 lse_kernel(const float2* __restrict__ part, int vtiles, int N, float* __restrict__ lse) {
   pdl_begin();
-  __shared__ float2 red[4];
+  __shared__ float2 red[kLseThreads / 32];
   const int n = blockIdx.x;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const float2* p = part + size_t(n) * vtiles;
   float m = -INFINITY, s = 0.f;
-  for (int vt = threadIdx.x; vt < vtiles; vt += 128) {
+#pragma unroll 4
+  for (int vt = threadIdx.x; vt < vtiles; vt += blockDim.x) {
     const float2 x = p[vt];
     ms_combine2(m, s, x.x, x.y);
   }
@@ -37,7 +42,7 @@ lse_kernel(const float2* __restrict__ part, int vtiles, int N, float* __restrict
   if (lane == 0) red[warp] = make_float2(m, s);
   __syncthreads();
   if (threadIdx.x == 0) {
-    for (int i = 1; i < 4; ++i) ms_combine2(m, s, red[i].x, red[i].y);
+    for (int i = 1; i < int(blockDim.x / 32); ++i) ms_combine2(m, s, red[i].x, red[i].y);
     lse[n] = (m + log2f(s)) * 0.6931471805599453f;  // partials are base 2
   }
 }
@@ -193,7 +198,8 @@ cudaError_t launch_score_finish(const jet_layout& lay, const ScorePlan& plan, vo
   const float* z_tgt = reinterpret_cast<const float*>(base + plan.ztgt_off);
   float* lse = reinterpret_cast<float*>(base + plan.lse_off);
   cudaError_t e =
-      launch_pdl(lse_kernel, dim3(unsigned(n.N)), dim3(128), 0, st, part, plan.vtiles, n.N, lse);
+      launch_pdl(lse_kernel, dim3(unsigned(n.N)), dim3(kLseThreads), 0, st, part, plan.vtiles,
+                 n.N, lse);
   if (e != cudaSuccess) return e;
   return launch_pdl(finish_kernel, dim3(unsigned((n.C + 127) / 128)), dim3(128), 0, st,
                     lay.tgt_offset, lay.tgt_row, n.C, n.N, n.T, z_tgt, lse, tok_logprob,
