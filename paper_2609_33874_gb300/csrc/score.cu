@@ -47,31 +47,39 @@ lse_kernel(const float2* __restrict__ part, int vtiles, int N, float* __restrict
   }
 }
 
-// one thread per candidate: its targets in t order
-__global__ void finish_kernel(const int32_t* __restrict__ tgt_offset, const int32_t* __restrict__ tgt_row,
-                              int C, int N, int T_, const float* __restrict__ z_tgt,
-                              const float* __restrict__ lse, float* __restrict__ tok_logprob,
-                              float* __restrict__ cand_score, int* status) {
+// one warp per candidate: lane t reads target t's logit and its row's lse
+// (32 targets at a time, all loads in flight together), then lane 0 adds the
+// log-probabilities in t order
+__global__ void __launch_bounds__(256)
+finish_kernel(const int32_t* __restrict__ tgt_offset, const int32_t* __restrict__ tgt_row, int C,
+              int N, int T_, const float* __restrict__ z_tgt, const float* __restrict__ lse,
+              float* __restrict__ tok_logprob, float* __restrict__ cand_score, int* status) {
   pdl_begin();
-  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  const int lane = threadIdx.x & 31;
+  const int c = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (c >= C) return;
   const int j0 = tgt_offset[c], j1 = tgt_offset[c + 1];
   if (j0 < 0 || j1 < j0 || j1 > T_) {
-    flag(status, JET_ERR_DEVICE);
+    if (lane == 0) flag(status, JET_ERR_DEVICE);
     return;
   }
   float acc = 0.f;
-  for (int j = j0; j < j1; ++j) {
-    const int n = tgt_row[j];
-    if (n < 0 || n >= N) {
-      flag(status, JET_ERR_DEVICE);
-      continue;
+  for (int jb = j0; jb < j1; jb += 32) {
+    const int j = jb + lane;
+    float ell = 0.f;
+    if (j < j1) {
+      const int n = tgt_row[j];
+      if (n < 0 || n >= N) {
+        flag(status, JET_ERR_DEVICE);
+      } else {
+        ell = z_tgt[j] - lse[n];
+        tok_logprob[j] = ell;
+      }
     }
-    const float ell = z_tgt[j] - lse[n];
-    tok_logprob[j] = ell;
-    acc += ell;
+    const int cnt = min(32, j1 - jb);
+    for (int t = 0; t < cnt; ++t) acc += __shfl_sync(0xffffffffu, ell, t);
   }
-  cand_score[c] = acc;
+  if (lane == 0) cand_score[c] = acc;
 }
 
 // one warp per request
@@ -201,7 +209,7 @@ cudaError_t launch_score_finish(const jet_layout& lay, const ScorePlan& plan, vo
       launch_pdl(lse_kernel, dim3(unsigned(n.N)), dim3(kLseThreads), 0, st, part, plan.vtiles,
                  n.N, lse);
   if (e != cudaSuccess) return e;
-  return launch_pdl(finish_kernel, dim3(unsigned((n.C + 127) / 128)), dim3(128), 0, st,
+  return launch_pdl(finish_kernel, dim3(unsigned((n.C + 7) / 8)), dim3(256), 0, st,
                     lay.tgt_offset, lay.tgt_row, n.C, n.N, n.T, z_tgt, lse, tok_logprob,
                     cand_score, status);
 }
