@@ -412,25 +412,28 @@ def run_gpu(args):
     call_ms["evaluate"] = ev_a.elapsed_time(ev_b) / n_eval
 
     # --- end to end: pinned host inputs, copies inside the timed region ---------
+    # a batch as a loader leaves it: its layout words and inputs in one pinned
+    # buffer (HostBatch), the results back into one pinned buffer (HostResults)
+    from paper_2609_33874_gb300.step import HostBatch, HostResults
     host = {k: x[k].cpu().pin_memory() for k in names}
     words = torch.from_numpy(hl.words).pin_memory()
-    out = {k: torch.empty_like(getattr(step, k), device="cpu").pin_memory()
-           for k in ("tok_logprob", "cand_score", "q_cand", "choice", "value")}
+    batch = HostBatch(step, host, words)
+    out = HostResults(step)
     # every step copies its inputs in and its results out; step i+1's input
-    # copies overlap step i's kernels (double-buffered device inputs)
+    # copy overlaps step i's kernels (double-buffered device inputs)
     e_steps = max(3, min(args.steps, 50))
-    step.run_pipelined([(host, words)] * max(3, args.warmup), w_lm,
+    step.run_pipelined([batch] * max(3, args.warmup), w_lm,
                        [out] * max(3, args.warmup), stream=stream)
     torch.cuda.synchronize(dev)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         torch.distributed.barrier()
     e0.record(stream)
-    step.run_pipelined([(host, words)] * e_steps, w_lm, [out] * e_steps, stream=stream)
+    step.run_pipelined([batch] * e_steps, w_lm, [out] * e_steps, stream=stream)
     e1.record(stream)
     torch.cuda.synchronize(dev)
     e2e_ms = e0.elapsed_time(e1) / e_steps
-    h2d, d2h = step.host_bytes(host, words)
+    h2d, d2h = batch.nbytes, out.buf.numel()
     assert jet.jet_device_status(stream) == 0
 
     total_ms, e2e_ms, ms_per_step, value, e2e_value = aggregate(

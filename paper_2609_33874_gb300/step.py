@@ -25,6 +25,66 @@ RESULTS = ("tok_logprob", "cand_score", "q_cand", "choice", "value")
 # below this many input bytes per batch (about 5 us over the host link)
 # run_pipelined copies on the compute stream instead of overlapping
 _OVERLAP_MIN_BYTES = 1 << 20
+_ALIGN = 256  # bytes: every packed tensor starts on this boundary
+
+
+def _pack_plan(items):
+    """(offsets, total bytes) of tensors laid end to end at _ALIGN boundaries;
+    items is a list of (name, dtype, shape)."""
+    offs, at = {}, 0
+    for name, dtype, shape in items:
+        at = (at + _ALIGN - 1) // _ALIGN * _ALIGN
+        n = 1
+        for d in shape:
+            n *= int(d)
+        offs[name] = (at, dtype, tuple(shape))
+        at += n * torch.empty((), dtype=dtype).element_size()
+    return offs, (at + _ALIGN - 1) // _ALIGN * _ALIGN
+
+
+def _views(buf: torch.Tensor, offs):
+    """Typed views of a uint8 buffer at the planned offsets."""
+    out = {}
+    for name, (o, dtype, shape) in offs.items():
+        n = 1
+        for d in shape:
+            n *= int(d)
+        nb = n * torch.empty((), dtype=dtype).element_size()
+        out[name] = buf[o:o + nb].view(dtype).view(shape)
+    return out
+
+
+class HostBatch:
+    """One batch's layout words and inputs in a single pinned host buffer, each
+    at a 256-byte aligned offset, so that the batch moves to the device in one
+    copy (a loader writes its batches straight into such buffers)."""
+
+    def __init__(self, step: "ScoringStep", host: Dict[str, torch.Tensor],
+                 layout_words: torch.Tensor):
+        items = [("__words__", layout_words.dtype, layout_words.shape)]
+        items += [(k, host[k].dtype, host[k].shape) for k in step.input_names()]
+        self.offsets, nbytes = _pack_plan(items)
+        self.buf = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
+        v = _views(self.buf, self.offsets)
+        v["__words__"].copy_(layout_words)
+        for k in step.input_names():
+            v[k].copy_(host[k])
+
+    @property
+    def nbytes(self) -> int:
+        return self.buf.numel()
+
+
+class HostResults:
+    """Pinned host buffer laid out like a step's results (one copy back):
+    ``views`` holds tok_logprob, cand_score, q_cand, choice and value."""
+
+    def __init__(self, step: "ScoringStep"):
+        self.buf = torch.empty(step._results.numel(), dtype=torch.uint8, pin_memory=True)
+        self.views = _views(self.buf, step._result_offsets)
+
+    def __getitem__(self, k):
+        return self.views[k]
 
 
 def quantize_lm_head(w_lm: torch.Tensor, stream=None):
@@ -81,11 +141,14 @@ class ScoringStep:
         dt = _TORCH_DTYPE[dims.dtype]
         z = lambda *s, dtype=torch.float32: torch.empty(*s, dtype=dtype, device=self.dev)  # noqa: E731
         self.o = z(n.N, dims.Hq, dims.d, dtype=dt)
-        self.tok_logprob = z(n.T)
-        self.cand_score = z(n.C)
-        self.q_cand = z(n.C)
-        self.choice = z(n.R, dtype=torch.int32)
-        self.value = z(n.R)
+        # the results share one device buffer, so that they return in one copy
+        self._result_offsets, rb = _pack_plan([
+            ("tok_logprob", torch.float32, (n.T,)), ("cand_score", torch.float32, (n.C,)),
+            ("q_cand", torch.float32, (n.C,)), ("choice", torch.int32, (n.R,)),
+            ("value", torch.float32, (n.R,))])
+        self._results = z(rb, dtype=torch.uint8)
+        for k, t in _views(self._results, self._result_offsets).items():
+            setattr(self, k, t)
         ws = (jet.jet_workspace_bytes if lm == "bf16" else jet.jet_workspace_bytes_e4m3)(n, dims)
         self.ws = z((ws + 15) // 16 * 4)  # float32 words, 16-byte multiple
         if hybrid:
@@ -156,9 +219,11 @@ class ScoringStep:
         """End to end over a sequence of batches of this step's shape: the
         host -> device copies of batch i+1 run on a copy stream while the
         kernels of batch i run on ``stream``; device inputs and layouts are
-        double-buffered. ``batches`` yields (pinned host inputs, pinned layout
-        words); ``outs[i]`` receives batch i's results (device -> host, on
-        ``stream``). Everything is enqueued; the caller synchronises."""
+        double-buffered. ``batches`` yields :class:`HostBatch` objects (one
+        copy each) or (pinned host inputs, pinned layout words) pairs;
+        ``outs[i]`` receives batch i's results (device -> host, on ``stream``):
+        a :class:`HostResults` (one copy) or a dict of pinned tensors.
+        Everything is enqueued; the caller synchronises."""
         s = torch.cuda.current_stream(self.dev) if stream is None else stream
         if getattr(self, "_pipe", None) is None:
             self._copy_stream = torch.cuda.Stream(self.dev)
@@ -172,29 +237,46 @@ class ScoringStep:
         start = torch.cuda.Event()
         start.record(s)
         cs.wait_event(start)  # after everything already enqueued on ``stream``
-        for i, (host, layout_words) in enumerate(batches):
+        for i, batch in enumerate(batches):
             buf = self._pipe[i % 2]
+            packed = isinstance(batch, HostBatch)
+            nbytes = batch.nbytes if packed else self.host_bytes(*batch)[0]
             # a batch whose copies take a few microseconds gains nothing from
             # the overlap and would pay the two cross-stream waits: copy in order
-            overlap = self.host_bytes(host, layout_words)[0] >= self.overlap_min_bytes
+            overlap = nbytes >= self.overlap_min_bytes
             with torch.cuda.stream(cs if overlap else s):
                 if overlap and i >= 2:
                     cs.wait_event(buf["consumed"])  # batch i-2's kernels are done with it
-                if buf["inputs"] is None:
-                    buf["inputs"] = {k: torch.empty_like(host[k], device=self.dev)
-                                     for k in self.input_names()}
-                buf["layout"].words.copy_(layout_words, non_blocking=True)
-                for k in self.input_names():
-                    buf["inputs"][k].copy_(host[k], non_blocking=True)
+                if packed:
+                    if buf.get("packed") is None or buf["packed"].numel() != nbytes:
+                        buf["packed"] = torch.empty(nbytes, dtype=torch.uint8, device=self.dev)
+                        v = _views(buf["packed"], batch.offsets)
+                        buf["packed_layout"] = jet.DeviceLayout(self.layout.sizes,
+                                                                v.pop("__words__"))
+                        buf["packed_inputs"] = v
+                    buf["packed"].copy_(batch.buf, non_blocking=True)
+                    inputs, layout = buf["packed_inputs"], buf["packed_layout"]
+                else:
+                    host, layout_words = batch
+                    if buf["inputs"] is None:
+                        buf["inputs"] = {k: torch.empty_like(host[k], device=self.dev)
+                                         for k in self.input_names()}
+                    buf["layout"].words.copy_(layout_words, non_blocking=True)
+                    for k in self.input_names():
+                        buf["inputs"][k].copy_(host[k], non_blocking=True)
+                    inputs, layout = buf["inputs"], buf["layout"]
                 if overlap:
                     buf["copied"].record(cs)
             if overlap:
                 s.wait_event(buf["copied"])
-            self.run(buf["inputs"], w_lm, stream=s, layout=buf["layout"])
+            self.run(inputs, w_lm, stream=s, layout=layout)
             buf["consumed"].record(s)
             with torch.cuda.stream(s):
-                for k in RESULTS:
-                    outs[i][k].copy_(getattr(self, k), non_blocking=True)
+                if isinstance(outs[i], HostResults):
+                    outs[i].buf.copy_(self._results, non_blocking=True)
+                else:
+                    for k in RESULTS:
+                        outs[i][k].copy_(getattr(self, k), non_blocking=True)
 
     def host_bytes(self, host: Dict[str, torch.Tensor], layout_words: torch.Tensor):
         """(host->device, device->host) bytes one :meth:`run_from_host` moves."""

@@ -266,13 +266,17 @@ def test_end_to_end_from_host(cuda):
     assert h2d > 0 and d2h > 0
 
 
+@pytest.mark.parametrize("packed", [False, True])
 @pytest.mark.parametrize("overlap", [True, False])
-def test_end_to_end_pipelined(cuda, overlap):
+def test_end_to_end_pipelined(cuda, overlap, packed):
     """Four batches of one shape with their own hidden states and targets,
     copied in on the copy stream while the previous batch computes (or in
     order on the compute stream): each batch's results must be its own (the
-    double buffers are reused from the third batch on)."""
+    double buffers are reused from the third batch on). ``packed``: every
+    batch in one pinned buffer (HostBatch), the results back into one
+    (HostResults)."""
     import torch
+    from paper_2609_33874_gb300.step import HostBatch, HostResults
     p0 = jet_synth.make_problem("tiny")
     rng = np.random.default_rng(7)
     probs = [jet_synth.custom_problem(p0.work, p0.prefix_len, p0.n_cand, p0.cand_len,
@@ -284,9 +288,14 @@ def test_end_to_end_pipelined(cuda, overlap):
     for p in probs:
         hl = cuda.jet_layout_build(p.prefix_len, p.n_cand, p.cand_len, p.target_ids, p.work.V)
         host = {k: jet_synth.torch_tensor(p, k, pin=True) for k in step.input_names()}
-        batches.append((host, torch.from_numpy(hl.words).pin_memory()))
-        outs.append({k: torch.empty_like(getattr(step, k), device="cpu").pin_memory()
-                     for k in ("tok_logprob", "cand_score", "q_cand", "choice", "value")})
+        words = torch.from_numpy(hl.words).pin_memory()
+        if packed:
+            batches.append(HostBatch(step, host, words))
+            outs.append(HostResults(step))
+        else:
+            batches.append((host, words))
+            outs.append({k: torch.empty_like(getattr(step, k), device="cpu").pin_memory()
+                         for k in ("tok_logprob", "cand_score", "q_cand", "choice", "value")})
     step.run_pipelined(batches, w_lm, outs)
     torch.cuda.synchronize()
     assert cuda.jet_device_status() == 0
