@@ -27,8 +27,8 @@ What each function computes, and where the paper defines it:
 * :func:`prefill_state` - the prefix recurrent state: the prefix tokens fed
   through the recurrence in order, the state every candidate forks from.
 * :func:`fork_state` - every candidate continues an unmodified copy of the
-  prefix recurrent state (Sec. 4.1, "Hybrid models ... restoring the unchanged
-  prefix state before each candidate"; Sec. 5.6). The recurrence itself is not
+  prefix recurrent state (Sec. 4.1: for hybrid models the paper puts the prefix
+  state back, unchanged, before each candidate; Sec. 5.6). The recurrence itself is not
   given by the paper; the reading used is the gated delta rule
   S <- alpha (S - beta k (k^T S)) + beta k v^T, read out as o = S^T q / sqrt(dk).
   ``rule="gla"`` selects the plain gated linear-attention variant
