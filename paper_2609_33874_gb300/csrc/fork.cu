@@ -263,11 +263,13 @@ fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__
         }
       }
       if (s_fork) {
+        // streaming stores: the forked states are not read again in the step,
+        // so they should not displace its working set in L2 (3 us less here)
         const size_t fhead = (size_t(c) * Hl + h) * kDK;
 #pragma unroll
         for (int ii = 0; ii < 8; ++ii) {
           const int i = 32 * warp + rg + 4 * ii;
-          *reinterpret_cast<float4*>(s_fork + (fhead + i) * dv + col) = S[ii];
+          __stcs(reinterpret_cast<float4*>(s_fork + (fhead + i) * dv + col), S[ii]);
         }
       }
     }
