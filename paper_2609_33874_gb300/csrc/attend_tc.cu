@@ -707,12 +707,18 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
           klo = max(0, fa - f0);
           khi = min(kBN, fb - f0 + 1);
         }
-        float mt = -INFINITY;
+        // the row's tile maximum through eight independent chains (one warp per
+        // scheduler runs this: a single 64-long chain would be pure latency)
+        float mq[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) mq[q] = -INFINITY;
 #pragma unroll
         for (int c = 0; c < kBN; ++c) {
           sv[c] = (c >= klo && c < khi) ? sv[c] * a.scale_log2 : -INFINITY;
-          mt = fmaxf(mt, sv[c]);
+          mq[c & 7] = fmaxf(mq[c & 7], sv[c]);
         }
+        const float mt = fmaxf(fmaxf(fmaxf(mq[0], mq[1]), fmaxf(mq[2], mq[3])),
+                               fmaxf(fmaxf(mq[4], mq[5]), fmaxf(mq[6], mq[7])));
         // P buffer b was last read by the P V of tile Tj - 2
         if (Tj >= 2 && !warp_mbar_wait(p_free + b, ((Tj - 2) >> 1) & 1, kWaitNs, abort_flag)) {
           ok = false;
@@ -746,21 +752,22 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         // P = 2^(s - m_used) as bf16, 128-byte swizzled; the row sum uses the
         // rounded values, which are what the tensor core multiplies
         uint8_t* pb = smem + G::kOffP + b * G::kPBytes;
-        float psum = 0.f;
+        float ps[8];  // one partial sum per 16-byte chunk, added as a tree
 #pragma unroll
         for (int cc = 0; cc < 8; ++cc) {
           uint32_t w[4];
+          ps[cc] = 0.f;
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const float x0 = ex2(sv[cc * 8 + 2 * q] - m_used);
             const float x1 = ex2(sv[cc * 8 + 2 * q + 1] - m_used);
             w[q] = pack_bf16(x0, x1);
             const __nv_bfloat162 hb = *reinterpret_cast<const __nv_bfloat162*>(&w[q]);
-            psum += __bfloat162float(hb.x) + __bfloat162float(hb.y);
+            ps[cc] += __bfloat162float(hb.x) + __bfloat162float(hb.y);
           }
           *reinterpret_cast<uint4*>(pb + sw128(i, cc)) = make_uint4(w[0], w[1], w[2], w[3]);
         }
-        l += psum;
+        l += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
         fence_proxy_async_smem();
         tc_fence_before();
         __syncwarp();
