@@ -194,7 +194,8 @@ fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__
   {
     float4 sp[8];
     const size_t head = (size_t(r) * Hl + h) * kDK;
-    if (q_rows && tid < kDK) qsh[tid] = to_f32(q_rows[(size_t(row_offset[r]) * Hl + h) * kDK + tid]);
+    if (q_rows && tid < kDK)
+      qsh[tid] = to_f32(q_rows[(size_t(row_offset[r]) * Hl + h) * kDK + tid]);
 #pragma unroll
     for (int ii = 0; ii < 8; ++ii) {
       const int i = 32 * warp + rg + 4 * ii;
