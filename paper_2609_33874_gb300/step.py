@@ -147,8 +147,7 @@ class ScoringStep:
             ("q_cand", torch.float32, (n.C,)), ("choice", torch.int32, (n.R,)),
             ("value", torch.float32, (n.R,))])
         self._results = z(rb, dtype=torch.uint8)
-        for k, t in _views(self._results, self._result_offsets).items():
-            setattr(self, k, t)
+        self._bind_results(self._results)
         ws = (jet.jet_workspace_bytes if lm == "bf16" else jet.jet_workspace_bytes_e4m3)(n, dims)
         self.ws = z((ws + 15) // 16 * 4)  # float32 words, 16-byte multiple
         if hybrid:
@@ -156,6 +155,19 @@ class ScoringStep:
             self.s_fork = z(n.C, dims.Hl, dims.dk, dims.dv) if keep_fork_state else None
         self._dev_inputs: Optional[Dict[str, torch.Tensor]] = None
         self.overlap_min_bytes = _OVERLAP_MIN_BYTES
+
+    def _bind_results(self, buf: torch.Tensor) -> None:
+        """Point tok_logprob, cand_score, q_cand, choice and value at ``buf``
+        (views made once per buffer: this runs once per pipelined batch)."""
+        if getattr(self, "_bound", None) is buf:
+            return
+        cache = self.__dict__.setdefault("_result_views", {})
+        views = cache.get(buf.data_ptr())
+        if views is None:
+            views = cache[buf.data_ptr()] = (buf, _views(buf, self._result_offsets))
+        for k, t in views[1].items():
+            setattr(self, k, t)
+        self._bound = buf
 
     # ------------------------------------------------------------------
     def run(self, x: Dict[str, torch.Tensor], w_lm: torch.Tensor, stream=None,
@@ -221,22 +233,31 @@ class ScoringStep:
         kernels of batch i run on ``stream``; device inputs and layouts are
         double-buffered. ``batches`` yields :class:`HostBatch` objects (one
         copy each) or (pinned host inputs, pinned layout words) pairs;
-        ``outs[i]`` receives batch i's results (device -> host, on ``stream``):
-        a :class:`HostResults` (one copy) or a dict of pinned tensors.
-        Everything is enqueued; the caller synchronises."""
+        ``outs[i]`` receives batch i's results: a :class:`HostResults` (one
+        copy, from a device buffer per pipeline slot, on a third stream, so the
+        compute stream runs batch after batch without waiting for it; the
+        step's own result tensors are then left untouched) or a dict of pinned
+        tensors (copied from the step's result tensors on ``stream``).
+        Everything is enqueued; ``stream`` ends after the last copy back, and
+        the caller synchronises."""
         s = torch.cuda.current_stream(self.dev) if stream is None else stream
         if getattr(self, "_pipe", None) is None:
             self._copy_stream = torch.cuda.Stream(self.dev)
+            self._out_stream = torch.cuda.Stream(self.dev)
             self._pipe = []
             for _ in range(2):
                 words = torch.empty_like(self.layout.words)
                 self._pipe.append(dict(
                     layout=jet.DeviceLayout(self.layout.sizes, words), inputs=None,
-                    copied=torch.cuda.Event(), consumed=torch.cuda.Event()))
-        cs = self._copy_stream
+                    copied=torch.cuda.Event(), consumed=torch.cuda.Event(),
+                    results=torch.empty_like(self._results), scored=torch.cuda.Event(),
+                    read=torch.cuda.Event()))
+        cs, os_ = self._copy_stream, self._out_stream
         start = torch.cuda.Event()
         start.record(s)
         cs.wait_event(start)  # after everything already enqueued on ``stream``
+        os_.wait_event(start)
+        own = self._results
         for i, batch in enumerate(batches):
             buf = self._pipe[i % 2]
             packed = isinstance(batch, HostBatch)
@@ -269,14 +290,34 @@ class ScoringStep:
                     buf["copied"].record(cs)
             if overlap:
                 s.wait_event(buf["copied"])
+            # a batch small enough to copy in order returns its results in order too
+            packed_out = isinstance(outs[i], HostResults) and overlap
+            if packed_out:
+                # the results of batch i go to this slot's own device buffer and
+                # back on a third stream, off the compute stream: batch i+1's
+                # kernels follow batch i's directly
+                if i >= 2:
+                    s.wait_event(buf["read"])  # batch i-2's results have left
+                self._bind_results(buf["results"])
+            else:
+                self._bind_results(own)
             self.run(inputs, w_lm, stream=s, layout=layout)
             buf["consumed"].record(s)
-            with torch.cuda.stream(s):
-                if isinstance(outs[i], HostResults):
-                    outs[i].buf.copy_(self._results, non_blocking=True)
-                else:
-                    for k in RESULTS:
-                        outs[i][k].copy_(getattr(self, k), non_blocking=True)
+            if packed_out:
+                buf["scored"].record(s)
+                os_.wait_event(buf["scored"])
+                with torch.cuda.stream(os_):
+                    outs[i].buf.copy_(buf["results"], non_blocking=True)
+                buf["read"].record(os_)
+            else:
+                with torch.cuda.stream(s):
+                    if isinstance(outs[i], HostResults):
+                        outs[i].buf.copy_(own, non_blocking=True)
+                    else:
+                        for k in RESULTS:
+                            outs[i][k].copy_(getattr(self, k), non_blocking=True)
+        self._bind_results(own)
+        s.wait_stream(os_)  # the caller's synchronisation covers the last copies
 
     def host_bytes(self, host: Dict[str, torch.Tensor], layout_words: torch.Tensor):
         """(host->device, device->host) bytes one :meth:`run_from_host` moves."""
