@@ -255,11 +255,14 @@ def _stack_launches(problem, w, spec) -> int:
     for l, kind in enumerate(spec.kinds):
         if kind == "full":
             zw, ow = (w.Hq + 2 * w.Hkv) * w.d, w.Hq * w.d
-            mixer = 1 + _attend_launches(problem, w)       # split + attention
+            # the mixer projection, split + attention
+            mixer = _proj_launches(N, zw, D) + 1 + _attend_launches(problem, w)
         else:
-            zw, ow = w.Hl * (2 * w.dk + w.dv) + 2 * w.Hl, w.Hl * w.dv
-            mixer = 2                                        # gates, fork (with the shared rows)
-        n += mixer + _proj_launches(N, zw, D) + resid(ow, True)
+            ow = w.Hl * w.dv
+            # the mixer projection, its reduce fused with the gates (or the
+            # gates after an unsplit one), the fork (with the shared rows)
+            mixer = 3
+        n += mixer + resid(ow, True)
         n += _proj_launches(N, 2 * Dff, D) + resid(Dff, l + 1 < len(spec.kinds))
     return n
 

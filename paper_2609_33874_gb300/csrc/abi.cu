@@ -517,10 +517,10 @@ extern "C" jet_status jet_stack_forward(const jet_layout* lay, const jet_dims* d
       JET_TRY(cuda_status(jet::launch_rmsnorm(x, Ly.g1, int(N), D, 1e-6f, w + plan.h, st)));
     const int zw = full ? (dims->Hq + 2 * dims->Hkv) * dims->d
                         : dims->Hl * (2 * dims->dk + dims->dv) + 2 * dims->Hl;
-    JET_TRY(cuda_status(jet::launch_proj(jet::kProjStore, w + plan.h, int(N), D, D, Ly.w_mix, zw,
-                                         w + plan.z, zw, nullptr, part, status, st)));
     int ow;
     if (full) {
+      JET_TRY(cuda_status(jet::launch_proj(jet::kProjStore, w + plan.h, int(N), D, D, Ly.w_mix,
+                                           zw, w + plan.z, zw, nullptr, part, status, st)));
       const int qw = dims->Hq * dims->d, kw = dims->Hkv * dims->d;
       JET_TRY(cuda_status(jet::launch_split_qkv(*lay, w + plan.z, qw, kw, w + plan.q, w + plan.kc,
                                                 w + plan.vc, status, st)));
@@ -532,9 +532,12 @@ extern "C" jet_status jet_stack_forward(const jet_layout* lay, const jet_dims* d
     } else {
       float* al = reinterpret_cast<float*>(w + plan.al);
       float* be = reinterpret_cast<float*>(w + plan.be);
-      JET_TRY(cuda_status(jet::launch_gates(*lay, w + plan.z, dims->Hl, dims->dv, w + plan.lqa,
-                                            w + plan.lqf, w + plan.lk, w + plan.lv, al, be,
-                                            status, st)));
+      // the mixer projection and the gates (q, normalised k, v, decay and write
+      // strength) in one pass over its partials
+      JET_TRY(cuda_status(jet::launch_proj_gates(*lay, w + plan.h, D, Ly.w_mix, zw, w + plan.z,
+                                                 dims->Hl, dims->dv, w + plan.lqa, w + plan.lqf,
+                                                 w + plan.lk, w + plan.lv, al, be, part, status,
+                                                 st)));
       // fed rows through the fork, shared rows from the prefix states: all N
       // rows of the mixer output
       JET_TRY(cuda_status(jet::launch_fork_state(*lay, *dims, stack->rule, Ly.s_prefix,

@@ -117,6 +117,16 @@ cudaError_t launch_proj(int epi, const void* x, int N, int K, int ldx, const voi
                         cudaStream_t st, const void* norm_g = nullptr, float norm_eps = 0.f,
                         void* norm_h = nullptr);
 size_t proj_partial_bytes(int N, int O, int K);
+// a linear layer's mixer projection z = x w^T (O = Hl (2 dk + dv) + 2 Hl) and
+// its gates (launch_gates) in one go: with a K split the partials are reduced
+// straight into the gates' outputs, without z
+cudaError_t launch_proj_gates(const jet_layout& lay, const void* x, int K, const void* w, int O,
+                              void* z, int Hl, int dv, void* lq_all, void* lq, void* lk, void* lv,
+                              float* alpha, float* beta, float* part, int* status,
+                              cudaStream_t st);
+cudaError_t launch_reduce_gates(const jet_layout& lay, const float* part, int splits, int Hl,
+                                int dv, void* lq_all, void* lq, void* lk, void* lv,
+                                float* alpha, float* beta, int* status, cudaStream_t st);
 cudaError_t launch_rmsnorm(const void* x, const void* g, int N, int D, float eps, void* h,
                            cudaStream_t st);
 cudaError_t launch_split_qkv(const jet_layout& lay, const void* z, int qw, int kw, void* q,

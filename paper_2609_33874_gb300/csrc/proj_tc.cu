@@ -469,7 +469,7 @@ Tiling tiling(int N, int O, int K, bool split) {
 template <int EPI>
 cudaError_t launch_epi(const void* x, int N, int K, int ldx, const void* w, int O, void* out,
                        int ldo, const void* res, float* part, int* status, cudaStream_t st,
-                       const Norm& nm) {
+                       const Norm& nm, int* splits_out = nullptr) {
   const Tiling tl = tiling(N, O, K, part != nullptr);
   const int n_tt = tl.n_tt, Nt = tl.Nt;
   ProjArgs a{};
@@ -502,6 +502,11 @@ cudaError_t launch_epi(const void* x, int N, int K, int ldx, const void* w, int 
   const int grid = std::max(1, std::min(a.units, sm_count()));
   e = launch_pdl(proj_tc_kernel<EPI>, dim3(grid), dim3(kThreads), smem, st, tmW, tmX, a);
   if (e != cudaSuccess) return e;
+  if (splits_out) {
+    // the caller reduces the partials itself
+    *splits_out = a.splits;
+    if (a.splits > 1) return cudaSuccess;
+  }
   const bool norm = EPI == kProjResid && nm.h != nullptr;
   if (norm && a.splits > 1 && ldo == O && O % 8 == 0)
     return launch_pdl(proj_reduce_norm_kernel, dim3(unsigned(N)), dim3(kNormThreads), 0, st,
@@ -527,6 +532,22 @@ cudaError_t launch_reduce(const ProjArgs& a, float* part, int N, int O, void* ou
 }
 
 }  // namespace
+
+cudaError_t launch_proj_gates(const jet_layout& lay, const void* x, int K, const void* w, int O,
+                              void* z, int Hl, int dv, void* lq_all, void* lq, void* lk, void* lv,
+                              float* alpha, float* beta, float* part, int* status,
+                              cudaStream_t st) {
+  const int N = lay.n.N;
+  if (N <= 0 || O <= 0) return cudaSuccess;
+  int splits = 1;
+  cudaError_t e = launch_epi<kProjStore>(x, N, K, K, w, O, z, O, nullptr, part, status, st,
+                                         Norm{nullptr, 0.f, nullptr}, &splits);
+  if (e != cudaSuccess) return e;
+  if (splits > 1)
+    return launch_reduce_gates(lay, part, splits, Hl, dv, lq_all, lq, lk, lv, alpha, beta, status,
+                               st);
+  return launch_gates(lay, z, Hl, dv, lq_all, lq, lk, lv, alpha, beta, status, st);
+}
 
 size_t proj_partial_bytes(int N, int O, int K) {
   const Tiling t = tiling(N, O, K, true);

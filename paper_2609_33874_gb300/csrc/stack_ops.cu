@@ -151,7 +151,90 @@ gates_kernel(const __nv_bfloat16* __restrict__ z, const int32_t* row_req,
   }
 }
 
+// The linear layer's mixer projection, split over K, reduced straight into
+// the gates: one warp per (row, head) sums its q, k, v and gate columns of the
+// f32 partials part[splits][N][zw] in split order, rounds each to bf16 as a
+// stored z would be, then does what gates_kernel does with z (the same
+// results without the z round trip and its reduce pass).
+__global__ void __launch_bounds__(256)
+reduce_gates_kernel(const float* __restrict__ part, int splits, const int32_t* row_req,
+                    const int32_t* row_cand, int N, int R, int Hl, int dv,
+                    __nv_bfloat16* __restrict__ lq_all, __nv_bfloat16* __restrict__ lq,
+                    __nv_bfloat16* __restrict__ lk, __nv_bfloat16* __restrict__ lv,
+                    float* __restrict__ alpha, float* __restrict__ beta, int* status) {
+  pdl_begin();
+  constexpr int dk = 128;
+  const int lane = threadIdx.x & 31;
+  const int wid = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (wid >= N * Hl) return;
+  const int n = wid / Hl, hh = wid % Hl;
+  const int zw = Hl * (2 * dk + dv) + 2 * Hl;
+  // four consecutive columns summed over the splits, rounded to bf16
+  auto sum4 = [&](int col) {
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+    for (int sp = 0; sp < splits; ++sp) {
+      const float4 x = *reinterpret_cast<const float4*>(part + (size_t(sp) * N + n) * zw + col);
+      acc.x += x.x; acc.y += x.y; acc.z += x.z; acc.w += x.w;
+    }
+    uint2 r;
+    *reinterpret_cast<__nv_bfloat162*>(&r.x) = __floats2bfloat162_rn(acc.x, acc.y);
+    *reinterpret_cast<__nv_bfloat162*>(&r.y) = __floats2bfloat162_rn(acc.z, acc.w);
+    return r;
+  };
+  auto sum1 = [&](int col) {
+    float acc = 0.f;
+    for (int sp = 0; sp < splits; ++sp) acc += part[(size_t(sp) * N + n) * zw + col];
+    return __float2bfloat16_rn(acc);
+  };
+  const uint2 qv = sum4(hh * dk + 4 * lane);
+  *reinterpret_cast<uint2*>(lq_all + (size_t(n) * Hl + hh) * dk + 4 * lane) = qv;
+  const int r = row_req[n];
+  if (r < 0 || r >= R) {
+    if (lane == 0) flag(status, JET_ERR_DEVICE);
+    return;
+  }
+  if (row_cand[n] < 0) return;  // the shared row only reads the prefix state
+  const int f = n - r - 1;
+  if (f < 0 || f >= N - R) {
+    if (lane == 0) flag(status, JET_ERR_DEVICE);
+    return;
+  }
+  *reinterpret_cast<uint2*>(lq + (size_t(f) * Hl + hh) * dk + 4 * lane) = qv;
+  const uint2 kv = sum4(Hl * dk + hh * dk + 4 * lane);
+  const float2 k01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kv.x));
+  const float2 k23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kv.y));
+  float ss = k01.x * k01.x + k01.y * k01.y + k23.x * k23.x + k23.y * k23.y;
+  ss = warp_sum(ss);
+  const float inv = ss > 0.f ? 1.f / sqrtf(ss) : 0.f;
+  uint2 kn;
+  *reinterpret_cast<__nv_bfloat162*>(&kn.x) = __floats2bfloat162_rn(k01.x * inv, k01.y * inv);
+  *reinterpret_cast<__nv_bfloat162*>(&kn.y) = __floats2bfloat162_rn(k23.x * inv, k23.y * inv);
+  *reinterpret_cast<uint2*>(lk + (size_t(f) * Hl + hh) * dk + 4 * lane) = kn;
+  __nv_bfloat16* vdst = lv + (size_t(f) * Hl + hh) * dv;
+  for (int j = lane; j < dv; j += 32) vdst[j] = sum1(2 * Hl * dk + hh * dv + j);
+  if (lane == 0) {
+    const float a = __bfloat162float(sum1(Hl * (2 * dk + dv) + hh));
+    const float b = __bfloat162float(sum1(Hl * (2 * dk + dv) + Hl + hh));
+    alpha[size_t(f) * Hl + hh] = 1.f / (1.f + expf(-a));
+    beta[size_t(f) * Hl + hh] = 1.f / (1.f + expf(-b));
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_reduce_gates(const jet_layout& lay, const float* part, int splits, int Hl,
+                                int dv, void* lq_all, void* lq, void* lk, void* lv,
+                                float* alpha, float* beta, int* status, cudaStream_t st) {
+  const jet_sizes& n = lay.n;
+  if (n.N <= 0) return cudaSuccess;
+  const int warps = n.N * Hl;
+  return launch_pdl(reduce_gates_kernel, dim3(unsigned((warps + 7) / 8)), dim3(256), 0, st, part,
+                    splits, lay.row_req, lay.row_cand, n.N, n.R, Hl, dv,
+                    static_cast<__nv_bfloat16*>(lq_all), static_cast<__nv_bfloat16*>(lq),
+                    static_cast<__nv_bfloat16*>(lk), static_cast<__nv_bfloat16*>(lv), alpha, beta,
+                    status);
+}
 
 cudaError_t launch_rmsnorm(const void* x, const void* g, int N, int D, float eps, void* h,
                            cudaStream_t st) {
