@@ -254,9 +254,10 @@ def _stack_launches(problem, w, spec) -> int:
     n = 1 if spec.kinds else 0                               # the first layer's RMSNorm
     for l, kind in enumerate(spec.kinds):
         if kind == "full":
-            zw, ow = (w.Hq + 2 * w.Hkv) * w.d, w.Hq * w.d
-            # the mixer projection, split + attention
-            mixer = _proj_launches(N, zw, D) + 1 + _attend_launches(problem, w)
+            ow = w.Hq * w.d
+            # the q/k/v projection, its reduce fused with the split (or the split
+            # after an unsplit one), the attention
+            mixer = 2 + _attend_launches(problem, w)
         else:
             ow = w.Hl * w.dv
             # the mixer projection, its reduce fused with the gates (or the

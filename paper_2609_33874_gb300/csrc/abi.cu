@@ -519,11 +519,12 @@ extern "C" jet_status jet_stack_forward(const jet_layout* lay, const jet_dims* d
                         : dims->Hl * (2 * dims->dk + dims->dv) + 2 * dims->Hl;
     int ow;
     if (full) {
-      JET_TRY(cuda_status(jet::launch_proj(jet::kProjStore, w + plan.h, int(N), D, D, Ly.w_mix,
-                                           zw, w + plan.z, zw, nullptr, part, status, st)));
+      // the q/k/v projection and its split into the step's query and candidate
+      // key/value buffers in one pass over its partials
       const int qw = dims->Hq * dims->d, kw = dims->Hkv * dims->d;
-      JET_TRY(cuda_status(jet::launch_split_qkv(*lay, w + plan.z, qw, kw, w + plan.q, w + plan.kc,
-                                                w + plan.vc, status, st)));
+      JET_TRY(cuda_status(jet::launch_proj_qkv(*lay, w + plan.h, D, Ly.w_mix, qw, kw, w + plan.z,
+                                               w + plan.q, w + plan.kc, w + plan.vc, part, status,
+                                               st)));
       JET_TRY(cuda_status(jet::launch_prefix_attend(*lay, *dims, plan.attn_plan, w + plan.q,
                                                     Ly.k_pre, Ly.v_pre, w + plan.kc,
                                                     w + plan.vc, w + plan.o, w + plan.attn,

@@ -124,6 +124,13 @@ cudaError_t launch_proj_gates(const jet_layout& lay, const void* x, int K, const
                               void* z, int Hl, int dv, void* lq_all, void* lq, void* lk, void* lv,
                               float* alpha, float* beta, float* part, int* status,
                               cudaStream_t st);
+// a full-attention layer's q/k/v projection (O = qw + 2 kw) and its split into q
+// and the fed rows' k and v (launch_split_qkv) in one go, likewise
+cudaError_t launch_proj_qkv(const jet_layout& lay, const void* x, int K, const void* w, int qw,
+                            int kw, void* z, void* q, void* kc, void* vc, float* part,
+                            int* status, cudaStream_t st);
+cudaError_t launch_reduce_qkv(const jet_layout& lay, const float* part, int splits, int qw,
+                              int kw, void* q, void* kc, void* vc, int* status, cudaStream_t st);
 cudaError_t launch_reduce_gates(const jet_layout& lay, const float* part, int splits, int Hl,
                                 int dv, void* lq_all, void* lq, void* lk, void* lv,
                                 float* alpha, float* beta, int* status, cudaStream_t st);

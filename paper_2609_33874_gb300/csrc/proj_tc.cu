@@ -549,6 +549,19 @@ cudaError_t launch_proj_gates(const jet_layout& lay, const void* x, int K, const
   return launch_gates(lay, z, Hl, dv, lq_all, lq, lk, lv, alpha, beta, status, st);
 }
 
+cudaError_t launch_proj_qkv(const jet_layout& lay, const void* x, int K, const void* w, int qw,
+                            int kw, void* z, void* q, void* kc, void* vc, float* part,
+                            int* status, cudaStream_t st) {
+  const int N = lay.n.N, O = qw + 2 * kw;
+  if (N <= 0 || O <= 0) return cudaSuccess;
+  int splits = 1;
+  cudaError_t e = launch_epi<kProjStore>(x, N, K, K, w, O, z, O, nullptr, part, status, st,
+                                         Norm{nullptr, 0.f, nullptr}, &splits);
+  if (e != cudaSuccess) return e;
+  if (splits > 1) return launch_reduce_qkv(lay, part, splits, qw, kw, q, kc, vc, status, st);
+  return launch_split_qkv(lay, z, qw, kw, q, kc, vc, status, st);
+}
+
 size_t proj_partial_bytes(int N, int O, int K) {
   const Tiling t = tiling(N, O, K, true);
   return t.splits > 1 ? size_t(t.splits) * N * O * sizeof(float) : 0;

@@ -151,6 +151,57 @@ gates_kernel(const __nv_bfloat16* __restrict__ z, const int32_t* row_req,
   }
 }
 
+// The full-attention layer's q/k/v projection, split over K, reduced straight
+// into q (every row) and the fed rows' k and v: one 512-thread block per row,
+// 8 columns a thread at a time, each summed over the partials
+// part[splits][N][qw + 2 kw] in split order and rounded to bf16 as a stored z
+// would be (the same results as the reduce and split_qkv_kernel).
+__global__ void __launch_bounds__(512)
+reduce_qkv_kernel(const float* __restrict__ part, int splits, const int32_t* row_req,
+                  const int32_t* row_cand, int N, int R, int qw, int kw,
+                  __nv_bfloat16* __restrict__ q, __nv_bfloat16* __restrict__ kc,
+                  __nv_bfloat16* __restrict__ vc, int* status) {
+  pdl_begin();
+  const int n = blockIdx.x;
+  if (n >= N) return;
+  const int r = row_req[n];
+  if (r < 0 || r >= R) {
+    if (threadIdx.x == 0) flag(status, JET_ERR_DEVICE);
+    return;
+  }
+  const bool fed = row_cand[n] >= 0;  // a shared row's key and value are the prefix's
+  const int f = n - r - 1;
+  if (fed && (f < 0 || f >= N - R)) {
+    if (threadIdx.x == 0) flag(status, JET_ERR_DEVICE);
+    return;
+  }
+  const int zw = qw + 2 * kw;
+  const int pieces = fed ? zw / 8 : qw / 8;
+  for (int e = threadIdx.x; e < pieces; e += blockDim.x) {
+    float acc[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc[i] = 0.f;
+#pragma unroll 4
+    for (int sp = 0; sp < splits; ++sp) {
+      const float4* pp = reinterpret_cast<const float4*>(part + (size_t(sp) * N + n) * zw + 8 * e);
+      const float4 a0 = pp[0], a1 = pp[1];
+      acc[0] += a0.x; acc[1] += a0.y; acc[2] += a0.z; acc[3] += a0.w;
+      acc[4] += a1.x; acc[5] += a1.y; acc[6] += a1.z; acc[7] += a1.w;
+    }
+    uint4 o;
+    __nv_bfloat162* po = reinterpret_cast<__nv_bfloat162*>(&o);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) po[i] = __floats2bfloat162_rn(acc[2 * i], acc[2 * i + 1]);
+    const int c = 8 * e;
+    if (c < qw)
+      *reinterpret_cast<uint4*>(q + size_t(n) * qw + c) = o;
+    else if (c < qw + kw)
+      *reinterpret_cast<uint4*>(kc + size_t(f) * kw + (c - qw)) = o;
+    else
+      *reinterpret_cast<uint4*>(vc + size_t(f) * kw + (c - qw - kw)) = o;
+  }
+}
+
 // The linear layer's mixer projection, split over K, reduced straight into
 // the gates: one warp per (row, head) sums its q, k, v and gate columns of the
 // f32 partials part[splits][N][zw] in split order, rounds each to bf16 as a
@@ -222,6 +273,15 @@ reduce_gates_kernel(const float* __restrict__ part, int splits, const int32_t* r
 }
 
 }  // namespace
+
+cudaError_t launch_reduce_qkv(const jet_layout& lay, const float* part, int splits, int qw,
+                              int kw, void* q, void* kc, void* vc, int* status, cudaStream_t st) {
+  const jet_sizes& n = lay.n;
+  if (n.N <= 0) return cudaSuccess;
+  return launch_pdl(reduce_qkv_kernel, dim3(unsigned(n.N)), dim3(512), 0, st, part, splits,
+                    lay.row_req, lay.row_cand, n.N, n.R, qw, kw, static_cast<__nv_bfloat16*>(q),
+                    static_cast<__nv_bfloat16*>(kc), static_cast<__nv_bfloat16*>(vc), status);
+}
 
 cudaError_t launch_reduce_gates(const jet_layout& lay, const float* part, int splits, int Hl,
                                 int dv, void* lq_all, void* lq, void* lk, void* lv,
