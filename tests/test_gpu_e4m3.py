@@ -105,6 +105,7 @@ E4M3_CASES = [
     (dict(V=1000, D=96), [4, 9], [3, 2], [1, 4, 2, 6, 3]),           # V % 128 != 0
     (dict(V=129, D=64), [2], [5], [1, 1, 2, 1, 40]),                 # one vocabulary tail row
     (dict(V=20000, D=256, w_std=0.05), [3] * 7, [4] * 7, [3] * 28),
+    (dict(V=1100, D=96), [5] * 4, [6] * 4, [4] * 24),                # odd tile count, ragged last tile
     (dict(V=5000, D=208), [2] * 3, [10] * 3, [10] * 30),             # two token tiles; D % 128 != 0
     (dict(V=1025, D=128), [2] * 6, [10] * 6, [11] * 60),             # three token tiles
 ]

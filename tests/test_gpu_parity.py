@@ -104,6 +104,10 @@ LM_CASES = [
     # three token tiles, vocabulary tail of one row
     (dict(V=1025, D=128, dtype="bf16"), [2] * 6, [10] * 6, [11] * 60),
     (dict(V=4096, D=64, dtype="bf16"), [2], [1], [1]),                  # a single row
+    # an odd number of vocabulary tiles, the last one ragged
+    (dict(V=1100, D=96, dtype="bf16"), [5] * 4, [6] * 4, [4] * 24),
+    # exactly 256 rows: the largest single token tile (512 TMEM columns)
+    (dict(V=3000, D=128, dtype="bf16"), [3] * 4, [21] * 4, [4] * 84),
 ]
 
 
