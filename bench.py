@@ -145,6 +145,23 @@ def oracle_step(problem):
     return O.score_step(lay, problem.f32("hidden"), problem.f32("w_lm"), mode)
 
 
+def step_config(args, problem, world: int) -> dict:
+    """The `config` of the step's JSON line (both arms): the workload and its sizes."""
+    w = problem.work
+    es = 2 if w.dtype == "bf16" else 4
+    return dict(workload=args.workload, R=problem.R, N=problem.N, T=len(problem.target_ids),
+                C=len(problem.cand_len), total_prefix=problem.total_prefix, Hq=w.Hq, Hkv=w.Hkv,
+                d=w.d, D=w.D, V=w.V, Hl=w.Hl,
+                parallelism=f"replicas{world}" if world > 1 else "single",
+                lm_head={"bf16": "bf16",
+                         "e4m3": "e4m3, one float32 scale per weight row and per token",
+                         "w4": "weights e2m1 with a power-of-two exponent per 32-element "
+                               "block and a float32 scale per row; hidden e4m3 per token"}[args.lm],
+                recurrence=(args.rule if w.Hl else None),
+                l2=f"inputs larger than L2: LM-head weights {w.V * w.D * es / 1e9:.2f} GB "
+                   f"streamed every step")
+
+
 def oracle_sample(name: str, R: int, k: int):
     import jet_synth
     p = jet_synth.make_problem(name, R=min(k, R))
@@ -508,17 +525,7 @@ def run_gpu(args):
         scaling="weak", vs_baseline=None,
         dtype=(f"bf16 (LM head {args.lm})" if low else "bf16") if w.dtype == "bf16" else "f32",
         data="synthetic",
-        config=dict(workload=args.workload, R=R, N=N, T=T, C=len(problem.cand_len),
-                    total_prefix=problem.total_prefix, Hq=w.Hq, Hkv=w.Hkv, d=w.d, D=w.D, V=w.V,
-                    Hl=w.Hl, parallelism=f"replicas{world}" if world > 1 else "single",
-                    lm_head={"bf16": "bf16",
-                             "e4m3": "e4m3, one float32 scale per weight row and per token",
-                             "w4": "weights e2m1 with a power-of-two exponent per 32-element "
-                                   "block and a float32 scale per row; hidden e4m3 per token"}[
-                                       args.lm],
-                    recurrence=(args.rule if w.Hl else None),
-                    l2=f"inputs larger than L2: LM-head weights {w.V * w.D * es / 1e9:.2f} GB "
-                       f"streamed every step"),
+        config=step_config(args, problem, world),
         clocks=clk,
         e2e=dict(value=round(e2e_value, 2), unit=UNIT, h2d_bytes_per_step=h2d,
                  d2h_bytes_per_step=d2h, ms_per_step=round(e2e_ms, 4)),
@@ -750,7 +757,7 @@ def run_reference(args):
         impl="reference", metric=METRIC, value=round(value, 4), unit=UNIT, n_gpus=world,
         steps=args.steps, warmup=args.warmup, ms_per_step=round(dt * 1e3, 2),
         higher_is_better=True, scaling="weak", vs_baseline=None, dtype="f64", data="synthetic",
-        config=dict(workload=args.workload, R=R),
+        config=step_config(args, jet_synth.make_problem(w, R=R), world),
         cpu_baseline=dict(value=round(value, 4), unit=UNIT, cores=_CORES, kind="oracle",
                           sample=desc),
         e2e=dict(value=round(value, 4), unit=UNIT, h2d_bytes_per_step=0, d2h_bytes_per_step=0),
