@@ -312,6 +312,70 @@ def test_end_to_end_pipelined(cuda, overlap, packed):
 
 
 # ---------------------------------------------------------------------------
+# candidate isolation on the GPU (Sec. 4.1): a candidate's log-probabilities
+# do not depend on which other candidates share its batch or in what order
+# ---------------------------------------------------------------------------
+def _row_map(n_cand, cand_len):
+    """Per request its shared row, per candidate its fed rows, per candidate
+    its targets (row and target order of the teacher-forced layout)."""
+    shared, fed, tgts = [], [], []
+    row = tgt = c = 0
+    for nc in n_cand:
+        shared.append(row)
+        row += 1
+        for _ in range(nc):
+            m = int(cand_len[c])
+            fed.append(list(range(row, row + m - 1)))
+            tgts.append(list(range(tgt, tgt + m)))
+            row += m - 1
+            tgt += m
+            c += 1
+    return shared, fed, tgts
+
+
+def test_candidates_are_isolated(cuda):
+    import torch
+    n_cand, cand_len = [4, 3], [3, 1, 4, 2, 2, 5, 1]
+    p = _custom("tiny", [40, 33], n_cand, cand_len, seed=51, V=3000, D=128, dtype="bf16")
+    step, x, w_lm = build_step(cuda, p)
+    step.run(x, w_lm)
+    torch.cuda.synchronize()
+    ell0, s0 = step.tok_logprob.cpu().numpy(), step.cand_score.cpu().numpy()
+    o0 = step.o.float().cpu().numpy()
+    # request 0's candidates reordered, request 1's second candidate removed
+    keep = [3, 0, 2, 1, 4, 6]
+    n_new = [4, 2]
+    shared, fed, tgts = _row_map(n_cand, cand_len)
+    ids = np.asarray(p.target_ids)
+    q = _custom("tiny", [40, 33], n_new, [cand_len[c] for c in keep], seed=51, V=3000, D=128,
+                dtype="bf16")
+    q.target_ids[:] = np.concatenate([ids[tgts[c]] for c in keep])
+    rows = [shared[0]] + sum((fed[c] for c in keep[:4]), []) + [shared[1]] + \
+        sum((fed[c] for c in keep[4:]), [])
+    R = len(n_cand)
+    req_of = np.repeat(np.arange(R), [1 + sum(cand_len[c] - 1 for c in range(sum(n_cand[:r]),
+                                                  sum(n_cand[:r + 1]))) for r in range(R)])
+    fed_rows = [r for r in rows if r not in shared]
+    fed_idx = torch.tensor([r - int(req_of[r]) - 1 for r in fed_rows], dtype=torch.long)
+    step2, _, _ = build_step(cuda, q)
+    sel = torch.tensor(rows, dtype=torch.long)
+    x2 = dict(x)
+    x2["q"] = x["q"][sel.to(x["q"].device)].contiguous()
+    x2["hidden"] = x["hidden"][sel.to(x["hidden"].device)].contiguous()
+    for k in ("k_cand", "v_cand"):
+        x2[k] = x[k][fed_idx.to(x[k].device)].contiguous()
+    step2.run(x2, w_lm)
+    torch.cuda.synchronize()
+    assert cuda.jet_device_status() == 0
+    ell1, s1 = step2.tok_logprob.cpu().numpy(), step2.cand_score.cpu().numpy()
+    np.testing.assert_allclose(s1, s0[keep], rtol=0, atol=1e-5)
+    np.testing.assert_allclose(ell1, np.concatenate([ell0[tgts[c]] for c in keep]), rtol=0,
+                               atol=1e-5)
+    # the attention rows too: each row sees the prefix and its own candidate only
+    np.testing.assert_allclose(step2.o.float().cpu().numpy(), o0[rows], rtol=0, atol=1e-2)
+
+
+# ---------------------------------------------------------------------------
 # evaluation helpers: gold NLL over equivalent labels, agreement
 # ---------------------------------------------------------------------------
 def test_evaluate_against_oracle(cuda):
