@@ -522,6 +522,39 @@ jet_status jet_decide(const jet_layout* lay, int32_t mode, const float* cand_sco
  */
 jet_status jet_device_status(void* stream, jet_status* out);
 
+/*
+ * jet_set_wait_budget_ns - budget of one bounded wait inside the tensor-core
+ * kernels (the attention, LM-head and projection kernels poll mbarriers
+ * between their roles). A wait that runs past it gives up: the kernel stops
+ * issuing work, lets the copies and tensor-core operations it already issued
+ * finish, frees its tensor memory, returns, and the next jet_device_status
+ * reports JET_ERR_TIMEOUT. 0 restores the default of 2 s. The value is read
+ * when an entry point launches a kernel, so it applies to later calls only;
+ * it is process-wide (all devices and threads). A short budget is how a
+ * caller (or a test) checks the timeout path without a stalled GPU.
+ * Returns the budget that was in force before the call.
+ */
+uint64_t jet_set_wait_budget_ns(uint64_t ns);
+
+/*
+ * jet_set_test_stall - test hook for the timeout path. While `on` is nonzero,
+ * every tensor-core kernel launched afterwards withholds its first load (the
+ * LM head and the projections their first operand stage, the attention its
+ * first query block), so that the role waiting for it waits for something
+ * nothing will provide: that wait runs out its budget (jet_set_wait_budget_ns)
+ * and the kernel ends as described there, reporting JET_ERR_TIMEOUT. Results
+ * of such calls are meaningless. Process-wide, read at launch; returns the
+ * previous setting. Off unless set.
+ */
+int32_t jet_set_test_stall(int32_t on);
+
+/*
+ * jet_launch_count - kernels this library has launched in this process so
+ * far (every successful launch by any entry point, on any device or thread).
+ * The difference across a region is the number of kernels it launched.
+ */
+uint64_t jet_launch_count(void);
+
 #ifdef __cplusplus
 }
 #endif

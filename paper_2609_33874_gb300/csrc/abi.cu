@@ -3,6 +3,7 @@
 // stream (except jet_device_status) or launches anything after a failed
 // check.
 #include <algorithm>
+#include <atomic>
 #include <cstdint>
 #include <mutex>
 
@@ -15,6 +16,19 @@ namespace jet {
 // Per-device status word written by kernels that meet an out-of-range layout
 // index or give up a bounded wait.
 __device__ int g_status_word;
+
+namespace {
+constexpr uint64_t kDefaultWaitNs = 2000000000ull;
+std::atomic<uint64_t> g_wait_ns{kDefaultWaitNs};
+std::atomic<uint64_t> g_launches{0};
+std::atomic<int> g_test_stall{0};
+}  // namespace
+
+uint64_t wait_budget_ns() { return g_wait_ns.load(std::memory_order_relaxed); }
+
+int test_stall() { return g_test_stall.load(std::memory_order_relaxed); }
+
+void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 int* device_status_ptr() {
   int dev = 0;
@@ -606,3 +620,11 @@ extern "C" jet_status jet_device_status(void* stream, jet_status* out) {
   *out = v;
   return JET_OK;
 }
+
+extern "C" uint64_t jet_set_wait_budget_ns(uint64_t ns) {
+  return jet::g_wait_ns.exchange(ns ? ns : jet::kDefaultWaitNs);
+}
+
+extern "C" uint64_t jet_launch_count(void) { return jet::g_launches.load(); }
+
+extern "C" int32_t jet_set_test_stall(int32_t on) { return jet::g_test_stall.exchange(on ? 1 : 0); }

@@ -42,7 +42,6 @@ constexpr int kBN = 64;       // keys per tile
 constexpr int kStages = 2;
 constexpr int kThreads = 224;
 constexpr int kSchedWarp = 6;  // the work-item scheduler
-constexpr uint64_t kWaitNs = 2000000000ull;
 constexpr uint64_t kDrainNs = 200000000ull;
 constexpr float kRescaleLog2 = 8.f;  // rescale O only when the max grows by > 2^8
 
@@ -83,6 +82,8 @@ struct AttArgs {
   int has_cand;      // the batch has fed candidate tokens (F > 0)
   int prefill;       // 1: causal self-attention over the prefixes (rows = prefix positions)
   float scale_log2;  // log2(e) / sqrt(d)
+  uint64_t wait_ns;  // budget of one bounded wait (jet_set_wait_budget_ns)
+  int hold_first;    // test hook (jet_set_test_stall): withhold the first query block
 };
 
 // SW128 K-major position of 16-byte chunk c of row i inside one 64-wide slice
@@ -407,7 +408,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       const int count = a.sorted ? *a.item_count : 0;
       for (int u = 0;; ++u) {
         const int slot = u & 1;
-        if (!mbar_wait(item_empty + slot, ((u >> 1) & 1) ^ 1u, kWaitNs, abort_flag)) {
+        if (!mbar_wait(item_empty + slot, ((u >> 1) & 1) ^ 1u, a.wait_ns, abort_flag)) {
           *abort_flag = 1;
           flag(a.status, JET_ERR_TIMEOUT);
           break;
@@ -464,7 +465,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       bool ok = true;
       for (int u = 0; ok; ++u) {
         const int slot = u & 1;
-        if (!mbar_wait(item_full + slot, (u >> 1) & 1, kWaitNs, abort_flag)) {
+        if (!mbar_wait(item_full + slot, (u >> 1) & 1, a.wait_ns, abort_flag)) {
           ok = false;
           break;
         }
@@ -472,17 +473,21 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         const ItemGeo e = ring[slot].e;
         // the query block: rb rows x g heads x d of the group, once the last
         // QK^T of the previous item has read the old one
-        if (v >= 1 && !mbar_wait(q_free, (v - 1) & 1, kWaitNs, abort_flag)) {
+        if (v >= 1 && !mbar_wait(q_free, (v - 1) & 1, a.wait_ns, abort_flag)) {
           ok = false;
           break;
         }
-        mbar_arrive_expect_tx(q_full, uint32_t(G::kSlices) * 64 * 2 * g * rb);
+        if (v == 0 && a.hold_first) {
+          // test hook: the first query block never lands
+        } else {
+          mbar_arrive_expect_tx(q_full, uint32_t(G::kSlices) * 64 * 2 * g * rb);
 #pragma unroll
-        for (int sl = 0; sl < G::kSlices; ++sl)
-          tma_load_3d(smem + sl * (kBV * 128), &tmQ, q_full, sl * 64, e.kh * g, e.n0 + e.row0,
-                      pol);
-        q_issued = 1;
-        q_par = v & 1;
+          for (int sl = 0; sl < G::kSlices; ++sl)
+            tma_load_3d(smem + sl * (kBV * 128), &tmQ, q_full, sl * 64, e.kh * g, e.n0 + e.row0,
+                        pol);
+          q_issued = 1;
+          q_par = v & 1;
+        }
         // K_j and V_j are issued as soon as their slots drain, whichever first
         int jk = 0, jv = 0;
         IdleClock clk;
@@ -526,7 +531,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
               progressed = true;
             }
           }
-          if (clk.expired(progressed, abort_flag, kWaitNs)) {
+          if (clk.expired(progressed, abort_flag, a.wait_ns)) {
             ok = false;
             break;
           }
@@ -554,17 +559,17 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       const uint32_t id_s = idesc_bf16_f32(kBV, kBN);
       const uint32_t id_o = idesc_bf16_f32(kBV, DH) | (1u << 16);  // B (V) is MN-major
       const uint32_t qs = smem_u32(smem);
-      bool ok = mbar_wait(qz_done, 0, kWaitNs, abort_flag);
+      bool ok = mbar_wait(qz_done, 0, a.wait_ns, abort_flag);
       int T = 0, v = 0;  // tiles and items processed so far
       for (int u = 0; ok; ++u) {
         const int slot = u & 1;
-        if (!mbar_wait(item_full + slot, (u >> 1) & 1, kWaitNs, abort_flag)) {
+        if (!mbar_wait(item_full + slot, (u >> 1) & 1, a.wait_ns, abort_flag)) {
           ok = false;
           break;
         }
         if (ring[slot].it.x < 0) break;
         const ItemGeo e = ring[slot].e;
-        if (!mbar_wait(q_full, v & 1, kWaitNs, abort_flag)) {
+        if (!mbar_wait(q_full, v & 1, a.wait_ns, abort_flag)) {
           ok = false;
           break;
         }
@@ -615,7 +620,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
               progressed = true;
             }
           }
-          if (clk.expired(progressed, abort_flag, kWaitNs)) ok = false;
+          if (clk.expired(progressed, abort_flag, a.wait_ns)) ok = false;
         }
         if (!ok) break;
         mbar_arrive(item_empty + slot);
@@ -654,7 +659,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
     int T = 0;
     for (int u = 0; ok; ++u) {
       const int slot = u & 1;
-      if (!warp_mbar_wait(item_full + slot, (u >> 1) & 1, kWaitNs, abort_flag)) {
+      if (!warp_mbar_wait(item_full + slot, (u >> 1) & 1, a.wait_ns, abort_flag)) {
         ok = false;
         break;
       }
@@ -677,7 +682,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       for (int j = 0; j < e.ntiles; ++j) {
         const int Tj = T + j;
         const int b = Tj & 1;
-        if (!warp_mbar_wait(s_full + b, (Tj >> 1) & 1, kWaitNs, abort_flag)) {
+        if (!warp_mbar_wait(s_full + b, (Tj >> 1) & 1, a.wait_ns, abort_flag)) {
           ok = false;
           break;
         }
@@ -720,7 +725,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         const float mt = fmaxf(fmaxf(fmaxf(mq[0], mq[1]), fmaxf(mq[2], mq[3])),
                                fmaxf(fmaxf(mq[4], mq[5]), fmaxf(mq[6], mq[7])));
         // P buffer b was last read by the P V of tile Tj - 2
-        if (Tj >= 2 && !warp_mbar_wait(p_free + b, ((Tj - 2) >> 1) & 1, kWaitNs, abort_flag)) {
+        if (Tj >= 2 && !warp_mbar_wait(p_free + b, ((Tj - 2) >> 1) & 1, a.wait_ns, abort_flag)) {
           ok = false;
           break;
         }
@@ -728,7 +733,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
           const float m_new = mt;
           if (j >= 1) {
             // O holds this item's P V so far: wait for the last one, rescale in TMEM
-            if (!warp_mbar_wait(p_free + ((Tj - 1) & 1), ((Tj - 1) >> 1) & 1, kWaitNs,
+            if (!warp_mbar_wait(p_free + ((Tj - 1) & 1), ((Tj - 1) >> 1) & 1, a.wait_ns,
                                 abort_flag)) {
               ok = false;
               break;
@@ -776,7 +781,7 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       if (!ok) break;
       // wait for the item's last P V, then write its output (or its partial)
       const int Tl = T + e.ntiles - 1;
-      if (!warp_mbar_wait(p_free + (Tl & 1), (Tl >> 1) & 1, kWaitNs, abort_flag)) {
+      if (!warp_mbar_wait(p_free + (Tl & 1), (Tl >> 1) & 1, a.wait_ns, abort_flag)) {
         ok = false;
         break;
       }
@@ -965,6 +970,8 @@ cudaError_t launch_dh(const jet_layout& lay, const jet_dims& d, const AttnPlan& 
     tmVc = tmV;
   }
   AttArgs a{};
+  a.wait_ns = wait_budget_ns();
+  a.hold_first = test_stall();
   a.prefix_offset = lay.prefix_offset;
   a.row_offset = lay.row_offset;
   a.req_order = lay.req_order;
@@ -1041,6 +1048,8 @@ cudaError_t launch_prefill_dh(const jet_layout& lay, const jet_dims& d, const vo
       !encode_3d(&tmV, v, n.total_prefix, d.Hkv, DH, 1, kBN))
     return cudaErrorInvalidValue;
   AttArgs a{};
+  a.wait_ns = wait_budget_ns();
+  a.hold_first = test_stall();
   a.prefix_offset = lay.prefix_offset;
   a.row_offset = lay.row_offset;
   a.req_order = lay.req_order;

@@ -38,6 +38,18 @@ struct ScorePlan {
 };
 ScorePlan score_plan(const jet_sizes& n);
 
+// ---- host-side run settings -------------------------------------------------------
+// Budget in nanoseconds of one bounded wait inside the tensor-core kernels
+// (jet_set_wait_budget_ns; 2 s unless set), read at every launch and passed
+// to the kernel as an argument.
+uint64_t wait_budget_ns();
+// Test hook (jet_set_test_stall): nonzero makes the tensor-core kernels
+// launched afterwards withhold their first load, so that a wait nothing will
+// satisfy runs out its budget.
+int test_stall();
+// Counts one kernel launch of this library (jet_launch_count).
+void note_launch();
+
 // ---- launches ------------------------------------------------------------------
 // Stream-ordered launch with programmatic stream serialization: the kernel may
 // begin (up to its pdl_begin()) while the previous kernel of the stream ends,
@@ -55,7 +67,9 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   attr.val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kernel, args...);
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, args...);
+  if (e == cudaSuccess) note_launch();
+  return e;
 }
 
 // ---- kernel launchers (stream-ordered; return the launch error) ---------------

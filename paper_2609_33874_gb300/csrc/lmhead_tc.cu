@@ -65,7 +65,6 @@ constexpr int kW4TileRows = kW4TileBytes / 128;  // 68
 constexpr int kRawBytes = 9216;     // one w4 tile (8,704 bytes) rounded up to 1 KB
 enum { kFmtBf16 = 0, kFmtE4m3 = 1, kFmtW4 = 2 };
 constexpr int kMaxNt = 256;
-constexpr uint64_t kWaitNs = 2000000000ull;  // budget of one wait
 constexpr uint64_t kDrainNs = 200000000ull;  // budget of the drain after an abort
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kNegBig = -1.0e30f;          // logit of a vocabulary row beyond V
@@ -88,6 +87,8 @@ struct TcArgs {
   int raw_slots;         // w4: 4-bit weight tiles in flight
   int a_slots;           // w4: widened weight tiles
   uint32_t tmem_cols;
+  uint64_t wait_ns;  // budget of one bounded wait (jet_set_wait_budget_ns)
+  int hold_first;    // test hook (jet_set_test_stall): withhold the first stage's loads
 };
 
 __device__ __forceinline__ void combine(float& m, float& s, float m2, float s2) {
@@ -244,11 +245,11 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
       const uint64_t pol_w = policy_evict_first(), pol_h = policy_evict_last();
       int s = 0, sr = 0;
       uint32_t ph = 0, rph = 0, issued = 0, issued_par = 0, rissued = 0, rissued_par = 0;
-      bool ok = true;
+      bool ok = true, hold = a.hold_first != 0;
       for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
         const int vt = u / a.n_tt, t0 = (u % a.n_tt) * a.Nt;
         for (int kb = 0; kb < a.nkb; ++kb) {
-          if (!mbar_wait(raw_empty + sr, rph ^ 1u, kWaitNs, abort_flag)) {
+          if (!mbar_wait(raw_empty + sr, rph ^ 1u, a.wait_ns, abort_flag)) {
             ok = false;
             break;
           }
@@ -262,14 +263,18 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
             sr = 0;
             rph ^= 1u;
           }
-          if (!mbar_wait(empty + s, ph ^ 1u, kWaitNs, abort_flag)) {
+          if (!mbar_wait(empty + s, ph ^ 1u, a.wait_ns, abort_flag)) {
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(full + s, b_bytes);
-          tma_load_2d(smem + size_t(s) * stage_bytes, &tmH, full + s, kb * kBKe, t0, pol_h);
-          issued |= 1u << s;
-          issued_par = (issued_par & ~(1u << s)) | (ph << s);
+          if (hold) {
+            hold = false;  // test hook: this stage never fills
+          } else {
+            mbar_arrive_expect_tx(full + s, b_bytes);
+            tma_load_2d(smem + size_t(s) * stage_bytes, &tmH, full + s, kb * kBKe, t0, pol_h);
+            issued |= 1u << s;
+            issued_par = (issued_par & ~(1u << s)) | (ph << s);
+          }
           if (++s == a.stages) {
             s = 0;
             ph ^= 1u;
@@ -289,20 +294,24 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
       const uint64_t pol_w = policy_evict_first(), pol_h = policy_evict_last();
       int s = 0;
       uint32_t ph = 0, issued = 0, issued_par = 0;
-      bool ok = true;
+      bool ok = true, hold = a.hold_first != 0;
       for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
         const int v0 = (u / a.n_tt) * kBM, t0 = (u % a.n_tt) * a.Nt;
         for (int kb = 0; kb < a.nkb; ++kb) {
-          if (!mbar_wait(empty + s, ph ^ 1u, kWaitNs, abort_flag)) {
+          if (!mbar_wait(empty + s, ph ^ 1u, a.wait_ns, abort_flag)) {
             ok = false;
             break;
           }
           uint8_t* sa = smem + size_t(s) * stage_bytes;
-          mbar_arrive_expect_tx(full + s, stage_bytes);
-          tma_load_2d(sa, &tmW, full + s, kb * kBKe, v0, pol_w);
-          tma_load_2d(sa + a_bytes, &tmH, full + s, kb * kBKe, t0, pol_h);
-          issued |= 1u << s;
-          issued_par = (issued_par & ~(1u << s)) | (ph << s);
+          if (hold) {
+            hold = false;  // test hook: this stage never fills
+          } else {
+            mbar_arrive_expect_tx(full + s, stage_bytes);
+            tma_load_2d(sa, &tmW, full + s, kb * kBKe, v0, pol_w);
+            tma_load_2d(sa + a_bytes, &tmH, full + s, kb * kBKe, t0, pol_h);
+            issued |= 1u << s;
+            issued_par = (issued_par & ~(1u << s)) | (ph << s);
+          }
           if (++s == a.stages) {
             s = 0;
             ph ^= 1u;
@@ -327,15 +336,15 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
       for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x, ++local) {
         const int buf = local & 1;
         const uint32_t tph = (local >> 1) & 1;
-        if (!mbar_wait(tempty + buf, tph ^ 1u, kWaitNs, abort_flag)) {
+        if (!mbar_wait(tempty + buf, tph ^ 1u, a.wait_ns, abort_flag)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + buf * buf_cols;
         for (int kb = 0; kb < a.nkb; ++kb) {
-          if (!mbar_wait(full + s, ph, kWaitNs, abort_flag) ||
-              (W4 && !mbar_wait(conv + ia, aph, kWaitNs, abort_flag))) {
+          if (!mbar_wait(full + s, ph, a.wait_ns, abort_flag) ||
+              (W4 && !mbar_wait(conv + ia, aph, a.wait_ns, abort_flag))) {
             ok = false;
             break;
           }
@@ -389,8 +398,8 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
         // other lanes' reads and writes after its wait
         bool got = true;
         if (lane == 0)
-          got = mbar_wait(raw_full + slot, rph, kWaitNs, abort_flag) &&
-                mbar_wait(aempty + ia, aph ^ 1u, kWaitNs, abort_flag);
+          got = mbar_wait(raw_full + slot, rph, a.wait_ns, abort_flag) &&
+                mbar_wait(aempty + ia, aph ^ 1u, a.wait_ns, abort_flag);
         if (!__shfl_sync(0xffffffffu, got, 0)) {
           ok = false;
           break;
@@ -428,7 +437,7 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
       const uint32_t tph = (local >> 1) & 1;
       const int vt = u / a.n_tt;
       const int v0 = vt * kBM, t0 = (u % a.n_tt) * a.Nt;
-      const bool ok = warp_mbar_wait(tfull + buf, tph, kWaitNs, abort_flag);
+      const bool ok = warp_mbar_wait(tfull + buf, tph, a.wait_ns, abort_flag);
       if (!ok || *abort_flag) *epi_abort = 1;
       named_bar_sync(1, 128);
       if (*epi_abort) break;
@@ -597,6 +606,8 @@ cudaError_t launch_head(const jet_layout& lay, const jet_dims& d, const ScorePla
   n_tt = (n.N + Nt - 1) / Nt;
   const int esize = F8 ? 1 : 2;
   TcArgs a{};
+  a.wait_ns = wait_budget_ns();
+  a.hold_first = test_stall();
   a.target_ids = lay.target_ids;
   a.tgt_row = lay.tgt_row;
   a.row_tgt_offset = lay.row_tgt_offset;

@@ -44,7 +44,6 @@ constexpr int kBM = 128;            // weight rows per tile (MMA M, TMEM lanes)
 constexpr int kBK = 64;             // bf16 elements per stage: 128 bytes
 constexpr int kThreads = 192;
 constexpr int kMaxNt = 256;
-constexpr uint64_t kWaitNs = 2000000000ull;
 constexpr uint64_t kDrainNs = 200000000ull;
 constexpr int kSmemLimit = 232448;
 // up-half exchange (64 lanes x 32 columns f32) + barriers and flags
@@ -60,6 +59,8 @@ struct ProjArgs {
   int pair;             // weight tiles per unit (1 or 2)
   int nbuf;             // accumulator sets (2: the epilogue overlaps the next unit)
   uint32_t tmem_cols, acc_cols;
+  uint64_t wait_ns;  // budget of one bounded wait (jet_set_wait_budget_ns)
+  int hold_first;    // test hook (jet_set_test_stall): withhold the first stage's loads
 };
 
 // unit u -> (weight tile, K split, token tile); the token tiles of one weight
@@ -132,22 +133,26 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
       const uint64_t pol_w = policy_evict_first(), pol_x = policy_evict_last();
       int s = 0;
       uint32_t ph = 0, issued = 0, issued_par = 0;
-      bool ok = true;
+      bool ok = true, hold = a.hold_first != 0;
       for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
         const Unit x = unit_of(a, u);
         const int o0 = x.ot * a.pair * kBM, t0 = x.t0;
         for (int kb = x.kb0; kb < x.kb1; ++kb) {
-          if (!mbar_wait(empty + s, ph ^ 1u, kWaitNs, abort_flag)) {
+          if (!mbar_wait(empty + s, ph ^ 1u, a.wait_ns, abort_flag)) {
             ok = false;
             break;
           }
           uint8_t* sa = smem + size_t(s) * stage_bytes;
-          mbar_arrive_expect_tx(full + s, stage_bytes);
-          for (int t = 0; t < a.pair; ++t)
-            tma_load_2d(sa + t * a_bytes, &tmW, full + s, kb * kBK, o0 + t * kBM, pol_w);
-          tma_load_2d(sa + a.pair * a_bytes, &tmX, full + s, kb * kBK, t0, pol_x);
-          issued |= 1u << s;
-          issued_par = (issued_par & ~(1u << s)) | (ph << s);
+          if (hold) {
+            hold = false;  // test hook: this stage never fills
+          } else {
+            mbar_arrive_expect_tx(full + s, stage_bytes);
+            for (int t = 0; t < a.pair; ++t)
+              tma_load_2d(sa + t * a_bytes, &tmW, full + s, kb * kBK, o0 + t * kBM, pol_w);
+            tma_load_2d(sa + a.pair * a_bytes, &tmX, full + s, kb * kBK, t0, pol_x);
+            issued |= 1u << s;
+            issued_par = (issued_par & ~(1u << s)) | (ph << s);
+          }
           if (++s == a.stages) {
             s = 0;
             ph ^= 1u;
@@ -171,7 +176,7 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
       for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x, ++local) {
         const int buf = local % a.nbuf;
         const uint32_t tph = (local / a.nbuf) & 1;
-        if (!mbar_wait(tempty + buf, tph ^ 1u, kWaitNs, abort_flag)) {
+        if (!mbar_wait(tempty + buf, tph ^ 1u, a.wait_ns, abort_flag)) {
           ok = false;
           break;
         }
@@ -179,7 +184,7 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
         const uint32_t d_tmem = tmem_base + uint32_t(buf * a.pair) * a.acc_cols;
         const Unit x = unit_of(a, u);
         for (int kb = x.kb0; kb < x.kb1; ++kb) {
-          if (!mbar_wait(full + s, ph, kWaitNs, abort_flag)) {
+          if (!mbar_wait(full + s, ph, a.wait_ns, abort_flag)) {
             ok = false;
             break;
           }
@@ -217,7 +222,7 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
       const uint32_t tph = (local / a.nbuf) & 1;
       const Unit x = unit_of(a, u);
       const int t0 = x.t0;
-      const bool ok = warp_mbar_wait(tfull + buf, tph, kWaitNs, abort_flag);
+      const bool ok = warp_mbar_wait(tfull + buf, tph, a.wait_ns, abort_flag);
       if (!ok || *abort_flag) *epi_abort = 1;
       named_bar_sync(1, 128);
       if (*epi_abort) break;
@@ -473,6 +478,8 @@ cudaError_t launch_epi(const void* x, int N, int K, int ldx, const void* w, int 
   const Tiling tl = tiling(N, O, K, part != nullptr);
   const int n_tt = tl.n_tt, Nt = tl.Nt;
   ProjArgs a{};
+  a.wait_ns = wait_budget_ns();
+  a.hold_first = test_stall();
   a.part = part;
   a.splits = part ? tl.splits : 1;
   a.out = static_cast<__nv_bfloat16*>(out);

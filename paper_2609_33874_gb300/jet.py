@@ -108,6 +108,9 @@ def _load() -> ctypes.CDLL:
         "jet_decide": (I, [ctypes.POINTER(jet_layout), I, P, P, P, P, P]),
         "jet_evaluate": (I, [ctypes.POINTER(jet_layout), P, P, P, P, P, P]),
         "jet_device_status": (I, [P, ctypes.POINTER(ctypes.c_int32)]),
+        "jet_set_wait_budget_ns": (ctypes.c_uint64, [ctypes.c_uint64]),
+        "jet_launch_count": (ctypes.c_uint64, []),
+        "jet_set_test_stall": (I, [I]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -123,7 +126,8 @@ DECLARED = ("jet_abi_version", "jet_status_string", "jet_layout_plan", "jet_layo
             "jet_fork_state", "jet_fork_state_rule", "jet_score_candidates", "jet_score_candidates_noalloc",
             "jet_quantize_rows_e4m3", "jet_workspace_bytes_e4m3", "jet_score_candidates_e4m3",
             "jet_w4_bytes", "jet_quantize_w4", "jet_score_candidates_w4",
-            "jet_stack_workspace_bytes", "jet_stack_forward", "jet_decide", "jet_evaluate", "jet_device_status")
+            "jet_stack_workspace_bytes", "jet_stack_forward", "jet_decide", "jet_evaluate", "jet_device_status",
+            "jet_set_wait_budget_ns", "jet_launch_count", "jet_set_test_stall")
 
 
 def library() -> ctypes.CDLL:
@@ -407,3 +411,20 @@ def jet_device_status(stream=None) -> int:
     out = ctypes.c_int32(0)
     _check(_lib.jet_device_status(_stream(stream), ctypes.byref(out)), "jet_device_status")
     return int(out.value)
+
+
+def jet_set_wait_budget_ns(ns: int) -> int:
+    """Budget of one bounded wait in the tensor-core kernels (0: the default
+    2 s); returns the previous budget."""
+    return int(_lib.jet_set_wait_budget_ns(int(ns)))
+
+
+def jet_launch_count() -> int:
+    """Kernels the library has launched in this process so far."""
+    return int(_lib.jet_launch_count())
+
+
+def jet_set_test_stall(on: bool) -> bool:
+    """Test hook: the tensor-core kernels launched while it is on withhold their
+    first load, so that a bounded wait runs out; returns the previous setting."""
+    return bool(_lib.jet_set_test_stall(1 if on else 0))

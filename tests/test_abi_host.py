@@ -18,7 +18,7 @@ FIELDS = ("prefix_offset", "cand_offset", "row_offset", "cand_row_offset", "tgt_
 
 def test_exports_every_declared_symbol(jet, repo_root):
     header = open(os.path.join(repo_root, "include", "jet.h")).read()
-    declared = set(re.findall(r"^\s*(?:jet_status|size_t|int32_t|const char\*)\s+(jet_\w+)\s*\(",
+    declared = set(re.findall(r"^\s*(?:jet_status|size_t|int32_t|uint64_t|const char\*)\s+(jet_\w+)\s*\(",
                               header, flags=re.M))
     assert len(declared) >= 12
     lib = ctypes.CDLL(jet.LIB_PATH)
