@@ -10,6 +10,14 @@ candidate sets (requests) scored per second.
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--R R]
     python bench.py --impl reference ...   # the fp64 CPU oracle on the host cores
 
+The default workload is the long-context batch (256 requests, prefixes of
+2,048-8,192 tokens, 16/2 heads, d 256, D 2,048, V 151,936, bf16): the largest
+single-GPU configuration and the one whose LM head is tensor-bound. On one GPU
+the same run then times the other four workloads (`per_workload`, each with
+its roofline, per-call breakdown and CPU-oracle sample) and the batch-size
+sweep R = 1, 2, 4, ..., 128 of the long-context batch (`sweep`); the headline
+`value` is the 256-request batch alone.
+
 Under torchrun (N > 1) every rank scores its own batch on its own GPU
 (independent replicas, no collective on the data path); rank 0 prints one
 JSON line with the whole-job throughput.
@@ -37,7 +45,9 @@ import numpy as np  # noqa: E402
 
 METRIC = "candidate sets scored/sec"
 UNIT = "sets/s"
-DEFAULT_WORKLOAD = "dense27b_mc"
+DEFAULT_WORKLOAD = "moe_a3b_long"
+# the other workloads, timed in the same default run (one GPU)
+EXTRA_WORKLOADS = ("tiny", "dense27b_mc", "binary", "ordinal_hybrid")
 L2_BYTES = 129 * 1024 * 1024
 
 
@@ -56,6 +66,89 @@ def _peaks():
 # ---------------------------------------------------------------------------
 # clocks during the timed region
 # ---------------------------------------------------------------------------
+class NvmlClocks:
+    """SM clock and clock-event reasons of one GPU, polled every `period_s`
+    through read-only NVML queries (clock, maximum clock, event reasons,
+    power) from a background thread, so that even a timed region of a few
+    tens of milliseconds holds many samples. Changes no setting."""
+    REASONS = ((0x4, "sw_power_cap"), (0x8, "hw_slowdown"), (0x20, "sw_thermal_slowdown"),
+               (0x40, "hw_thermal_slowdown"), (0x80, "hw_power_brake_slowdown"))
+
+    def __init__(self, uuid: str | None, period_s: float = 0.001):
+        import ctypes
+        self.period = period_s
+        self.samples = []
+        self.t_on = self.t_off = None
+        self.stop_evt = threading.Event()
+        self.thread = None
+        self.lib = self.h = None
+        try:
+            lib = ctypes.CDLL("libnvidia-ml.so.1")
+            if lib.nvmlInit_v2() != 0:
+                return
+            h = ctypes.c_void_p()
+            ok = False
+            for cand in ([f"GPU-{uuid}", str(uuid)] if uuid else []):
+                if lib.nvmlDeviceGetHandleByUUID(cand.encode(), ctypes.byref(h)) == 0:
+                    ok = True
+                    break
+            if not ok:
+                return
+            self.reasons_fn = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+                getattr(lib, "nvmlDeviceGetCurrentClocksThrottleReasons")
+            mx = ctypes.c_uint()
+            if lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) != 0:
+                return
+            self.smax = float(mx.value)
+            self.lib, self.h = lib, h
+        except (OSError, AttributeError):
+            self.lib = None
+
+    @property
+    def available(self) -> bool:
+        return self.lib is not None
+
+    def start(self):
+        if self.available:
+            self.thread = threading.Thread(target=self._poll, daemon=True)
+            self.thread.start()
+
+    def _poll(self):
+        import ctypes
+        mhz, rsn, mw = ctypes.c_uint(), ctypes.c_ulonglong(), ctypes.c_uint()
+        while not self.stop_evt.is_set():
+            t = time.time()
+            if self.lib.nvmlDeviceGetClockInfo(self.h, 1, ctypes.byref(mhz)) == 0 and \
+                    self.reasons_fn(self.h, ctypes.byref(rsn)) == 0:
+                self.lib.nvmlDeviceGetPowerUsage(self.h, ctypes.byref(mw))
+                self.samples.append((t, float(mhz.value), int(rsn.value), mw.value / 1e3))
+            time.sleep(self.period)
+
+    def mark(self, on: bool):
+        if on:
+            self.t_on = time.time()
+        else:
+            self.t_off = time.time()
+
+    def stop(self):
+        if not self.available:
+            return None
+        self.stop_evt.set()
+        if self.thread:
+            self.thread.join(timeout=2)
+        inside = [x for x in self.samples if self.t_on and self.t_off and
+                  self.t_on <= x[0] <= self.t_off]
+        window = "timed"
+        if not inside:
+            inside, window = self.samples, "warmup+timed"
+        if not inside:
+            return None
+        reasons = sorted({name for x in inside for bit, name in self.REASONS if x[2] & bit})
+        return dict(sm_mhz=statistics.median(x[1] for x in inside), sm_max_mhz=self.smax,
+                    reasons=reasons, samples=len(inside), window=window,
+                    power_w_max=round(max(x[3] for x in inside), 1), source="nvml, 1 ms")
+
+
 class ClockSampler:
     QUERY = ("timestamp,index,uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -217,74 +310,6 @@ def _call(ms: float, nbytes: int, peaks) -> dict:
                 achieved_gbs=round(gbs, 1), frac=round(gbs / peaks["hbm"], 4))
 
 
-def _attend_launches(problem, w) -> int:
-    """Kernels jet_prefix_attend launches for this batch: the float32 path is
-    prefix + merge; the bf16 path is the work-list kernel (or the counter
-    reset), the persistent tensor-core kernel and a chunk combine when the
-    plan splits the longest prefix (the library's plan: near-equal chunks of
-    at least 640 keys and no finer than half of one SM's share of the key
-    tiles over 152 SMs)."""
-    if w.dtype != "bf16":
-        return 2
-    g = w.Hq // w.Hkv
-    R, N = problem.R, problem.N
-    max_prefix = int(problem.prefix_len.max())
-    total_prefix = int(problem.prefix_len.sum())
-    avg_vecs = (N * g + R - 1) // R
-    qv = max(1, 128 // g) * g  # whole rows of g heads per query block
-    groups = R * w.Hkv * max(1, (avg_vecs + qv - 1) // qv)
-    share = groups * (total_prefix / R / 64.0 + 0.5) / 152
-    chunk = max(640, int(share / 2.0 + 0.999) * 64)
-    chunk = min(chunk, max(1, (max_prefix + 63) // 64) * 64)
-    splits = (max_prefix + chunk - 1) // chunk
-    return 2 + (1 if splits > 1 else 0)
-
-
-def _proj_launches(N: int, O: int, K: int) -> int:
-    """Kernels one projection launches: the GEMM, plus the reduce of a split K
-    (the library's rule: row tiles of at most 256, two weight tiles per unit
-    for row tiles of at most 128, K split until the units cover 152 SMs twice
-    with at least 8 K slices each)."""
-    n_tt = (N + 255) // 256
-    Nt = ((N + n_tt - 1) // n_tt + 15) // 16 * 16
-    n_tt = (N + Nt - 1) // Nt
-    otiles = (O + 127) // 128
-    pair = 2 if (otiles >= 2 and Nt <= 128) else 1
-    units = (otiles + pair - 1) // pair * n_tt
-    nkb = (K + 63) // 64
-    splits = 1
-    while units * splits < 2 * 152 and nkb // (splits + 1) >= 8:
-        splits += 1
-    return 1 + (1 if splits > 1 else 0)
-
-
-def _stack_launches(problem, w, spec) -> int:
-    """Kernels one jet_stack_forward launches (the copy of x0 aside)."""
-    N, D, Dff = problem.N, w.D, spec.Dff
-
-    def resid(K, norm):
-        # a residual projection; the RMSNorm after it shares the reduce of a
-        # split K, else it is a launch of its own
-        k = _proj_launches(N, D, K)
-        return k + (1 if norm and k == 1 else 0)
-
-    n = 1 if spec.kinds else 0                               # the first layer's RMSNorm
-    for l, kind in enumerate(spec.kinds):
-        if kind == "full":
-            ow = w.Hq * w.d
-            # the q/k/v projection, its reduce fused with the split (or the split
-            # after an unsplit one), the attention
-            mixer = 2 + _attend_launches(problem, w)
-        else:
-            ow = w.Hl * w.dv
-            # the mixer projection, its reduce fused with the gates (or the
-            # gates after an unsplit one), the fork (with the shared rows)
-            mixer = 3
-        n += mixer + resid(ow, True)
-        n += _proj_launches(N, 2 * Dff, D) + resid(Dff, l + 1 < len(spec.kinds))
-    return n
-
-
 def aggregate(total_ms: float, e2e_ms: float, R: int, steps: int, world: int, device=None):
     """Whole-job numbers of N independent replicas: the slowest rank's timed
     regions (max over ranks) and the sets all ranks scored per second.
@@ -310,28 +335,32 @@ def _dist():
 # ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
-def run_gpu(args):
-    import torch
-    world, rank, local = _dist()
-    if world > 1:
-        import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    dev = torch.device("cuda", local)
-    torch.cuda.set_device(dev)
+def _device_inputs(problem, names, dev, src=None):
+    """The step's inputs on the device: drawn for `problem`, or (src given) the
+    leading rows of a larger batch's device tensors - a batch of the first R
+    requests of a draw is the leading part of every packed input."""
+    import jet_synth
+    if src is None:
+        return {k: jet_synth.torch_tensor(problem, k, device=dev) for k in names}
+    P, N, F = problem.total_prefix, problem.N, problem.N - problem.R
+    rows = dict(q=N, hidden=N, k_pre=P, v_pre=P, k_cand=F, v_cand=F, lq=F, lk=F, lv=F, alpha=F,
+                beta=F, s_prefix=problem.R)
+    return {k: src[k][:rows[k]] for k in names}
 
-    from paper_2609_33874_gb300 import build as _build
-    if rank == 0:
-        _build.build()
-    if world > 1:
-        torch.distributed.barrier()
+
+def _measure(args, problem, dev, stream, peaks, world=1, src=None, w_lm=None, clocks=None,
+             e2e=False, evaluate=False):
+    """Times `args.steps` scoring steps of `problem` (inputs resident in HBM)
+    after `args.warmup` untimed ones, then the per-call breakdown, and returns
+    the numbers of one JSON record (the headline line or a `per_workload` /
+    `sweep` entry). With e2e the step is also timed end to end from pinned
+    host memory."""
+    import torch
     import jet_synth
     from paper_2609_33874_gb300 import jet
     from paper_2609_33874_gb300.step import ScoringStep
-
-    w = jet_synth.WORKLOADS[args.workload]
-    R = args.R or w.R
-    problem = jet_synth.make_problem(w, R=R)
+    w = problem.work
+    R = problem.R
     dtype = jet.DTYPE_BF16 if w.dtype == "bf16" else jet.DTYPE_F32
     dims = jet.make_dims(dtype, Hq=w.Hq, Hkv=w.Hkv, d=w.d, D=w.D, Hl=w.Hl, dk=w.dk, dv=w.dv)
     hl = jet.jet_layout_build(problem.prefix_len, problem.n_cand, problem.cand_len,
@@ -340,26 +369,17 @@ def run_gpu(args):
     step = ScoringStep(hl, dims, jet.MODES[w.mode], device=dev, hybrid=w.Hl > 0,
                        keep_fork_state=w.Hl > 0, lm=args.lm, rule=args.rule)
     names = step.input_names()
-    x = {k: jet_synth.torch_tensor(problem, k, device=dev) for k in names}
-    w_lm = jet_synth.torch_tensor(problem, "w_lm", device=dev)
-    if low:
-        # model state: the weights are quantised once, outside the timed region
-        from paper_2609_33874_gb300.step import quantize_lm_head, quantize_lm_head_w4
-        w_lm = (quantize_lm_head_w4 if args.lm == "w4" else quantize_lm_head)(w_lm)
-        torch.cuda.synchronize(dev)
-    stream = torch.cuda.Stream(dev)
+    x = _device_inputs(problem, names, dev, src)
+    if w_lm is None:
+        w_lm = jet_synth.torch_tensor(problem, "w_lm", device=dev)
+        if low:
+            # model state: the weights are quantised once, outside the timed region
+            from paper_2609_33874_gb300.step import quantize_lm_head, quantize_lm_head_w4
+            w_lm = (quantize_lm_head_w4 if args.lm == "w4" else quantize_lm_head)(w_lm)
+            torch.cuda.synchronize(dev)
 
-    # --- device-resident timed region -------------------------------------
     # the per-call breakdown (taken outside the timed steps): attend | fork | score | decide
-    n_ev = args.steps
-    call_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(n_ev)]
-    uuid = None
-    try:
-        uuid = str(torch.cuda.get_device_properties(dev).uuid)
-    except Exception:
-        pass
-    clocks = ClockSampler(uuid)
-    clocks.start()
+    call_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
 
     def one_step(i=None):
         d, lay = step.dims, step.layout
@@ -387,24 +407,28 @@ def run_gpu(args):
         for _ in range(args.warmup):
             one_step()
     torch.cuda.synchronize(dev)
-    assert jet.jet_device_status(stream) == 0, "kernel reported an invalid layout index"
+    assert jet.jet_device_status(stream) == 0, "a kernel reported an error status"
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize(dev)
-    clocks.mark(True)
+    if clocks:
+        clocks.mark(True)
+    n0 = jet.jet_launch_count()
     t_start.record(stream)
     with torch.cuda.stream(stream):
         for _ in range(args.steps):
             one_step()   # no events between the calls: each call's kernels may
                          # start while the previous call's last kernel ends
     t_end.record(stream)
+    launches = jet.jet_launch_count() - n0
     torch.cuda.synchronize(dev)
-    clocks.mark(False)
+    if clocks:
+        clocks.mark(False)
     if world > 1:
         torch.distributed.barrier()
     total_ms = t_start.elapsed_time(t_end)
-    clk = clocks.stop()
+    clk = clocks.stop() if clocks else None
     # the per-call breakdown: the same steps again with events between the calls
     with torch.cuda.stream(stream):
         for i in range(args.steps):
@@ -413,55 +437,58 @@ def run_gpu(args):
     call_ms = {name: statistics.mean(ev[k].elapsed_time(ev[k + 1]) for ev in call_ev)
                for k, name in enumerate(("attend", "fork", "score", "decide"))}
 
-    # --- evaluation helper (after the step, outside it): gold NLL + agreement,
-    # with every request's first candidate taken as the gold label
-    gold = torch.zeros(step.C, dtype=torch.uint8, device=dev)
-    gold[torch.as_tensor(hl.array("cand_offset")[:-1], dtype=torch.long, device=dev)] = 1
-    nll = torch.empty(step.R, dtype=torch.float32, device=dev)
-    correct = torch.empty(step.R, dtype=torch.int32, device=dev)
-    ev_a, ev_b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    n_eval = 20
-    with torch.cuda.stream(stream):
-        jet.jet_evaluate(step.layout, step.cand_score, step.choice, gold, nll, correct,
-                         stream=stream)
-        ev_a.record(stream)
-        for _ in range(n_eval):
+    if evaluate:
+        # evaluation helper (after the step, outside it): gold NLL + agreement,
+        # with every request's first candidate taken as the gold label
+        gold = torch.zeros(step.C, dtype=torch.uint8, device=dev)
+        gold[torch.as_tensor(hl.array("cand_offset")[:-1], dtype=torch.long, device=dev)] = 1
+        nll = torch.empty(step.R, dtype=torch.float32, device=dev)
+        correct = torch.empty(step.R, dtype=torch.int32, device=dev)
+        ev_a, ev_b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        n_eval = 20
+        with torch.cuda.stream(stream):
             jet.jet_evaluate(step.layout, step.cand_score, step.choice, gold, nll, correct,
                              stream=stream)
-        ev_b.record(stream)
-    torch.cuda.synchronize(dev)
-    call_ms["evaluate"] = ev_a.elapsed_time(ev_b) / n_eval
+            ev_a.record(stream)
+            for _ in range(n_eval):
+                jet.jet_evaluate(step.layout, step.cand_score, step.choice, gold, nll, correct,
+                                 stream=stream)
+            ev_b.record(stream)
+        torch.cuda.synchronize(dev)
+        call_ms["evaluate"] = ev_a.elapsed_time(ev_b) / n_eval
 
-    # --- end to end: pinned host inputs, copies inside the timed region ---------
-    # a batch as a loader leaves it: its layout words and inputs in one pinned
-    # buffer (HostBatch), the results back into one pinned buffer (HostResults)
-    from paper_2609_33874_gb300.step import HostBatch, HostResults
-    host = {k: x[k].cpu().pin_memory() for k in names}
-    words = torch.from_numpy(hl.words).pin_memory()
-    batch = HostBatch(step, host, words)
-    out = HostResults(step)
-    # every step copies its inputs in and its results out; step i+1's input
-    # copy overlaps step i's kernels (double-buffered device inputs)
-    e_steps = max(3, min(args.steps, 50))
-    step.run_pipelined([batch] * max(3, args.warmup), w_lm,
-                       [out] * max(3, args.warmup), stream=stream)
-    torch.cuda.synchronize(dev)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    if world > 1:
-        torch.distributed.barrier()
-    e0.record(stream)
-    step.run_pipelined([batch] * e_steps, w_lm, [out] * e_steps, stream=stream)
-    e1.record(stream)
-    torch.cuda.synchronize(dev)
-    e2e_ms = e0.elapsed_time(e1) / e_steps
-    h2d, d2h = batch.nbytes, out.buf.numel()
+    e2e_ms, h2d, d2h = None, 0, 0
+    if e2e:
+        # end to end: pinned host inputs, copies inside the timed region. A
+        # batch as a loader leaves it: its layout words and inputs in one
+        # pinned buffer (HostBatch), the results back into one pinned buffer
+        # (HostResults); step i+1's input copy overlaps step i's kernels
+        from paper_2609_33874_gb300.step import HostBatch, HostResults
+        host = {k: x[k].cpu().pin_memory() for k in names}
+        words = torch.from_numpy(hl.words).pin_memory()
+        batch = HostBatch(step, host, words)
+        out = HostResults(step)
+        e_steps = max(3, min(args.steps, 50))
+        step.run_pipelined([batch] * max(3, args.warmup), w_lm,
+                           [out] * max(3, args.warmup), stream=stream)
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        if world > 1:
+            torch.distributed.barrier()
+        e0.record(stream)
+        step.run_pipelined([batch] * e_steps, w_lm, [out] * e_steps, stream=stream)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms = e0.elapsed_time(e1) / e_steps
+        h2d, d2h = batch.nbytes, out.buf.numel()
+        del host, batch, out
     assert jet.jet_device_status(stream) == 0
 
-    total_ms, e2e_ms, ms_per_step, value, e2e_value = aggregate(
-        total_ms, e2e_ms, R, args.steps, world, device=dev)
+    total_ms, e2e_agg, ms_per_step, value, e2e_value = aggregate(
+        total_ms, e2e_ms if e2e_ms is not None else total_ms / args.steps, R, args.steps, world,
+        device=dev)
 
     # --- roofline of the dominant kernel (the LM head) ----------------------
-    peaks = _peaks()
     N, T = problem.N, len(problem.target_ids)
     es = 2 if w.dtype == "bf16" else 4
     vtiles = (w.V + 127) // 128
@@ -477,10 +504,10 @@ def run_gpu(args):
     # measured bf16 peak x the nominal 2x of 8-bit operands
     tc_peak = peaks["bf16"] * (2 if low else 1)
     ridge = tc_peak * 1e12 / (peaks["hbm"] * 1e9)
-    kernel_file = "paper_2609_33874_gb300/csrc/lmhead_tc.cu" if w.dtype == "bf16" and \
-        os.path.exists(os.path.join(ROOT, "paper_2609_33874_gb300/csrc/lmhead_tc.cu")) \
-        else "paper_2609_33874_gb300/csrc/lmhead_simt.cu"
-    traffic = _traffic(kernel_file, args.workload + (":" + args.lm if low else ""))
+    kernel_file = ("paper_2609_33874_gb300/csrc/lmhead_tc.cu" if w.dtype == "bf16"
+                   else "paper_2609_33874_gb300/csrc/lmhead_simt.cu")
+    wl_key = problem_key(args, problem)
+    traffic = _traffic(kernel_file, wl_key + (":" + args.lm if low else ""))
     if w.dtype != "bf16":
         # float32 FMA: SMs x 128 lanes x 2 flop x the maximum SM clock
         sms = torch.cuda.get_device_properties(dev).multi_processor_count
@@ -496,6 +523,7 @@ def run_gpu(args):
         ach = lm_flops / score_avg_s / 1e12
         roof = dict(bound="tensor", achieved=round(ach, 1), peak=round(tc_peak, 1), unit="TFLOP/s",
                     frac=round(ach / tc_peak, 4), traffic=traffic)
+        roof["frac_of_sustained"] = round(ach / (peaks["bf16_sustained"] * (2 if low else 1)), 4)
     roof.update(kernel="jet_score_candidates" + (f"_{args.lm} (quantise hidden + {args.lm} LM head "
                                                  "+ lse merge)" if low else
                                                  " (LM head + lse merge)"),
@@ -509,57 +537,165 @@ def run_gpu(args):
     calls = dict(attend=_call(call_ms["attend"], attn_bytes, peaks),
                  score=dict(ms=round(call_ms["score"], 4), bound=roof["bound"],
                             frac=roof["frac"]),
-                 decide=dict(ms=round(call_ms["decide"], 4)),
-                 evaluate=dict(ms=round(call_ms["evaluate"], 4),
-                               note="outside the step: gold NLL over equivalent labels and "
-                                    "agreement, back to back"))
+                 decide=dict(ms=round(call_ms["decide"], 4)))
+    if "evaluate" in call_ms:
+        calls["evaluate"] = dict(ms=round(call_ms["evaluate"], 4),
+                                 note="outside the step: gold NLL over equivalent labels and "
+                                      "agreement, back to back")
     if w.Hl:
         fork_bytes = (R * w.Hl * w.dk * w.dv * 4 + len(problem.cand_len) * w.Hl * w.dk * w.dv * 4
                       + F * w.Hl * (2 * w.dk + 2 * w.dv) * es + F * w.Hl * 8)
         calls["fork"] = _call(call_ms["fork"], fork_bytes, peaks)
+    rec = dict(value=round(value, 2), unit=UNIT, ms_per_step=round(ms_per_step, 4),
+               clocks=clk, gpu_launches=int(launches), roofline=roof, calls=calls,
+               config=step_config(args, problem, world))
+    if e2e:
+        rec["e2e"] = dict(value=round(e2e_value, 2), unit=UNIT, h2d_bytes_per_step=h2d,
+                          d2h_bytes_per_step=d2h, ms_per_step=round(e2e_agg, 4))
+    del x, step
+    return rec, w_lm
 
-    launches_per_step = _attend_launches(problem, w) + (1 if w.Hl else 0) + 3 + 1 + (1 if low else 0)
+
+def problem_key(args, problem) -> str:
+    """Name of a timed batch: the workload, and R where it is a smaller batch."""
+    full = problem.work.R
+    return args.workload if problem.R == full else f"{args.workload}:R={problem.R}"
+
+
+def run_gpu(args):
+    import torch
+    world, rank, local = _dist()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+
+    from paper_2609_33874_gb300 import build as _build
+    if rank == 0:
+        _build.build()
+    if world > 1:
+        torch.distributed.barrier()
+    import jet_synth
+
+    w = jet_synth.WORKLOADS[args.workload]
+    R = args.R or w.R
+    problem = jet_synth.make_problem(w, R=R)
+    stream = torch.cuda.Stream(dev)
+    peaks = _peaks()
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        pass
+    clocks = NvmlClocks(uuid)
+    if not clocks.available:
+        clocks = ClockSampler(uuid)
+    clocks.start()
+
+    # --- the headline batch: device-resident steps, per-call breakdown, e2e
+    from paper_2609_33874_gb300.step import ScoringStep  # noqa: F401  (loads the library)
+    head, w_lm = _measure(args, problem, dev, stream, peaks, world=world, clocks=clocks,
+                          e2e=not args.no_e2e, evaluate=True)
+    low = args.lm != "bf16"
     result = dict(
-        metric=METRIC, value=round(value, 2), unit=UNIT, n_gpus=world, steps=args.steps,
-        warmup=args.warmup, ms_per_step=round(ms_per_step, 4), higher_is_better=True,
+        metric=METRIC, value=head["value"], unit=UNIT, n_gpus=world, steps=args.steps,
+        warmup=args.warmup, ms_per_step=head["ms_per_step"], higher_is_better=True,
         scaling="weak", vs_baseline=None,
         dtype=(f"bf16 (LM head {args.lm})" if low else "bf16") if w.dtype == "bf16" else "f32",
         data="synthetic",
-        config=step_config(args, problem, world),
-        clocks=clk,
-        e2e=dict(value=round(e2e_value, 2), unit=UNIT, h2d_bytes_per_step=h2d,
-                 d2h_bytes_per_step=d2h, ms_per_step=round(e2e_ms, 4)),
-        gpu_launches=launches_per_step * args.steps,
-        roofline=roof,
-        calls=calls,
+        config=head["config"],
+        clocks=head["clocks"],
+        e2e=head.get("e2e"),
+        gpu_launches=head["gpu_launches"],
+        roofline=head["roofline"],
+        calls=head["calls"],
     )
+    extras = world == 1 and not args.headline_only
     if rank == 0 and world == 1 and not args.no_cpu_baseline and not low:
         result["cpu_baseline"] = cpu_baseline(args.workload, R, args.cpu_sample)
+
+    if extras and args.workload == DEFAULT_WORKLOAD and R == w.R:
+        # the batch-size sweep: the first R requests of the same draw, sliced
+        # from the headline batch's device inputs
+        src = _device_inputs(problem, _input_names(problem), dev)
+        sweep = []
+        r = 1
+        while r < R:
+            sub = jet_synth.make_problem(w, R=r)
+            rec, _ = _measure(args, sub, dev, stream, peaks, src=src, w_lm=w_lm)
+            sweep.append(dict(R=r, N=sub.N, value=rec["value"], ms_per_step=rec["ms_per_step"],
+                              gpu_launches=rec["gpu_launches"], roofline=_brief(rec["roofline"]),
+                              calls=rec["calls"]))
+            r *= 2
+        sweep.append(dict(R=R, N=problem.N, value=head["value"], ms_per_step=head["ms_per_step"],
+                          gpu_launches=head["gpu_launches"], roofline=_brief(head["roofline"]),
+                          calls=head["calls"]))
+        result["sweep"] = sweep
+        del src
+    del w_lm
+    torch.cuda.empty_cache()
+
+    if extras and args.workload == DEFAULT_WORKLOAD and not low:
+        # the other workloads: the same step, timed the same way, each with its
+        # own roofline, per-call breakdown and CPU-oracle sample
+        per = {}
+        saved = args.workload
+        for name in EXTRA_WORKLOADS:
+            args.workload = name
+            wp = jet_synth.make_problem(name)
+            rec, wl = _measure(args, wp, dev, stream, peaks)
+            del wl
+            torch.cuda.empty_cache()
+            if not args.no_cpu_baseline:
+                rec["cpu_baseline"] = cpu_baseline(name, wp.R, args.cpu_sample)
+            rec["dtype"] = "bf16" if wp.work.dtype == "bf16" else "f32"
+            per[name] = rec
+            wp.drop()
+        args.workload = saved
+        result["per_workload"] = per
     if world > 1:
         torch.distributed.destroy_process_group()
     if rank == 0:
         print(json.dumps(result), flush=True)
 
 
+def _input_names(problem):
+    """The step's input names for this problem's workload."""
+    names = ["q", "k_pre", "v_pre", "k_cand", "v_cand", "hidden"]
+    if problem.work.Hl:
+        names += ["s_prefix", "lq", "lk", "lv", "alpha", "beta"]
+    return names
+
+
+def _brief(roof):
+    return {k: roof[k] for k in ("bound", "achieved", "peak", "unit", "frac") if k in roof}
+
+
 # ---------------------------------------------------------------------------
 # the prefill (a "next" row, one GPU): causal attention over the prefixes
 # ---------------------------------------------------------------------------
 def _time_stream(fn, stream, warmup, steps):
-    """Average milliseconds of fn() over `steps` launches on `stream` (CUDA
-    events on that stream, after `warmup` untimed calls)."""
+    """Average milliseconds of fn() over `steps` calls on `stream` (CUDA events
+    on that stream, after `warmup` untimed calls) and the library's kernel
+    launches inside the timed calls."""
     import torch
+    from paper_2609_33874_gb300 import jet
     with torch.cuda.stream(stream):
         for _ in range(warmup):
             fn()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n0 = jet.jet_launch_count()
     e0.record(stream)
     with torch.cuda.stream(stream):
         for _ in range(steps):
             fn()
     e1.record(stream)
+    launches = jet.jet_launch_count() - n0
     torch.cuda.synchronize()
-    return e0.elapsed_time(e1) / steps
+    return e0.elapsed_time(e1) / steps, launches
 
 
 def _roof(flops, nbytes, ms, peaks):
@@ -605,8 +741,9 @@ def run_prefill(args):
     o = torch.empty(p.total_prefix, w.Hq, w.d, dtype=torch.bfloat16, device=dev)
     wsb = jet.jet_prefill_workspace_bytes(hl.sizes, dims)
     ws = torch.empty((wsb + 15) // 16 * 4, dtype=torch.float32, device=dev)
-    ms = _time_stream(lambda: jet.jet_prefill_attend(lay, dims, q, k, v, o, ws, stream=stream),
-                      stream, args.warmup, args.steps)
+    ms, n_att = _time_stream(
+        lambda: jet.jet_prefill_attend(lay, dims, q, k, v, o, ws, stream=stream),
+        stream, args.warmup, args.steps)
     assert jet.jet_device_status(stream) == 0
     del q, k, v, o, ws
     # S = QK^T and O = PV over the causal triangle (keys 0..p of position p)
@@ -616,7 +753,7 @@ def run_prefill(args):
     roof.update(kernel="jet_prefill_attend (work list + attend_prefix_tc_kernel, causal)",
                 algorithmic_flops=flops, algorithmic_bytes=nbytes, traffic=None,
                 peak_source=peaks["source"])
-    parts["attend"] = dict(ms=round(ms, 4), roofline=roof, launches=2)
+    parts["attend"] = dict(ms=round(ms, 4), roofline=roof, launches=n_att)
 
     if w.Hl > 0:
         ldims = jet.make_dims(jet.DTYPE_BF16, Hl=w.Hl, dk=w.dk, dv=w.dv, D=w.D)
@@ -625,7 +762,7 @@ def run_prefill(args):
         lo = torch.empty(p.total_prefix, w.Hl, w.dv, dtype=torch.bfloat16, device=dev)
         s_out = torch.empty(R, w.Hl, w.dk, w.dv, dtype=torch.float32, device=dev)
         rule = jet.RULES[args.rule]
-        ms_s = _time_stream(
+        ms_s, n_scan = _time_stream(
             lambda: jet.jet_prefill_state(lay, ldims, t["lq_pre"], t["lk_pre"], t["lv_pre"],
                                           t["alpha_pre"], t["beta_pre"], lo, s_out,
                                           s_init=t["s_prefix"], rule=rule, stream=stream),
@@ -647,7 +784,7 @@ def run_prefill(args):
                      peak_basis="fp32 FMA: 152 SMs x 128 lanes x 2 flop x max SM clock",
                      algorithmic_flops=sflops, algorithmic_bytes=sbytes, traffic=None,
                      peak_source=peaks["source"])
-        parts["state"] = dict(ms=round(ms_s, 4), roofline=sroof, launches=1)
+        parts["state"] = dict(ms=round(ms_s, 4), roofline=sroof, launches=n_scan)
         del t, lo, s_out
     p.drop()
     total_ms = sum(x["ms"] for x in parts.values())
@@ -660,7 +797,7 @@ def run_prefill(args):
                     max_prefix=int(P.max()), Hq=w.Hq, Hkv=w.Hkv, d=w.d, Hl=w.Hl,
                     rule=args.rule if w.Hl > 0 else None),
         roofline=dom["roofline"], parts=parts,
-        gpu_launches=sum(x["launches"] for x in parts.values()) * args.steps)), flush=True)
+        gpu_launches=sum(x["launches"] for x in parts.values()))), flush=True)
 
 
 def run_stack(args):
@@ -704,8 +841,8 @@ def run_stack(args):
         jet.jet_decide(step.layout, step.mode, step.cand_score, step.q_cand, step.choice,
                        step.value, stream=stream)
 
-    ms = _time_stream(one, stream, args.warmup, args.steps)
-    ms_stack = _time_stream(lambda: stack.forward(x0, stream=stream), stream, 2, args.steps)
+    ms, n_fwd = _time_stream(one, stream, args.warmup, args.steps)
+    ms_stack, _ = _time_stream(lambda: stack.forward(x0, stream=stream), stream, 2, args.steps)
     assert jet.jet_device_status(stream) == 0
     N = p.N
     # the stack's projections: weight bytes once per call, 2 N K O flops each
@@ -729,7 +866,7 @@ def run_stack(args):
                     Dff=spec.Dff, R=R, N=N, D=w.D, rule=args.rule),
         roofline=roof, parts=dict(stack_ms=round(ms_stack, 4),
                                   score_and_decide_ms=round(ms - ms_stack, 4)),
-        gpu_launches=(_stack_launches(p, w, spec) + 4) * args.steps)), flush=True)
+        gpu_launches=n_fwd)), flush=True)
 
 
 # ---------------------------------------------------------------------------
@@ -742,7 +879,7 @@ def run_reference(args):
     import jet_synth
     w = jet_synth.WORKLOADS[args.workload]
     R = args.R or w.R
-    k = args.ref_sample
+    k = args.ref_sample or args.cpu_sample
     p = oracle_sample(args.workload, R, k)
     for _ in range(args.warmup):
         oracle_step(p)
@@ -774,9 +911,14 @@ def main():
     ap.add_argument("--R", type=int, default=0, help="requests per batch (default: the workload's)")
     ap.add_argument("--cpu-sample", type=int, default=16,
                     help="requests in the CPU-oracle baseline sample")
-    ap.add_argument("--ref-sample", type=int, default=1,
-                    help="requests per step of the reference arm")
+    ap.add_argument("--ref-sample", type=int, default=0,
+                    help="requests per step of the reference arm (default: --cpu-sample, so "
+                         "that both CPU figures time the same sample)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true",
+                    help="skip the end-to-end timing (profiling runs: device inputs only)")
+    ap.add_argument("--headline-only", action="store_true",
+                    help="time the headline batch only (no per-workload lines, no sweep)")
     ap.add_argument("--rule", default="delta", choices=["delta", "gla"],
                     help="recurrence of the linear-attention fork (hybrid workloads)")
     ap.add_argument("--lm", default="bf16", choices=["bf16", "e4m3", "w4"],
@@ -806,6 +948,7 @@ def main():
             ap.error("--sweep runs on one GPU")
         args.no_cpu_baseline = True
         full = jet_synth.WORKLOADS[args.workload].R
+        args.headline_only = True
         r = 1
         while r <= full:
             args.R = r
