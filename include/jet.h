@@ -365,21 +365,22 @@ jet_status jet_score_candidates_e4m3(const jet_layout* lay, const jet_dims* dims
  *   nearest with ties to the even code, saturated at +-6. A row of zeros gets
  *   s = 0, zero codes and e = -5.
  *
- * Tiled layout of the codes (the order the LM head streams them): one tile of
- * 8,704 bytes per (vocabulary tile vt of 128 rows, K slice kb of 128
- * elements), tile index vt * ceil(D / 128) + kb. Bytes [0, 8192): row r of
- * the tile (vocabulary row 128 vt + r) has 64 bytes at r * 64; its 16-byte
- * chunk c (elements 128 kb + 32 c .. + 31) is stored in slot c ^ ((r >> 1) & 3).
- * A chunk is four little-endian 32-bit words of 8 elements each: nibble k
- * (bits 4k .. 4k+3) holds the magnitude (3 bits) of element k of the word in
- * its low bits and, in bit 3, the sign of element 4 + k / 2 (k even) or k / 2
- * (k odd). Bytes [8192, 8704):
- * the block exponents, int8, row r's four at 8192 + 4 r + c. Rows past V and
- * elements past D are zero codes.
+ * Layout of the w4 buffer (what the block-scaled tensor-core path reads):
+ * with Vp = 128 ceil(V / 128) rows and Kp = 128 ceil(D / 128) codes per row,
+ *   - a code region of Vp * Kp / 2 bytes, row-major: code k of row v is the
+ *     nibble (k & 1) of byte v * Kp / 2 + k / 2 (element 2 j in the low nibble
+ *     of byte j), in the OCP E2M1 encoding (sign in bit 3);
+ *   - then a scale-factor region of one 512-byte chunk per (vocabulary tile vt
+ *     of 128 rows, K slice kb of 128 codes), chunk index vt ceil(D / 128) + kb:
+ *     byte 16 i + 4 j + c of a chunk is the UE8M0 factor 127 + e of block c of
+ *     the slice in row 32 j + i of the tile (the order in which one tcgen05.cp
+ *     of 32 x 128 bits places the chunk in tensor memory for the block-scaled
+ *     MMA). Rows past V and codes past D are zero codes; their blocks have
+ *     e = -5.
  */
 
-/* Bytes of the tiled 4-bit codes of a [V, D] matrix:
- * ceil(V / 128) * ceil(D / 128) * 8704; 0 on invalid arguments. */
+/* Bytes of the w4 buffer of a [V, D] matrix (codes and scale factors):
+ * ceil(V / 128) * ceil(D / 128) * (8192 + 512); 0 on invalid arguments. */
 size_t jet_w4_bytes(int64_t V, int64_t D);
 
 /*
@@ -396,11 +397,13 @@ jet_status jet_quantize_w4(const void* w, int64_t V, int64_t D, uint8_t* w4, flo
  * jet_score_candidates_w4 - jet_score_candidates with a 4-bit LM head:
  *   hidden      [N, D] bf16     quantised per row (token) to e4m3 into the
  *                               workspace, as in jet_score_candidates_e4m3
- *   w4          tiled codes of w_lm from jet_quantize_w4 with the same V, D
+ *   w4          codes and scale factors of w_lm from jet_quantize_w4 with the
+ *               same V, D (32-byte aligned, else JET_ERR_ALIGN)
  *   w_scale     [V] float32     their per-row scales
  * The logit is z[n, v] = s_h[n] s_w[v] sum_k decode(h_q[n, k]) 2^e value(code),
- * accumulated in float32 on the tensor cores (each 2^e value(code) is an e4m3
- * value, widened on chip); log-softmax, gather and sums as in
+ * accumulated in float32 on the tensor cores by the block-scaled MMA (E2M1
+ * weight codes with one UE8M0 factor 2^e per 32-element block, e4m3 hidden
+ * codes: every product is exact); log-softmax, gather and sums as in
  * jet_score_candidates. dims as for jet_score_candidates_e4m3; workspace
  * jet_workspace_bytes_e4m3().
  */

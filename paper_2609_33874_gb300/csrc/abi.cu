@@ -389,6 +389,7 @@ extern "C" jet_status jet_score_candidates_w4(const jet_layout* lay, const jet_d
   if (plan.score.vtiles > 65535) return JET_ERR_CAPACITY;
   JET_TRY(check_ptr(hidden, n.N));
   JET_TRY(check_ptr(w4, n.V));
+  if ((reinterpret_cast<uintptr_t>(w4) & 31u) != 0) return JET_ERR_ALIGN;  // the TMA's 4-bit map
   JET_TRY(check_ptr(w_scale, n.V));
   JET_TRY(check_ptr(tok_logprob, n.T));
   JET_TRY(check_ptr(cand_score, n.C));

@@ -124,10 +124,6 @@ __device__ __forceinline__ void tmem_st_32cols(uint32_t taddr, const float (&v)[
       : "memory");
 }
 
-__device__ __forceinline__ void tmem_wait_st() {
-  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-}
-
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }

@@ -16,10 +16,12 @@ int* device_status_ptr();
 
 // ---- workspace plans -----------------------------------------------------------
 constexpr int kVocabTile = 128;  // vocabulary entries per LM-head partial
-// 4-bit weights: one tile per (128 vocabulary rows, 128-element K slice):
-// 128 x 64 bytes of packed E2M1 codes, then 128 x 4 block exponents
+// 4-bit weights, per (128 vocabulary rows, 128-element K slice): 128 x 64
+// bytes of packed E2M1 codes (in the row-major code region) and a 512-byte
+// chunk of UE8M0 block scale factors (in the scale region after it)
 constexpr int kW4CodeBytes = kVocabTile * 64;
-constexpr int kW4TileBytes = kW4CodeBytes + kVocabTile * 4;
+constexpr int kW4ScaleBytes = 512;
+constexpr int kW4TileBytes = kW4CodeBytes + kW4ScaleBytes;
 
 struct AttnPlan {
   int splits;    // prefix chunks per (request, key/value head)

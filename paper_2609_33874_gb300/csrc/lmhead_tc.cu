@@ -30,15 +30,20 @@
 //
 // The w4 instantiation (4-bit weights: E2M1 codes with a power-of-two exponent
 // per 32-element block under a float32 row scale) streams the weights at half
-// the e4m3 bytes. It keeps three rings: hidden-state tiles and 4-bit weight
-// tiles (128 rows x 128 codes and their exponents, 8,704 bytes, one TMA box of
-// the pre-tiled buffer), both issued by the producer as far ahead as they
-// fit, and two widened e4m3 weight tiles that only live from their
-// conversion to their MMA. Eight converter warps (warps 6..13, a
-// thread per vocabulary row and half slice) widen every code to the e4m3 value
-// 2^e value(code) - exact, since e >= -5 keeps it a normal e4m3 number - into
-// the same 128-byte-swizzled operand tile the e4m3 instantiation loads by TMA.
-// The MMA, the scales and the epilogue are the e4m3 instantiation's.
+// the e4m3 bytes and multiplies them on the block-scaled tensor-core path:
+// the TMA unpacks a 128 x 128 tile of packed codes into the padded layout
+// tcgen05.mma kind::mxf8f6f4 reads for E2M1 operands (16 codes in the low 8
+// bytes of each 16-byte chunk, 128-byte swizzled like an e4m3 tile), a bulk
+// copy brings the tile's 512-byte chunk of UE8M0 block scale factors, and the
+// MMA thread moves the chunk into TMEM (tcgen05.cp, 32 x 128 bits replicated
+// to the four lane quadrants: row 32 j + i of the tile at lane 32 j + i,
+// column j, byte = block) before the four block-scaled MMAs of the slice.
+// The hidden states' scale factors are all 1 (their float32 per-token scale
+// is applied in the epilogue, as in the e4m3 instantiation); the hardware
+// reads them at lane n % 32, column n / 32, so eight columns of 0x7F cover
+// any token tile. Each product 2^e value(code) x code(h) is exact and
+// accumulated in float32, so the arithmetic is the same as widening the codes
+// to e4m3, without any widening work on the SMs.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -58,13 +63,14 @@ constexpr int kBM = kVocabTile;     // 128 vocabulary rows per tile (MMA M, TMEM
 constexpr int kBK = 64;             // bf16 hidden elements per stage: 128 bytes
 constexpr int kBKBytes = 128;       // bytes of one K slice of a row, either element type
 constexpr int kThreads = 192;
-constexpr int kThreadsW4 = 448;     // + eight converter warps
-constexpr int kConvWarps = 8;
-constexpr int kMaxRawSlots = 12;
-constexpr int kW4TileRows = kW4TileBytes / 128;  // 68
-constexpr int kRawBytes = 9216;     // one w4 tile (8,704 bytes) rounded up to 1 KB
 enum { kFmtBf16 = 0, kFmtE4m3 = 1, kFmtW4 = 2 };
 constexpr int kMaxNt = 256;
+// w4: token tiles of at most 224 columns leave room in TMEM (512 columns) for
+// the two accumulators, the hidden side's 8 scale columns and 4 scale
+// columns per stage for the weights
+constexpr int kMaxNtW4 = 224;
+constexpr int kSfbCols = 8;
+constexpr int kSfaSlot = 8;   // TMEM columns per stage's weight scale factors (4 used)
 constexpr uint64_t kDrainNs = 200000000ull;  // budget of the drain after an abort
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kNegBig = -1.0e30f;          // logit of a vocabulary row beyond V
@@ -80,13 +86,14 @@ struct TcArgs {
   float* z_tgt;
   const float* w_scale;  // e4m3: [V] per vocabulary row
   const float* h_scale;  // e4m3: [N] per token
-  const uint8_t* w4;     // w4: tiled codes and exponents
+  const uint8_t* w4_sf;  // w4: the scale-factor region, one 512-byte chunk per tile
   int* status;
   int N, T, V, D;
   int Nt, n_tt, units, nkb, stages, vtiles;
-  int raw_slots;         // w4: 4-bit weight tiles in flight
-  int a_slots;           // w4: widened weight tiles
   uint32_t tmem_cols;
+  uint32_t buf_cols;     // columns of one accumulator
+  uint32_t sfb_col;      // w4: the hidden side's scale factors (all 1)
+  uint32_t sfa_col;      // w4: the weight scale factors, kSfaSlot columns per stage
   uint64_t wait_ns;  // budget of one bounded wait (jet_set_wait_budget_ns)
   int hold_first;    // test hook (jet_set_test_stall): withhold the first stage's loads
 };
@@ -133,64 +140,80 @@ constexpr uint32_t idesc_e4m3_f32(int M, int N) {
   return (1u << 4) | (uint32_t(N >> 3) << 17) | (uint32_t(M >> 4) << 24);
 }
 
-// Widen blocks 2 h and 2 h + 1 of row r of a landed w4 tile into the e4m3
-// operand tile (128-byte swizzle: row r at (r / 8) KB + (r % 8) 128 B, 16-byte
-// chunk j in slot j ^ (r % 8)). Per 32-element block: the e4m3 codes of
-// 2^e x {0, .5, 1, 1.5, 2, 3, 4, 6} are ((e + 7) << 3) + {-, -8, 0, 4, 8, 12,
-// 16, 20} (0 for the zero code), an 8-entry byte table that prmt indexes by
-// the 3 magnitude bits of 4 nibbles at a time. The stored sign bits are
-// permuted so that the word's bits 7, 15, 23, 31 are the signs of its
-// elements 0..3 and bits 3, 11, 19, 27 those of elements 4..7.
-__device__ __forceinline__ void widen_w4_row(const uint8_t* raw, uint8_t* A, int r, int h) {
-  const uint32_t ex = *reinterpret_cast<const uint32_t*>(raw + kW4CodeBytes + r * 4);
-  uint8_t* row = A + (r >> 3) * 1024 + (r & 7) * 128;
-#pragma unroll
-  for (int c = 2 * h; c < 2 * h + 2; ++c) {
-    const uint4 q = *reinterpret_cast<const uint4*>(raw + r * 64 + 16 * (c ^ ((r >> 1) & 3)));
-    const uint32_t base = uint32_t(int(int8_t(uint8_t(ex >> (8 * c)))) + 7) << 3;
-    // bytes {0, base - 8, base, base + 4} and {base + 8, + 12, + 16, + 20}
-    const uint32_t lo = base * 0x01010100u + 0x03FFF800u;
-    const uint32_t hi = base * 0x01010101u + 0x14100C08u;
-    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
-    uint32_t o[8];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const uint32_t m = w[i] & 0x77777777u;
-      o[2 * i] = __byte_perm(lo, hi, m) | (w[i] & 0x80808080u);
-      o[2 * i + 1] = __byte_perm(lo, hi, m >> 16) | ((w[i] << 4) & 0x80808080u);
-    }
-    *reinterpret_cast<uint4*>(row + 16 * ((2 * c) ^ (r & 7))) = make_uint4(o[0], o[1], o[2], o[3]);
-    *reinterpret_cast<uint4*>(row + 16 * ((2 * c + 1) ^ (r & 7))) =
-        make_uint4(o[4], o[5], o[6], o[7]);
-  }
+// D (+)= (A x sf_A) (B x sf_B)^T with A E2M1 codes and B e4m3 codes in shared
+// memory, one UE8M0 scale factor per 32-element block of K in TMEM (K = 32:
+// the instruction descriptor's scale-factor ids pick the byte)
+__device__ __forceinline__ void mma_mx(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                       uint32_t idesc, uint32_t sfa_tmem, uint32_t sfb_tmem,
+                                       uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %6, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X "
+      "[%0], %1, %2, %3, [%4], [%5], p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(sfa_tmem), "r"(sfb_tmem), "r"(accumulate)
+      : "memory");
+}
+
+// Instruction descriptor of kind::mxf8f6f4 with block scaling: A E2M1
+// (format 5), B e4m3 (format 0), both K-major, UE8M0 scale factors, shape
+// M x N; block `k` of the 4 in a scale-factor word for both operands.
+__host__ __device__ constexpr uint32_t idesc_mx_e2m1_e4m3(int M, int N, int k) {
+  return (uint32_t(k) << 4) | (5u << 7) | (0u << 10) | (uint32_t(N >> 3) << 17) | (1u << 23) |
+         (uint32_t(M >> 4) << 24) | (uint32_t(k) << 29);
+}
+
+// A 32 x 16-byte matrix in shared memory (rows 16 bytes apart) into TMEM,
+// replicated to all four 32-lane quadrants: row i at lane 32 q + i, its four
+// 32-bit words in columns taddr .. taddr + 3.
+__device__ __forceinline__ void tmem_cp_32x128(uint32_t taddr, uint32_t smem_addr) {
+  uint64_t d = 0;
+  d |= uint64_t((smem_addr >> 4) & 0x3FFFu);  // start address
+  d |= uint64_t(1) << 16;                     // leading byte offset (one 16-byte column)
+  d |= uint64_t(128 >> 4) << 32;              // stride byte offset: 8 rows x 16 bytes
+  d |= uint64_t(1) << 46;                     // descriptor version (sm_100 family)
+  asm volatile("tcgen05.cp.cta_group::1.32x128b.warpx4 [%0], %1;" ::"r"(taddr), "l"(d)
+               : "memory");
+}
+
+// untiled bulk copy global -> shared memory, completing `bytes` on `bar`
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes,
+                                          uint64_t* bar, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1], %2, [%3], %4;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_8cols(uint32_t taddr, uint32_t v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %1, %1, %1, %1, %1, %1, %1};" ::"r"(taddr),
+      "r"(v)
+      : "memory");
 }
 
 template <int FMT>
-__global__ void __launch_bounds__(FMT == kFmtW4 ? kThreadsW4 : kThreads, 1)
+__global__ void __launch_bounds__(kThreads, 1)
 lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmH,
                  const TcArgs a) {
-  constexpr bool F8 = FMT != kFmtBf16;   // e4m3 operands in the MMA
-  constexpr bool W4 = FMT == kFmtW4;     // weights widened on chip from 4-bit codes
+  constexpr bool F8 = FMT != kFmtBf16;   // 8-bit hidden codes in the MMA
+  constexpr bool W4 = FMT == kFmtW4;     // 4-bit weights, block-scaled MMA
   constexpr int kBKe = F8 ? kBKBytes : kBK;  // elements of one K slice
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   const uint32_t a_bytes = kBM * 128, b_bytes = uint32_t(a.Nt) * 128;
-  // a stage holds the weight and hidden tiles of one K slice; for w4 it holds
-  // the hidden tile only, the weights going through the rings after it
-  const uint32_t stage_bytes = W4 ? b_bytes : a_bytes + b_bytes;
-  uint8_t* aring = smem + size_t(a.stages) * stage_bytes;             // w4: widened tiles
-  uint8_t* rawb = aring + (W4 ? size_t(a.a_slots) * a_bytes : 0);     // w4: 4-bit tiles
-  float2* red = reinterpret_cast<float2*>(rawb + (W4 ? size_t(a.raw_slots) * kRawBytes : 0));
+  // a stage holds the weight and hidden tiles of one K slice (w4: the weight
+  // tile as the TMA unpacks it, 1 byte per code) and, for w4, the slice's
+  // 512-byte scale-factor chunk (in a 1 KB slot, keeping stages 1 KB aligned)
+  const uint32_t stage_bytes = a_bytes + b_bytes + (W4 ? 1024u : 0u);
+  float2* red = reinterpret_cast<float2*>(smem + size_t(a.stages) * stage_bytes);
   int4* hits = reinterpret_cast<int4*>(red + 4 * kMaxNt);                          // [128]
   float* hs = reinterpret_cast<float*>(hits + 128);                                // [256]
   uint64_t* full = reinterpret_cast<uint64_t*>(hs + kMaxNt);
   uint64_t* empty = full + a.stages;
-  uint64_t* conv = empty + a.stages;     // w4: a widened tile is ready
-  uint64_t* aempty = conv + a.a_slots;   // w4: ... has been consumed by its MMAs
-  uint64_t* raw_full = aempty + a.a_slots;  // w4: a 4-bit tile has landed
-  uint64_t* raw_empty = raw_full + a.raw_slots;  // w4: ... has been widened
-  uint64_t* tfull = raw_empty + a.raw_slots;
+  uint64_t* tfull = empty + a.stages;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
@@ -203,14 +226,6 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
     for (int s = 0; s < a.stages; ++s) {
       mbar_init(full + s, 1);
       mbar_init(empty + s, 1);
-    }
-    for (int s = 0; s < a.a_slots; ++s) {
-      mbar_init(conv + s, kConvWarps);
-      mbar_init(aempty + s, 1);
-    }
-    for (int s = 0; s < a.raw_slots; ++s) {
-      mbar_init(raw_full + s, 1);
-      mbar_init(raw_empty + s, kConvWarps);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(tfull + b, 1);
@@ -235,68 +250,31 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const uint32_t buf_cols = a.tmem_cols / 2;
+  const uint32_t buf_cols = a.buf_cols;
+  if (W4) {
+    // the hidden side's scale factors: 1 (UE8M0 127) in every byte the MMA
+    // may read, written once by the epilogue warps (each to its lane quadrant)
+    if (warp >= 2) {
+      tmem_st_8cols(tmem_base + (uint32_t(32 * (warp & 3)) << 16) + a.sfb_col, 0x7F7F7F7Fu);
+      tmem_wait_st();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+  }
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
-    if (lane == 0 && W4) {
-      // per K slice, in order: the 4-bit weight tile into its ring, then the
-      // hidden tile into the stage
+    if (lane == 0) {
       const uint64_t pol_w = policy_evict_first(), pol_h = policy_evict_last();
-      int s = 0, sr = 0;
-      uint32_t ph = 0, rph = 0, issued = 0, issued_par = 0, rissued = 0, rissued_par = 0;
-      bool ok = true, hold = a.hold_first != 0;
-      for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-        const int vt = u / a.n_tt, t0 = (u % a.n_tt) * a.Nt;
-        for (int kb = 0; kb < a.nkb; ++kb) {
-          if (!mbar_wait(raw_empty + sr, rph ^ 1u, a.wait_ns, abort_flag)) {
-            ok = false;
-            break;
-          }
-          // the tile is 68 rows of 128 bytes of the w4 buffer's 2-D view
-          mbar_arrive_expect_tx(raw_full + sr, kW4TileBytes);
-          tma_load_2d(rawb + size_t(sr) * kRawBytes, &tmW, raw_full + sr, 0,
-                      (vt * a.nkb + kb) * kW4TileRows, pol_w);
-          rissued |= 1u << sr;
-          rissued_par = (rissued_par & ~(1u << sr)) | (rph << sr);
-          if (++sr == a.raw_slots) {
-            sr = 0;
-            rph ^= 1u;
-          }
-          if (!mbar_wait(empty + s, ph ^ 1u, a.wait_ns, abort_flag)) {
-            ok = false;
-            break;
-          }
-          if (hold) {
-            hold = false;  // test hook: this stage never fills
-          } else {
-            mbar_arrive_expect_tx(full + s, b_bytes);
-            tma_load_2d(smem + size_t(s) * stage_bytes, &tmH, full + s, kb * kBKe, t0, pol_h);
-            issued |= 1u << s;
-            issued_par = (issued_par & ~(1u << s)) | (ph << s);
-          }
-          if (++s == a.stages) {
-            s = 0;
-            ph ^= 1u;
-          }
-        }
-      }
-      if (!ok) {
-        *abort_flag = 1;
-        flag(a.status, JET_ERR_TIMEOUT);
-        for (int t = 0; t < a.raw_slots; ++t)
-          if (rissued & (1u << t))
-            mbar_wait(raw_full + t, (rissued_par >> t) & 1u, kDrainNs, nullptr);
-        for (int t = 0; t < a.stages; ++t)
-          if (issued & (1u << t)) mbar_wait(full + t, (issued_par >> t) & 1u, kDrainNs, nullptr);
-      }
-    } else if (lane == 0) {
-      const uint64_t pol_w = policy_evict_first(), pol_h = policy_evict_last();
+      // the weight bytes one stage brings: bf16 or e4m3 tile, or packed
+      // 4-bit codes (half the unpacked tile) and their scale-factor chunk
+      const uint32_t w_tx = W4 ? a_bytes / 2 + kW4ScaleBytes : a_bytes;
       int s = 0;
       uint32_t ph = 0, issued = 0, issued_par = 0;
       bool ok = true, hold = a.hold_first != 0;
       for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-        const int v0 = (u / a.n_tt) * kBM, t0 = (u % a.n_tt) * a.Nt;
+        const int vt = u / a.n_tt, v0 = vt * kBM, t0 = (u % a.n_tt) * a.Nt;
         for (int kb = 0; kb < a.nkb; ++kb) {
           if (!mbar_wait(empty + s, ph ^ 1u, a.wait_ns, abort_flag)) {
             ok = false;
@@ -306,9 +284,13 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
           if (hold) {
             hold = false;  // test hook: this stage never fills
           } else {
-            mbar_arrive_expect_tx(full + s, stage_bytes);
+            mbar_arrive_expect_tx(full + s, w_tx + b_bytes);
             tma_load_2d(sa, &tmW, full + s, kb * kBKe, v0, pol_w);
             tma_load_2d(sa + a_bytes, &tmH, full + s, kb * kBKe, t0, pol_h);
+            if (W4)
+              bulk_load(sa + a_bytes + b_bytes,
+                        a.w4_sf + (size_t(vt) * a.nkb + kb) * kW4ScaleBytes, kW4ScaleBytes,
+                        full + s, pol_w);
             issued |= 1u << s;
             issued_par = (issued_par & ~(1u << s)) | (ph << s);
           }
@@ -330,8 +312,8 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       const uint32_t idesc = F8 ? idesc_e4m3_f32(kBM, a.Nt) : idesc_bf16_f32(kBM, a.Nt);
-      int s = 0, local = 0, ia = 0;
-      uint32_t ph = 0, aph = 0;
+      int s = 0, local = 0;
+      uint32_t ph = 0;
       bool ok = true;
       for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x, ++local) {
         const int buf = local & 1;
@@ -343,36 +325,39 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + buf * buf_cols;
         for (int kb = 0; kb < a.nkb; ++kb) {
-          if (!mbar_wait(full + s, ph, a.wait_ns, abort_flag) ||
-              (W4 && !mbar_wait(conv + ia, aph, a.wait_ns, abort_flag))) {
+          if (!mbar_wait(full + s, ph, a.wait_ns, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t ss = smem_u32(smem + size_t(s) * stage_bytes);
-          const uint32_t sa = W4 ? smem_u32(aring + size_t(ia) * a_bytes) : ss;
-          const uint32_t sb = W4 ? ss : ss + a_bytes;
-          // 32 bytes of K per instruction: 16 bf16 or 32 e4m3 elements
+          const uint32_t sa = smem_u32(smem + size_t(s) * stage_bytes);
+          const uint32_t sb = sa + a_bytes;
+          if (W4) {
+            // the slice's weight scale factors into this stage's 4 columns;
+            // the MMAs after it in this thread's order read them
+            const uint32_t sfa = tmem_base + a.sfa_col + kSfaSlot * s;
+            tmem_cp_32x128(sfa, sb + b_bytes);
 #pragma unroll
-          for (int k = 0; k < kBKBytes / 32; ++k) {
-            if (F8)
-              mma_e4m3(d_tmem, desc_k_sw128(sa + 32 * k), desc_k_sw128(sb + 32 * k), idesc,
-                       (kb | k) != 0);
-            else
-              mma_f16(d_tmem, desc_k_sw128(sa + 32 * k), desc_k_sw128(sb + 32 * k), idesc,
-                      (kb | k) != 0);
+            for (int k = 0; k < 4; ++k)
+              mma_mx(d_tmem, desc_k_sw128(sa + 32 * k), desc_k_sw128(sb + 32 * k),
+                     idesc_mx_e2m1_e4m3(kBM, a.Nt, k), sfa, tmem_base + a.sfb_col,
+                     (kb | k) != 0);
+          } else {
+            // 32 bytes of K per instruction: 16 bf16 or 32 e4m3 elements
+#pragma unroll
+            for (int k = 0; k < kBKBytes / 32; ++k) {
+              if (F8)
+                mma_e4m3(d_tmem, desc_k_sw128(sa + 32 * k), desc_k_sw128(sb + 32 * k), idesc,
+                         (kb | k) != 0);
+              else
+                mma_f16(d_tmem, desc_k_sw128(sa + 32 * k), desc_k_sw128(sb + 32 * k), idesc,
+                        (kb | k) != 0);
+            }
           }
           mma_commit(empty + s);  // frees the stage once these MMAs have read it
           if (++s == a.stages) {
             s = 0;
             ph ^= 1u;
-          }
-          if (W4) {
-            mma_commit(aempty + ia);  // ... and the widened tile
-            if (++ia == a.a_slots) {
-              ia = 0;
-              aph ^= 1u;
-            }
           }
         }
         if (!ok) break;
@@ -384,47 +369,6 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
         mma_commit(drain);
         mbar_wait(drain, 0, kDrainNs, nullptr);
       }
-    }
-  } else if (W4 && warp >= 6) {
-    // ------------------------------------------------------------ w4 converter
-    const int r = (threadIdx.x - 192) & (kBM - 1);  // vocabulary row of the tile
-    const int hh = (threadIdx.x - 192) >> 7;         // which half of the K slice
-    int ia = 0, slot = 0;
-    uint32_t aph = 0, rph = 0;
-    bool ok = true;
-    for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
-      for (int kb = 0; kb < a.nkb; ++kb) {
-        // one lane waits for the tile and the free slot; __syncwarp orders the
-        // other lanes' reads and writes after its wait
-        bool got = true;
-        if (lane == 0)
-          got = mbar_wait(raw_full + slot, rph, a.wait_ns, abort_flag) &&
-                mbar_wait(aempty + ia, aph ^ 1u, a.wait_ns, abort_flag);
-        if (!__shfl_sync(0xffffffffu, got, 0)) {
-          ok = false;
-          break;
-        }
-        __syncwarp();
-        widen_w4_row(rawb + size_t(slot) * kRawBytes, aring + size_t(ia) * a_bytes, r, hh);
-        fence_proxy_async_shared();  // the widened tile is read by the tensor core
-        __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(conv + ia);
-          mbar_arrive(raw_empty + slot);
-        }
-        if (++ia == a.a_slots) {
-          ia = 0;
-          aph ^= 1u;
-        }
-        if (++slot == a.raw_slots) {
-          slot = 0;
-          rph ^= 1u;
-        }
-      }
-    }
-    if (!ok) {
-      *abort_flag = 1;
-      if (lane == 0) flag(a.status, JET_ERR_TIMEOUT);
     }
   } else {
     // ------------------------------------------------------------ epilogue
@@ -569,16 +513,19 @@ bool encode_kmajor(CUtensorMap* map, const void* base, int rows, int D, int box_
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// the tiled w4 buffer as a [tiles * 68, 128] byte matrix, one tile per box
-bool encode_w4_tiles(CUtensorMap* map, const void* base, int tiles) {
+// the 4-bit code region [rows, kd] (kd codes per row, two per byte, element
+// 2 j in the low nibble of byte j; kd a multiple of 128): boxes of 128 codes x
+// 128 rows, unpacked by the TMA to one byte per code (16 codes in the low 8
+// bytes of each 16-byte chunk), 128-byte swizzled
+bool encode_w4_codes(CUtensorMap* map, const void* base, int rows, int kd) {
   auto fn = encode_fn();
   if (!fn) return false;
-  const cuuint64_t dims[2] = {128, cuuint64_t(tiles) * kW4TileRows};
-  const cuuint64_t strides[1] = {128};
-  const cuuint32_t box[2] = {128, cuuint32_t(kW4TileRows)};
+  const cuuint64_t dims[2] = {cuuint64_t(kd), cuuint64_t(rows)};
+  const cuuint64_t strides[1] = {cuuint64_t(kd) / 2};
+  const cuuint32_t box[2] = {128, cuuint32_t(kBM)};
   const cuuint32_t estr[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(base), dims, strides, box,
-            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_16U4_ALIGN16B, 2, const_cast<void*>(base), dims, strides,
+            box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -594,14 +541,15 @@ int sm_count() {
 namespace {
 
 // one launch of the LM head on bf16 operands, or e4m3 hidden codes with e4m3
-// or tiled 4-bit weights, per-row weight scales and per-token hidden scales
+// or block-scaled 4-bit weights, per-row weight scales and per-token hidden scales
 template <int FMT>
 cudaError_t launch_head(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
                         const void* hidden, const float* h_scale, const void* w_lm,
                         const float* w_scale, void* ws, int* status, cudaStream_t st) {
   constexpr bool F8 = FMT != kFmtBf16, W4 = FMT == kFmtW4;
   const jet_sizes& n = lay.n;
-  int n_tt = (n.N + kMaxNt - 1) / kMaxNt;
+  const int max_nt = W4 ? kMaxNtW4 : kMaxNt;
+  int n_tt = (n.N + max_nt - 1) / max_nt;
   const int Nt = ((n.N + n_tt - 1) / n_tt + 15) / 16 * 16;
   n_tt = (n.N + Nt - 1) / Nt;
   const int esize = F8 ? 1 : 2;
@@ -617,7 +565,6 @@ cudaError_t launch_head(const jet_layout& lay, const jet_dims& d, const ScorePla
   a.z_tgt = reinterpret_cast<float*>(base + plan.ztgt_off);
   a.w_scale = w_scale;
   a.h_scale = h_scale;
-  a.w4 = W4 ? static_cast<const uint8_t*>(w_lm) : nullptr;
   a.status = status;
   a.N = n.N;
   a.T = n.T;
@@ -628,29 +575,33 @@ cudaError_t launch_head(const jet_layout& lay, const jet_dims& d, const ScorePla
   a.units = plan.vtiles * n_tt;
   a.vtiles = plan.vtiles;
   a.nkb = (d.D * esize + kBKBytes - 1) / kBKBytes;
-  a.tmem_cols = Nt <= 128 ? 256 : 512;
   const int a_bytes = kBM * kBKBytes, b_bytes = Nt * kBKBytes;
-  int room = kSmemLimit - 1024 - kFixedSmem;
-  int stage_bytes = a_bytes + b_bytes;
-  a.raw_slots = a.a_slots = 0;
+  const int stage_bytes = a_bytes + b_bytes + (W4 ? 1024 : 0);
+  a.stages = std::min(8, (kSmemLimit - 1024 - kFixedSmem) / stage_bytes);
+  if (a.stages < 2) return cudaErrorInvalidValue;
   if (W4) {
-    // two widened tiles; the rest split between hidden tiles and 4-bit tiles
-    stage_bytes = b_bytes;
-    a.a_slots = 2;
-    room -= a.a_slots * a_bytes;
-    a.stages = std::min(8, room / (b_bytes + kRawBytes));
-    a.raw_slots = std::min(kMaxRawSlots, (room - a.stages * b_bytes) / kRawBytes);
-    if (a.stages < 2 || a.raw_slots < 2) return cudaErrorInvalidValue;
+    // accumulators at columns 0 and buf_cols, then the hidden side's scale
+    // factors, then the weight scale factors (a slot of 8 columns per stage)
+    a.buf_cols = uint32_t(Nt + 31) / 32 * 32;
+    a.sfb_col = 2 * a.buf_cols;
+    a.sfa_col = a.sfb_col + kSfbCols;
+    a.tmem_cols = 512;
+    while (a.stages > 2 && a.sfa_col + kSfaSlot * a.stages > a.tmem_cols) --a.stages;
+    if (a.sfa_col + kSfaSlot * a.stages > a.tmem_cols) return cudaErrorInvalidValue;
   } else {
-    a.stages = std::min(8, room / stage_bytes);
+    a.tmem_cols = Nt <= 128 ? 256 : 512;
+    a.buf_cols = a.tmem_cols / 2;
   }
-  const size_t smem = 1024 + size_t(a.stages) * stage_bytes + size_t(a.a_slots) * a_bytes +
-                      size_t(a.raw_slots) * kRawBytes + kFixedSmem;
+  const size_t smem = 1024 + size_t(a.stages) * stage_bytes + kFixedSmem;
 
   CUtensorMap tmW, tmH;
   if (!encode_kmajor(&tmH, hidden, n.N, d.D, Nt, esize)) return cudaErrorInvalidValue;
   if (W4) {
-    if (!encode_w4_tiles(&tmW, w_lm, plan.vtiles * a.nkb)) return cudaErrorInvalidValue;
+    // the code region covers whole tiles: ceil(V / 128) * 128 rows of
+    // ceil(D / 128) * 128 codes; the scale-factor region follows it
+    const int rows = plan.vtiles * kBM, kd = a.nkb * 128;
+    if (!encode_w4_codes(&tmW, w_lm, rows, kd)) return cudaErrorInvalidValue;
+    a.w4_sf = static_cast<const uint8_t*>(w_lm) + size_t(rows) * (kd / 2);
   } else if (!encode_kmajor(&tmW, w_lm, n.V, d.D, kBM, esize)) {
     return cudaErrorInvalidValue;
   }
@@ -660,7 +611,7 @@ cudaError_t launch_head(const jet_layout& lay, const jet_dims& d, const ScorePla
   int sms = sm_count();
   if (d.max_sms > 0) sms = std::min(sms, d.max_sms);
   const int grid = std::max(1, std::min(a.units, sms));
-  return launch_pdl(lmhead_tc_kernel<FMT>, dim3(grid), dim3(W4 ? kThreadsW4 : kThreads), smem, st,
+  return launch_pdl(lmhead_tc_kernel<FMT>, dim3(grid), dim3(kThreads), smem, st,
                     tmW, tmH, a);
 }
 

@@ -10,8 +10,10 @@
 // 32-element block, a power-of-two exponent e in [-5, 0] over OCP FP4 E2M1
 // codes: s = amax / 6, inv = 6 / amax, t = blockmax * inv, e = the smallest
 // value in [-5, 0] with t <= 6 * 2^e (0 if none), code = e2m1(x * (inv * 2^-e))
-// rounded to nearest even and saturated at +-6. They are written in the
-// tiled layout the LM head streams (see include/jet.h).
+// rounded to nearest even and saturated at +-6. They are written as the
+// block-scaled LM head reads them (include/jet.h): a row-major region of
+// packed codes, then one 512-byte chunk of UE8M0 factors 127 + e per
+// (128-row tile, 128-code slice).
 #include <cuda_fp8.h>
 
 #include "jet_device.cuh"
@@ -96,7 +98,8 @@ quantize_w4_kernel(const __nv_bfloat16* __restrict__ x, int V, int D, int rows_p
   }
   const float inv = amax > 0.f ? __fdiv_rn(6.f, amax) : 0.f;
   const int r = v & (kVocabTile - 1), vt = v / kVocabTile;
-  const int c = lane >> 3;  // the 32-element block (16-byte chunk) of the slice
+  const int c = lane >> 3;  // the 32-element block of the slice
+  const size_t sf_off = size_t(rows_pad) * nkb * 64;  // the scale factors follow the codes
   for (int kb = 0; kb < nkb; ++kb) {
     const int k = kb * 128 + lane * 4;
     float f[4] = {0.f, 0.f, 0.f, 0.f};
@@ -116,35 +119,18 @@ quantize_w4_kernel(const __nv_bfloat16* __restrict__ x, int V, int D, int rows_p
     for (int ee = 0; ee >= -5; --ee, thr *= 0.5f)
       if (t <= thr) e = ee;
     const float inv_b = __fmul_rn(inv, __int_as_float((127 - e) << 23));  // inv * 2^-e, exact
-    // magnitudes (3 bits) and signs of this lane's 4 elements; a 32-bit word
-    // of the tile holds 8 elements (this lane and its odd/even partner), and
-    // the sign bit of nibble k belongs to element 4 + k / 2 (k even) or k / 2
-    // (k odd) of the word, so that the LM head's widening finds every sign
-    // one shift away from bit 7 of the output byte
-    uint32_t mag = 0, sgn = 0;
+    // four codes, element 2 j in the low nibble of byte j
+    uint32_t code = 0;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const uint32_t cd = e2m1_code(__fmul_rn(f[i], inv_b));
-      mag |= (cd & 7u) << (4 * i);
-      sgn |= (cd >> 3) << i;
-    }
-    const uint32_t psg = __shfl_xor_sync(0xffffffffu, sgn, 1);
-    const bool odd = lane & 1;
-    // even lane (elements 0..3 of the word): nibble signs p0, o0, p1, o1;
-    // odd lane (elements 4..7): o2, p2, o3, p3 (o = own, p = partner)
-    const uint32_t s4 = odd ? ((sgn >> 2) & 1u) | (((psg >> 2) & 1u) << 1) |
-                                  (((sgn >> 3) & 1u) << 2) | (((psg >> 3) & 1u) << 3)
-                            : (psg & 1u) | ((sgn & 1u) << 1) | (((psg >> 1) & 1u) << 2) |
-                                  (((sgn >> 1) & 1u) << 3);
-    uint32_t code = mag;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) code |= ((s4 >> i) & 1u) << (4 * i + 3);
-    uint8_t* tile = w4 + (size_t(vt) * nkb + kb) * kW4TileBytes;
-    // chunk c of row r sits in slot c ^ ((r >> 1) & 3): the converter's
-    // 16-byte reads of 8 consecutive rows then hit 8 different bank groups
-    *reinterpret_cast<uint16_t*>(tile + r * 64 + 16 * (c ^ ((r >> 1) & 3)) + 2 * (lane & 7)) =
+    for (int i = 0; i < 4; ++i) code |= e2m1_code(__fmul_rn(f[i], inv_b)) << (4 * i);
+    *reinterpret_cast<uint16_t*>(w4 + size_t(v) * (nkb * 64) + kb * 64 + 2 * lane) =
         uint16_t(code);
-    if ((lane & 7) == 0) tile[kW4CodeBytes + r * 4 + c] = uint8_t(int8_t(e));
+    // the block's exponent as a UE8M0 scale factor, in the order one
+    // tcgen05.cp (32 x 128 bits) brings a 512-byte chunk into TMEM: row
+    // 32 j + i of the tile, block c of the slice at byte 16 i + 4 j + c
+    if ((lane & 7) == 0)
+      w4[sf_off + (size_t(vt) * nkb + kb) * 512 + 16 * (r & 31) + 4 * (r >> 5) + c] =
+          uint8_t(127 + e);
   }
 }
 

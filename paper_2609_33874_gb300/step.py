@@ -98,7 +98,7 @@ def quantize_lm_head(w_lm: torch.Tensor, stream=None):
 
 
 def quantize_lm_head_w4(w_lm: torch.Tensor, stream=None):
-    """Tiled 4-bit codes (uint8, jet_w4_bytes(V, D) bytes) and per-row float32
+    """4-bit codes and block scale factors (uint8, jet_w4_bytes(V, D) bytes) and per-row float32
     scales [V] of the bf16 LM-head weights (jet_quantize_w4), for a step built
     with lm="w4"."""
     V, D = w_lm.shape

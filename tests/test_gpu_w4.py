@@ -1,7 +1,7 @@
 """GPU parity of the 4-bit (w4) LM head through the C ABI: the quantiser's
 codes, block exponents and scales against the oracle's own quantisation of the
-same bf16 weights (bit-exact, after undoing the tiled layout the library
-documents), and token log-probabilities / candidate scores against the
+same bf16 weights (bit-exact, after reading back the code and scale-factor
+layout the library documents), and token log-probabilities / candidate scores against the
 oracle's 4-bit model (each side quantises the weights and hidden states
 itself)."""
 import dataclasses
@@ -32,26 +32,22 @@ def _bf16_device(x32):
 
 
 def untile(buf, V, D):
-    """(codes [Vp, Kp] 0..15, exps [Vp, Kp / 32] int8) from the tiled layout:
-    tile (vt, kb) of 8,704 bytes; row r's 16-byte chunk c in slot
-    c ^ ((r >> 1) & 3); 32-bit words of 8 elements whose nibble k holds element
-    k's magnitude and the sign of element 4 + k / 2 (k even) or k / 2 (k odd);
-    then the rows' four block exponents."""
+    """(codes [Vp, Kp] 0..15, exps [Vp, Kp / 32] int8) from the documented
+    layout: a row-major code region of Vp = 128 ceil(V / 128) rows of
+    Kp = 128 ceil(D / 128) codes, element 2 j of a row in the low nibble of its
+    byte j; then one 512-byte chunk of UE8M0 scale factors per (vocabulary
+    tile vt, K slice kb), chunk index vt * ceil(D / 128) + kb, holding row
+    32 j + i of the tile's factor for block c of the slice at byte
+    16 i + 4 j + c (factor = 127 + e)."""
     nvt, nkb = -(-V // 128), -(-D // 128)
-    t = np.asarray(buf, dtype=np.uint8).reshape(nvt, nkb, 8704)
-    chunks = t[:, :, :8192].reshape(nvt, nkb, 128, 4, 16)
-    r = np.arange(128)
-    logical = np.stack([chunks[:, :, r, c ^ ((r >> 1) & 3), :] for c in range(4)], axis=3)
-    by = logical.reshape(nvt, nkb, 128, 64)
-    nib = np.stack([by & 15, by >> 4], axis=-1).reshape(nvt, nkb, 128, 16, 8)  # words x nibbles
-    # the sign of element j of a word is bit 3 of nibble 2 j + 1 (j < 4) or
-    # 2 (j - 4) (j >= 4)
-    where = np.array([1, 3, 5, 7, 0, 2, 4, 6])
-    nib = (nib & 7) | (nib[..., where] & 8)
-    nib = nib.reshape(nvt, nkb, 128, 128)
-    codes = nib.transpose(0, 2, 1, 3).reshape(nvt * 128, nkb * 128)
-    exps = t[:, :, 8192:].view(np.int8).reshape(nvt, nkb, 128, 4)
-    exps = exps.transpose(0, 2, 1, 3).reshape(nvt * 128, nkb * 4)
+    Vp, Kp = nvt * 128, nkb * 128
+    b = np.asarray(buf, dtype=np.uint8)
+    assert b.size == Vp * Kp // 2 + nvt * nkb * 512
+    by = b[:Vp * Kp // 2].reshape(Vp, Kp // 2)
+    codes = np.stack([by & 15, by >> 4], axis=-1).reshape(Vp, Kp)
+    sf = b[Vp * Kp // 2:].reshape(nvt, nkb, 32, 4, 4)          # [vt, kb, i, j, c]
+    e = sf.astype(np.int16) - 127
+    exps = e.transpose(0, 3, 2, 1, 4).reshape(Vp, nkb * 4).astype(np.int8)  # row 32 j + i
     return codes, exps
 
 
