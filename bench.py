@@ -249,7 +249,9 @@ def step_config(args, problem, world: int) -> dict:
                 lm_head={"bf16": "bf16",
                          "e4m3": "e4m3, one float32 scale per weight row and per token",
                          "w4": "weights e2m1 with a power-of-two exponent per 32-element "
-                               "block and a float32 scale per row; hidden e4m3 per token"}[args.lm],
+                               "block and a float32 scale per row; hidden e4m3 per token",
+                         "mxfp8": "weights and hidden states e4m3 with a shared power-of-two "
+                                  "scale per 32-element block (MXFP8)"}[args.lm],
                 recurrence=(args.rule if w.Hl else None),
                 l2=f"inputs larger than L2: LM-head weights {w.V * w.D * es / 1e9:.2f} GB "
                    f"streamed every step")
@@ -374,8 +376,10 @@ def _measure(args, problem, dev, stream, peaks, world=1, src=None, w_lm=None, cl
         w_lm = jet_synth.torch_tensor(problem, "w_lm", device=dev)
         if low:
             # model state: the weights are quantised once, outside the timed region
-            from paper_2609_33874_gb300.step import quantize_lm_head, quantize_lm_head_w4
-            w_lm = (quantize_lm_head_w4 if args.lm == "w4" else quantize_lm_head)(w_lm)
+            from paper_2609_33874_gb300.step import (quantize_lm_head, quantize_lm_head_mxfp8,
+                                                     quantize_lm_head_w4)
+            w_lm = {"w4": quantize_lm_head_w4, "e4m3": quantize_lm_head,
+                    "mxfp8": quantize_lm_head_mxfp8}[args.lm](w_lm)
             torch.cuda.synchronize(dev)
 
     # the per-call breakdown (taken outside the timed steps): attend | fork | score | decide
@@ -496,8 +500,13 @@ def _measure(args, problem, dev, stream, peaks, world=1, src=None, w_lm=None, cl
     if low:
         # w_lm codes (+ block exponents for w4) + row scales, bf16 hidden in, its
         # codes out and back, scales
-        w_bytes = w.V * w.D if args.lm == "e4m3" else w.V * w.D // 2 + w.V * ((w.D + 31) // 32)
-        lm_bytes = w_bytes + w.V * 4 + N * w.D * 2 + 2 * N * w.D + N * 4 + vtiles * N * 8 + T * 4
+        nb = (w.D + 31) // 32
+        w_bytes = {"e4m3": w.V * w.D + w.V * 4, "w4": w.V * w.D // 2 + w.V * nb + w.V * 4,
+                   "mxfp8": w.V * w.D + w.V * nb}[args.lm]
+        # hidden: bf16 in, its codes out and back, its scales (per token, or
+        # per 32-element block for mxfp8)
+        h_scales = N * nb if args.lm == "mxfp8" else N * 4
+        lm_bytes = w_bytes + N * w.D * 2 + 2 * N * w.D + h_scales + vtiles * N * 8 + T * 4
     lm_flops = 2.0 * N * w.D * w.V
     score_avg_s = call_ms["score"] / 1e3
     # e4m3 tensor peak (both low-precision heads multiply e4m3 operands): the
@@ -921,10 +930,12 @@ def main():
                     help="time the headline batch only (no per-workload lines, no sweep)")
     ap.add_argument("--rule", default="delta", choices=["delta", "gla"],
                     help="recurrence of the linear-attention fork (hybrid workloads)")
-    ap.add_argument("--lm", default="bf16", choices=["bf16", "e4m3", "w4"],
+    ap.add_argument("--lm", default="bf16", choices=["bf16", "e4m3", "w4", "mxfp8"],
                     help="LM head precision: bf16 (the workload's), e4m3 codes with one "
                          "scale per weight row and per token (the paper's 8-bit weights), or "
-                         "w4: 4-bit weights in 32-element blocks (the paper's 4-bit weights)")
+                         "w4: 4-bit weights in 32-element blocks (the paper's 4-bit weights), "
+                         "or mxfp8: e4m3 weights and hidden states in 32-element blocks with "
+                         "power-of-two block scales")
     ap.add_argument("--stack", default=None,
                     help="time a hybrid decoder stack (e.g. hybrid4) over the workload's rows, "
                          "then the LM head and the decision (one GPU)")

@@ -413,6 +413,54 @@ jet_status jet_score_candidates_w4(const jet_layout* lay, const jet_dims* dims,
                                    size_t ws_bytes, void* stream);
 
 /*
+ * MXFP8 LM head (the microscaling form of the paper's 8-bit weights, Appendix
+ * A: 8-bit codes in 32-element blocks that each carry a scale). Every row of
+ * the weights and of the hidden states is cut into 32-element blocks (the last
+ * may be shorter); block b gets the shared exponent
+ *   X = floor(log2(max |x| over the block)) - 8, clamped to [-127, 127]
+ *   (-127 for a block of zeros or of subnormal maxima),
+ * stored as the UE8M0 byte X + 127, and its elements the OCP FP8 E4M3 codes of
+ * x * 2^-X (nearest, ties to even, saturating at +-448). The value of a code
+ * is 2^X decode(code); there is no further per-row scale.
+ *
+ * Layout of an MXFP8 weight buffer for [V, D] (jet_mxfp8_bytes(V, D) bytes):
+ *   - codes [V, D] row-major (V D bytes, rounded up to 256);
+ *   - then one 512-byte chunk of scale factors per (vocabulary tile vt of 128
+ *     rows, K slice kb of 128 elements), chunk vt ceil(D / 128) + kb, byte
+ *     16 i + 4 j + c holding block c of the slice of row 128 vt + 32 j + i
+ *     (127 for rows past V).
+ */
+size_t jet_mxfp8_bytes(int64_t V, int64_t D);
+
+/*
+ * jet_quantize_mxfp8 - quantise the bf16 matrix w [V, D] (device, row-major)
+ * into `out` (jet_mxfp8_bytes(V, D) bytes, 16-byte aligned). Errors:
+ * JET_ERR_ARG, JET_ERR_SHAPE (D not a positive multiple of 16), JET_ERR_ALIGN.
+ * Done once per model.
+ */
+jet_status jet_quantize_mxfp8(const void* w, int64_t V, int64_t D, uint8_t* out, void* stream);
+
+/* Workspace bytes of jet_score_candidates_mxfp8 (the bf16 path's, the hidden
+ * states' codes and their scale factors); 0 on invalid arguments. */
+size_t jet_workspace_bytes_mxfp8(const jet_sizes* n, const jet_dims* dims);
+
+/*
+ * jet_score_candidates_mxfp8 - jet_score_candidates with an MXFP8 LM head:
+ *   hidden      [N, D] bf16     quantised to MXFP8 into the workspace
+ *   w_mx        the weights from jet_quantize_mxfp8 with the same V, D
+ * The logit is z[n, v] = sum_b 2^(X_h[n, b] + X_w[v, b]) sum_{k in b}
+ * decode(h_q[n, k]) decode(w_q[v, k]), accumulated in float32 on the tensor
+ * cores by the block-scaled MMA (both sets of scale factors applied by the
+ * hardware); log-softmax, gather and sums as in jet_score_candidates. dims:
+ * dtype JET_DTYPE_BF16, D a positive multiple of 16; workspace
+ * jet_workspace_bytes_mxfp8().
+ */
+jet_status jet_score_candidates_mxfp8(const jet_layout* lay, const jet_dims* dims,
+                                      const void* hidden, const uint8_t* w_mx,
+                                      float* tok_logprob, float* cand_score, void* ws,
+                                      size_t ws_bytes, void* stream);
+
+/*
  * Hybrid decoder stacks (Sec. 4.1: hybrid models keep a recurrent state per
  * linear-attention layer, restored for every candidate, and reuse the prefix
  * cache at attention layers). jet_stack_forward runs L pre-norm decoder

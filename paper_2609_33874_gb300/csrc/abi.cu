@@ -143,6 +143,34 @@ E4m3Plan e4m3_plan(const jet_sizes& n, int D) {
   return p;
 }
 
+// scratch of the MXFP8 score path: the bf16 path's plan, then the hidden
+// states' codes [N, D] and their scale factors (two 512-byte chunks per token
+// tile and K slice)
+struct MxPlan {
+  jet::ScorePlan score;
+  size_t hq_off, hsf_off, bytes;
+  int Nt, n_tt;
+};
+
+MxPlan mx_plan(const jet_sizes& n, int D) {
+  auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
+  MxPlan p{};
+  p.score = jet::score_plan(n);
+  jet::mx_token_tiling(n.N > 0 ? n.N : 1, &p.Nt, &p.n_tt);
+  const size_t nkb = size_t(D + 127) / 128;
+  p.hq_off = up(p.score.bytes);
+  p.hsf_off = p.hq_off + up(size_t(n.N) * size_t(D));
+  p.bytes = p.hsf_off + size_t(p.n_tt) * nkb * 2 * jet::kW4ScaleBytes;
+  return p;
+}
+
+// bytes of the MXFP8 weight buffer: codes [V, D], then one 512-byte chunk of
+// scale factors per (128-row tile, 128-element K slice)
+size_t mx_weight_bytes(int64_t V, int64_t D) {
+  const size_t codes = (size_t(V) * size_t(D) + 255) & ~size_t(255);
+  return codes + size_t((V + 127) / 128) * size_t((D + 127) / 128) * jet::kW4ScaleBytes;
+}
+
 jet_status cuda_status(cudaError_t e) { return e == cudaSuccess ? JET_OK : JET_ERR_CUDA; }
 
 #define JET_TRY(expr)            \
@@ -402,6 +430,62 @@ extern "C" jet_status jet_score_candidates_w4(const jet_layout* lay, const jet_d
   JET_TRY(cuda_status(jet::launch_quantize_e4m3(hidden, n.N, dims->D, h_q, h_scale, st)));
   JET_TRY(cuda_status(jet::launch_lmhead_w4(*lay, *dims, plan.score, h_q, h_scale, w4, w_scale,
                                             ws, status, st)));
+  return cuda_status(
+      jet::launch_score_finish(*lay, plan.score, ws, tok_logprob, cand_score, status, st));
+}
+
+extern "C" size_t jet_mxfp8_bytes(int64_t V, int64_t D) {
+  if (V < 1 || D < 16 || D % 16 != 0 || V > (int64_t(1) << 30) || D > (int64_t(1) << 20)) return 0;
+  return mx_weight_bytes(V, D);
+}
+
+extern "C" jet_status jet_quantize_mxfp8(const void* w, int64_t V, int64_t D, uint8_t* out,
+                                         void* stream) {
+  if (V < 1) return JET_ERR_ARG;
+  if (D < 16 || D % 16 != 0) return JET_ERR_SHAPE;
+  if (V > (int64_t(1) << 30) || D > (int64_t(1) << 20)) return JET_ERR_CAPACITY;
+  JET_TRY(check_ptr(w, V));
+  JET_TRY(check_ptr(out, V));
+  const int vtiles = int((V + 127) / 128);
+  uint8_t* sf = out + ((size_t(V) * size_t(D) + 255) & ~size_t(255));
+  return cuda_status(jet::launch_quantize_mx(w, int(V), int(D), vtiles * 128, 128, 1, out, sf,
+                                             static_cast<cudaStream_t>(stream)));
+}
+
+extern "C" size_t jet_workspace_bytes_mxfp8(const jet_sizes* n, const jet_dims* d) {
+  if (!n || !d || n->R < 0 || n->N < 0 || n->V < 1 || d->D < 16) return 0;
+  size_t a = 0;
+  if (d->Hq > 0 && d->Hkv > 0 && d->Hq % d->Hkv == 0 && d->d > 0) a = jet::attn_plan(*n, *d).bytes;
+  const size_t b = mx_plan(*n, d->D).bytes;
+  return a > b ? a : b;
+}
+
+extern "C" jet_status jet_score_candidates_mxfp8(const jet_layout* lay, const jet_dims* dims,
+                                                 const void* hidden, const uint8_t* w_mx,
+                                                 float* tok_logprob, float* cand_score, void* ws,
+                                                 size_t ws_bytes, void* stream) {
+  JET_TRY(check_layout(lay));
+  JET_TRY(check_e4m3_dims(dims));
+  const jet_sizes& n = lay->n;
+  if (n.R == 0) return JET_OK;
+  const MxPlan plan = mx_plan(n, dims->D);
+  if (plan.score.vtiles > 65535) return JET_ERR_CAPACITY;
+  JET_TRY(check_ptr(hidden, n.N));
+  JET_TRY(check_ptr(w_mx, n.V));
+  JET_TRY(check_ptr(tok_logprob, n.T));
+  JET_TRY(check_ptr(cand_score, n.C));
+  if (!ws || ws_bytes < plan.bytes) return JET_ERR_WORKSPACE;
+  if (!aligned16(ws)) return JET_ERR_ALIGN;
+  int* status = jet::device_status_ptr();
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint8_t* h_q = static_cast<uint8_t*>(ws) + plan.hq_off;
+  uint8_t* h_sf = static_cast<uint8_t*>(ws) + plan.hsf_off;
+  // the hidden states into codes and per-token-tile scale-factor chunks
+  JET_TRY(cuda_status(jet::launch_quantize_mx(hidden, n.N, dims->D, plan.n_tt * 256, plan.Nt, 2,
+                                              h_q, h_sf, st)));
+  const uint8_t* w_sf = w_mx + ((size_t(n.V) * size_t(dims->D) + 255) & ~size_t(255));
+  JET_TRY(cuda_status(jet::launch_lmhead_mx(*lay, *dims, plan.score, h_q, h_sf, w_mx, w_sf, ws,
+                                            status, st)));
   return cuda_status(
       jet::launch_score_finish(*lay, plan.score, ws, tok_logprob, cand_score, status, st));
 }

@@ -165,6 +165,20 @@ cudaError_t launch_lmhead_w4(const jet_layout& lay, const jet_dims& d, const Sco
 // 4-bit quantisation of a bf16 matrix [V, D] into the tiled layout, scales [V]
 cudaError_t launch_quantize_w4(const void* x, int V, int D, uint8_t* w4, float* scale,
                                cudaStream_t st);
+// MXFP8 quantisation (e4m3 codes, a UE8M0 factor per 32-element block) of
+// the bf16 matrix x [rows, D]: `slots` row slots in groups of 128 * halves,
+// slot rs of group g being row g * tile_rows + rs (rs < tile_rows); codes
+// row-major [rows, D], factors in 512-byte chunks per (group, K slice, half)
+cudaError_t launch_quantize_mx(const void* x, int rows, int D, int slots, int tile_rows,
+                               int halves, uint8_t* codes, uint8_t* sf, cudaStream_t st);
+// the MXFP8 LM head's token tiles: at most 224 rows (a multiple of 16) each
+void mx_token_tiling(int N, int* Nt, int* n_tt);
+// the LM head on MXFP8 weights (codes [V, D], factors per 128-row tile and K
+// slice) and MXFP8 hidden states (codes [N, D], factors per token tile and K
+// slice, two chunks each)
+cudaError_t launch_lmhead_mx(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
+                             const uint8_t* h_q, const uint8_t* h_sf, const uint8_t* w_q,
+                             const uint8_t* w_sf, void* ws, int* status, cudaStream_t st);
 // per-row e4m3 quantisation of a bf16 matrix [rows, D] (D multiple of 16)
 cudaError_t launch_quantize_e4m3(const void* x, int rows, int D, uint8_t* q, float* scale,
                                  cudaStream_t st);

@@ -63,12 +63,11 @@ constexpr int kBM = kVocabTile;     // 128 vocabulary rows per tile (MMA M, TMEM
 constexpr int kBK = 64;             // bf16 hidden elements per stage: 128 bytes
 constexpr int kBKBytes = 128;       // bytes of one K slice of a row, either element type
 constexpr int kThreads = 192;
-enum { kFmtBf16 = 0, kFmtE4m3 = 1, kFmtW4 = 2 };
+enum { kFmtBf16 = 0, kFmtE4m3 = 1, kFmtW4 = 2, kFmtMx8 = 3 };
 constexpr int kMaxNt = 256;
-// w4: token tiles of at most 224 columns leave room in TMEM (512 columns) for
-// the two accumulators, the hidden side's 8 scale columns and 4 scale
-// columns per stage for the weights
-constexpr int kMaxNtW4 = 224;
+// block-scaled formats: token tiles of at most 224 columns leave room in TMEM
+// (512 columns) for the two accumulators and the scale-factor slots
+constexpr int kMaxNtBs = 224;
 constexpr int kSfbCols = 8;
 constexpr int kSfaSlot = 8;   // TMEM columns per stage's weight scale factors (4 used)
 constexpr uint64_t kDrainNs = 200000000ull;  // budget of the drain after an abort
@@ -86,14 +85,16 @@ struct TcArgs {
   float* z_tgt;
   const float* w_scale;  // e4m3: [V] per vocabulary row
   const float* h_scale;  // e4m3: [N] per token
-  const uint8_t* w4_sf;  // w4: the scale-factor region, one 512-byte chunk per tile
+  const uint8_t* w_sf;   // w4, mxfp8: the weights' scale factors, a 512-byte chunk per tile
+  const uint8_t* h_sf;   // mxfp8: the hidden states' scale factors, two chunks per tile
   int* status;
   int N, T, V, D;
   int Nt, n_tt, units, nkb, stages, vtiles;
   uint32_t tmem_cols;
   uint32_t buf_cols;     // columns of one accumulator
-  uint32_t sfb_col;      // w4: the hidden side's scale factors (all 1)
-  uint32_t sfa_col;      // w4: the weight scale factors, kSfaSlot columns per stage
+  uint32_t sfb_col;      // the hidden side's scale factors: w4 one slot (all 1),
+                         // mxfp8 kSfaSlot columns per stage
+  uint32_t sfa_col;      // the weight scale factors, kSfaSlot columns per stage
   uint64_t wait_ns;  // budget of one bounded wait (jet_set_wait_budget_ns)
   int hold_first;    // test hook (jet_set_test_stall): withhold the first stage's loads
 };
@@ -155,11 +156,12 @@ __device__ __forceinline__ void mma_mx(uint32_t d_tmem, uint64_t a_desc, uint64_
       : "memory");
 }
 
-// Instruction descriptor of kind::mxf8f6f4 with block scaling: A E2M1
-// (format 5), B e4m3 (format 0), both K-major, UE8M0 scale factors, shape
-// M x N; block `k` of the 4 in a scale-factor word for both operands.
-__host__ __device__ constexpr uint32_t idesc_mx_e2m1_e4m3(int M, int N, int k) {
-  return (uint32_t(k) << 4) | (5u << 7) | (0u << 10) | (uint32_t(N >> 3) << 17) | (1u << 23) |
+// Instruction descriptor of kind::mxf8f6f4 with block scaling: A of format
+// `afmt` (E2M1 = 5, e4m3 = 0), B e4m3 (format 0), both K-major, UE8M0 scale
+// factors, shape M x N; block `k` of the 4 in a scale-factor word for both
+// operands.
+__host__ __device__ constexpr uint32_t idesc_mx(uint32_t afmt, int M, int N, int k) {
+  return (uint32_t(k) << 4) | (afmt << 7) | (0u << 10) | (uint32_t(N >> 3) << 17) | (1u << 23) |
          (uint32_t(M >> 4) << 24) | (uint32_t(k) << 29);
 }
 
@@ -199,15 +201,18 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
                  const TcArgs a) {
   constexpr bool F8 = FMT != kFmtBf16;   // 8-bit hidden codes in the MMA
   constexpr bool W4 = FMT == kFmtW4;     // 4-bit weights, block-scaled MMA
+  constexpr bool MX = FMT == kFmtMx8;    // e4m3 blocks on both sides, block-scaled MMA
+  constexpr bool ROWSC = FMT == kFmtE4m3 || W4;  // float32 scales per weight row and token
   constexpr int kBKe = F8 ? kBKBytes : kBK;  // elements of one K slice
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   const uint32_t a_bytes = kBM * 128, b_bytes = uint32_t(a.Nt) * 128;
   // a stage holds the weight and hidden tiles of one K slice (w4: the weight
-  // tile as the TMA unpacks it, 1 byte per code) and, for w4, the slice's
-  // 512-byte scale-factor chunk (in a 1 KB slot, keeping stages 1 KB aligned)
-  const uint32_t stage_bytes = a_bytes + b_bytes + (W4 ? 1024u : 0u);
+  // tile as the TMA unpacks it, 1 byte per code) and the slice's scale-factor
+  // chunks: w4 the weights' 512 bytes (in a 1 KB slot), mxfp8 also the hidden
+  // states' two chunks (a 2 KB slot), keeping stages 1 KB aligned
+  const uint32_t stage_bytes = a_bytes + b_bytes + (W4 ? 1024u : MX ? 2048u : 0u);
   float2* red = reinterpret_cast<float2*>(smem + size_t(a.stages) * stage_bytes);
   int4* hits = reinterpret_cast<int4*>(red + 4 * kMaxNt);                          // [128]
   float* hs = reinterpret_cast<float*>(hits + 128);                                // [256]
@@ -268,8 +273,10 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
     if (lane == 0) {
       const uint64_t pol_w = policy_evict_first(), pol_h = policy_evict_last();
       // the weight bytes one stage brings: bf16 or e4m3 tile, or packed
-      // 4-bit codes (half the unpacked tile) and their scale-factor chunk
-      const uint32_t w_tx = W4 ? a_bytes / 2 + kW4ScaleBytes : a_bytes;
+      // 4-bit codes (half the unpacked tile) and their scale-factor chunk;
+      // mxfp8 adds both operands' chunks
+      const uint32_t w_tx = W4 ? a_bytes / 2 + kW4ScaleBytes
+                               : MX ? a_bytes + 3 * kW4ScaleBytes : a_bytes;
       int s = 0;
       uint32_t ph = 0, issued = 0, issued_par = 0;
       bool ok = true, hold = a.hold_first != 0;
@@ -287,10 +294,14 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
             mbar_arrive_expect_tx(full + s, w_tx + b_bytes);
             tma_load_2d(sa, &tmW, full + s, kb * kBKe, v0, pol_w);
             tma_load_2d(sa + a_bytes, &tmH, full + s, kb * kBKe, t0, pol_h);
-            if (W4)
+            if (W4 || MX)
               bulk_load(sa + a_bytes + b_bytes,
-                        a.w4_sf + (size_t(vt) * a.nkb + kb) * kW4ScaleBytes, kW4ScaleBytes,
+                        a.w_sf + (size_t(vt) * a.nkb + kb) * kW4ScaleBytes, kW4ScaleBytes,
                         full + s, pol_w);
+            if (MX)
+              bulk_load(sa + a_bytes + b_bytes + kW4ScaleBytes,
+                        a.h_sf + (size_t(u % a.n_tt) * a.nkb + kb) * 2 * kW4ScaleBytes,
+                        2 * kW4ScaleBytes, full + s, pol_h);
             issued |= 1u << s;
             issued_par = (issued_par & ~(1u << s)) | (ph << s);
           }
@@ -332,16 +343,21 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
           tc_fence_after();
           const uint32_t sa = smem_u32(smem + size_t(s) * stage_bytes);
           const uint32_t sb = sa + a_bytes;
-          if (W4) {
-            // the slice's weight scale factors into this stage's 4 columns;
-            // the MMAs after it in this thread's order read them
+          if (W4 || MX) {
+            // the slice's weight scale factors into this stage's 4 columns
+            // (mxfp8: the hidden states' too, 4 columns per 128 token rows);
+            // the MMAs after them in this thread's order read them
             const uint32_t sfa = tmem_base + a.sfa_col + kSfaSlot * s;
+            const uint32_t sfb = MX ? tmem_base + a.sfb_col + kSfaSlot * s : tmem_base + a.sfb_col;
             tmem_cp_32x128(sfa, sb + b_bytes);
+            if (MX) {
+              tmem_cp_32x128(sfb, sb + b_bytes + kW4ScaleBytes);
+              if (a.Nt > 128) tmem_cp_32x128(sfb + 4, sb + b_bytes + 2 * kW4ScaleBytes);
+            }
 #pragma unroll
             for (int k = 0; k < 4; ++k)
               mma_mx(d_tmem, desc_k_sw128(sa + 32 * k), desc_k_sw128(sb + 32 * k),
-                     idesc_mx_e2m1_e4m3(kBM, a.Nt, k), sfa, tmem_base + a.sfb_col,
-                     (kb | k) != 0);
+                     idesc_mx(W4 ? 5u : 0u, kBM, a.Nt, k), sfa, sfb, (kb | k) != 0);
           } else {
             // 32 bytes of K per instruction: 16 bf16 or 32 e4m3 elements
 #pragma unroll
@@ -390,9 +406,10 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
       const uint32_t tl = tcol + (uint32_t(32 * q) << 16);
       const int ncols = min(a.Nt, a.N - t0);
       const bool row_valid = v0 + vrow < a.V;
-      // e4m3: this row's weight scale, and the unit's token scales in shared memory
+      // e4m3, w4: this row's weight scale, and the unit's token scales in
+      // shared memory (mxfp8 needs none: its block scales are in the MMA)
       float wsc = 1.f;
-      if (F8) {
+      if (ROWSC) {
         wsc = row_valid ? a.w_scale[v0 + vrow] : 0.f;
         for (int c = et; c < ncols; c += 128) hs[c] = a.h_scale[t0 + c];
         named_bar_sync(1, 128);
@@ -424,7 +441,7 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
           if (hv.y == q) {
             const float z = tmem_ld_1col(tl + uint32_t(hv.w));
             tmem_wait_ld();
-            if (lane == hv.z) a.z_tgt[hv.x] = F8 ? z * wsc * hs[hv.w] : z;
+            if (lane == hv.z) a.z_tgt[hv.x] = ROWSC ? z * wsc * hs[hv.w] : z;
           }
         }
         named_bar_sync(1, 128);
@@ -435,7 +452,7 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant_
         float v[32];
         tmem_ld_32cols(tl + uint32_t(c0), v);
         tmem_wait_ld();
-        if (F8) {
+        if (ROWSC) {
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] *= wsc * hs[c0 + i];
         }
@@ -545,13 +562,18 @@ namespace {
 template <int FMT>
 cudaError_t launch_head(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
                         const void* hidden, const float* h_scale, const void* w_lm,
-                        const float* w_scale, void* ws, int* status, cudaStream_t st) {
-  constexpr bool F8 = FMT != kFmtBf16, W4 = FMT == kFmtW4;
+                        const float* w_scale, void* ws, int* status, cudaStream_t st,
+                        const uint8_t* w_sf = nullptr, const uint8_t* h_sf = nullptr) {
+  constexpr bool F8 = FMT != kFmtBf16, W4 = FMT == kFmtW4, MX = FMT == kFmtMx8;
   const jet_sizes& n = lay.n;
-  const int max_nt = W4 ? kMaxNtW4 : kMaxNt;
-  int n_tt = (n.N + max_nt - 1) / max_nt;
-  const int Nt = ((n.N + n_tt - 1) / n_tt + 15) / 16 * 16;
-  n_tt = (n.N + Nt - 1) / Nt;
+  int n_tt = 0, Nt = 0;
+  if (W4 || MX) {
+    mx_token_tiling(n.N, &Nt, &n_tt);
+  } else {
+    n_tt = (n.N + kMaxNt - 1) / kMaxNt;
+    Nt = ((n.N + n_tt - 1) / n_tt + 15) / 16 * 16;
+    n_tt = (n.N + Nt - 1) / Nt;
+  }
   const int esize = F8 ? 1 : 2;
   TcArgs a{};
   a.wait_ns = wait_budget_ns();
@@ -576,18 +598,23 @@ cudaError_t launch_head(const jet_layout& lay, const jet_dims& d, const ScorePla
   a.vtiles = plan.vtiles;
   a.nkb = (d.D * esize + kBKBytes - 1) / kBKBytes;
   const int a_bytes = kBM * kBKBytes, b_bytes = Nt * kBKBytes;
-  const int stage_bytes = a_bytes + b_bytes + (W4 ? 1024 : 0);
+  const int stage_bytes = a_bytes + b_bytes + (W4 ? 1024 : MX ? 2048 : 0);
   a.stages = std::min(8, (kSmemLimit - 1024 - kFixedSmem) / stage_bytes);
   if (a.stages < 2) return cudaErrorInvalidValue;
-  if (W4) {
+  if (W4 || MX) {
     // accumulators at columns 0 and buf_cols, then the hidden side's scale
-    // factors, then the weight scale factors (a slot of 8 columns per stage)
+    // factors (w4: one slot of 1s; mxfp8: a slot of 8 columns per stage), then
+    // the weight scale factors (a slot of 8 columns per stage)
     a.buf_cols = uint32_t(Nt + 31) / 32 * 32;
-    a.sfb_col = 2 * a.buf_cols;
-    a.sfa_col = a.sfb_col + kSfbCols;
     a.tmem_cols = 512;
-    while (a.stages > 2 && a.sfa_col + kSfaSlot * a.stages > a.tmem_cols) --a.stages;
-    if (a.sfa_col + kSfaSlot * a.stages > a.tmem_cols) return cudaErrorInvalidValue;
+    auto fits = [&](int stages) {
+      const uint32_t sfb_cols = MX ? uint32_t(kSfaSlot * stages) : uint32_t(kSfbCols);
+      return 2 * a.buf_cols + sfb_cols + kSfaSlot * stages <= a.tmem_cols;
+    };
+    while (a.stages > 2 && !fits(a.stages)) --a.stages;
+    if (!fits(a.stages)) return cudaErrorInvalidValue;
+    a.sfb_col = 2 * a.buf_cols;
+    a.sfa_col = a.sfb_col + (MX ? kSfaSlot * a.stages : kSfbCols);
   } else {
     a.tmem_cols = Nt <= 128 ? 256 : 512;
     a.buf_cols = a.tmem_cols / 2;
@@ -601,9 +628,13 @@ cudaError_t launch_head(const jet_layout& lay, const jet_dims& d, const ScorePla
     // ceil(D / 128) * 128 codes; the scale-factor region follows it
     const int rows = plan.vtiles * kBM, kd = a.nkb * 128;
     if (!encode_w4_codes(&tmW, w_lm, rows, kd)) return cudaErrorInvalidValue;
-    a.w4_sf = static_cast<const uint8_t*>(w_lm) + size_t(rows) * (kd / 2);
+    a.w_sf = static_cast<const uint8_t*>(w_lm) + size_t(rows) * (kd / 2);
   } else if (!encode_kmajor(&tmW, w_lm, n.V, d.D, kBM, esize)) {
     return cudaErrorInvalidValue;
+  }
+  if (MX) {
+    a.w_sf = w_sf;
+    a.h_sf = h_sf;
   }
   cudaError_t e = cudaFuncSetAttribute(lmhead_tc_kernel<FMT>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
@@ -627,6 +658,20 @@ cudaError_t launch_lmhead_e4m3(const jet_layout& lay, const jet_dims& d, const S
                                const uint8_t* h_q, const float* h_scale, const uint8_t* w_q,
                                const float* w_scale, void* ws, int* status, cudaStream_t st) {
   return launch_head<kFmtE4m3>(lay, d, plan, h_q, h_scale, w_q, w_scale, ws, status, st);
+}
+
+cudaError_t launch_lmhead_mx(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,
+                             const uint8_t* h_q, const uint8_t* h_sf, const uint8_t* w_q,
+                             const uint8_t* w_sf, void* ws, int* status, cudaStream_t st) {
+  return launch_head<kFmtMx8>(lay, d, plan, h_q, nullptr, w_q, nullptr, ws, status, st, w_sf,
+                              h_sf);
+}
+
+void mx_token_tiling(int N, int* Nt, int* n_tt) {
+  int tt = (N + kMaxNtBs - 1) / kMaxNtBs;
+  const int nt = ((N + tt - 1) / tt + 15) / 16 * 16;
+  *Nt = nt;
+  *n_tt = (N + nt - 1) / nt;
 }
 
 cudaError_t launch_lmhead_w4(const jet_layout& lay, const jet_dims& d, const ScorePlan& plan,

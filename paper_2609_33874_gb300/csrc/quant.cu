@@ -134,6 +134,61 @@ quantize_w4_kernel(const __nv_bfloat16* __restrict__ x, int V, int D, int rows_p
   }
 }
 
+// MXFP8 (e4m3 codes, one UE8M0 scale factor per 32-element block): one warp
+// per row slot. Row slots come in groups of 128 * halves; slot rs of group g
+// is matrix row g * tile_rows + rs when rs < tile_rows (and that row exists),
+// padding otherwise. Per 128-element slice kb the group's scale factors form
+// `halves` 512-byte chunks, chunk (g * nkb + kb) * halves + rs / 128, in the
+// order one tcgen05.cp (32 x 128 bits) places a chunk in TMEM: slot
+// 32 j + i of the 128 at byte 16 i + 4 j + block. Codes are written row-major
+// [rows, D] for the rows that exist; padding slots get factor 127 and no codes.
+// X = floor(log2(block max)) - 8 from the float's exponent field (clamped to
+// -127 below), element code = e4m3(x * 2^-X), nearest even, saturating.
+__global__ void __launch_bounds__(32 * kRowsPerBlock)
+quantize_mx_kernel(const __nv_bfloat16* __restrict__ x, int rows, int D, int slots,
+                   int tile_rows, int halves, int nkb, uint8_t* __restrict__ codes,
+                   uint8_t* __restrict__ sf) {
+  pdl_begin();
+  const int lane = threadIdx.x & 31;
+  const int slot = blockIdx.x * kRowsPerBlock + (threadIdx.x >> 5);
+  if (slot >= slots) return;
+  const int G = 128 * halves;
+  const int g = slot / G, rs = slot % G;
+  const int row = g * tile_rows + rs;
+  const bool real = rs < tile_rows && row < rows;
+  const __nv_bfloat16* xr = x + size_t(real ? row : 0) * D;
+  const int r = rs & 127, c = lane >> 3;
+  for (int kb = 0; kb < nkb; ++kb) {
+    const int k = kb * 128 + lane * 4;
+    float f[4] = {0.f, 0.f, 0.f, 0.f};
+    if (real && k < D) {
+      const uint2 q = *reinterpret_cast<const uint2*>(xr + k);
+      const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&q.x));
+      const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&q.y));
+      f[0] = a.x; f[1] = a.y; f[2] = b.x; f[3] = b.y;
+    }
+    float bmax = fmaxf(fmaxf(fabsf(f[0]), fabsf(f[1])), fmaxf(fabsf(f[2]), fabsf(f[3])));
+#pragma unroll
+    for (int o = 1; o < 8; o <<= 1) bmax = fmaxf(bmax, __shfl_xor_sync(0xffffffffu, bmax, o));
+    // floor(log2(bmax)) is the exponent field minus 127 for a normal float;
+    // zero and subnormal maxima clamp to X = -127
+    const int ef = (__float_as_int(bmax) >> 23) & 0xFF;
+    const int X = ef == 0 ? -127 : max(ef - 127 - 8, -127);
+    const float scale = __int_as_float((127 - X) << 23);  // 2^-X, exact (X <= 119)
+    if (real && k < D) {
+      uint32_t w = 0;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        w |= uint32_t(__nv_cvt_float_to_fp8(__fmul_rn(f[i], scale), __NV_SATFINITE, __NV_E4M3))
+             << (8 * i);
+      *reinterpret_cast<uint32_t*>(codes + size_t(row) * D + k) = w;
+    }
+    if ((lane & 7) == 0)
+      sf[(size_t(g * nkb + kb) * halves + (rs >> 7)) * 512 + 16 * (r & 31) + 4 * (r >> 5) + c] =
+          uint8_t(real ? X + 127 : 127);
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_quantize_w4(const void* x, int V, int D, uint8_t* w4, float* scale,
@@ -152,6 +207,19 @@ cudaError_t launch_quantize_e4m3(const void* x, int rows, int D, uint8_t* q, flo
   return launch_pdl(quantize_e4m3_kernel, dim3(unsigned((rows + kRowsPerBlock - 1) / kRowsPerBlock)),
                     dim3(32 * kRowsPerBlock), 0, st, static_cast<const __nv_bfloat16*>(x), rows, D,
                     q, scale);
+}
+
+}  // namespace jet
+
+namespace jet {
+
+cudaError_t launch_quantize_mx(const void* x, int rows, int D, int slots, int tile_rows,
+                               int halves, uint8_t* codes, uint8_t* sf, cudaStream_t st) {
+  if (slots <= 0) return cudaSuccess;
+  const int nkb = (D + 127) / 128;
+  return launch_pdl(quantize_mx_kernel, dim3(unsigned((slots + kRowsPerBlock - 1) / kRowsPerBlock)),
+                    dim3(32 * kRowsPerBlock), 0, st, static_cast<const __nv_bfloat16*>(x), rows, D,
+                    slots, tile_rows, halves, nkb, codes, sf);
 }
 
 }  // namespace jet

@@ -101,6 +101,11 @@ def _load() -> ctypes.CDLL:
         "jet_quantize_w4": (I, [P, ctypes.c_int64, ctypes.c_int64, P, P, P]),
         "jet_score_candidates_w4": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
                                         P, P, P, P, P, P, SZ, P]),
+        "jet_mxfp8_bytes": (SZ, [ctypes.c_int64, ctypes.c_int64]),
+        "jet_quantize_mxfp8": (I, [P, ctypes.c_int64, ctypes.c_int64, P, P]),
+        "jet_workspace_bytes_mxfp8": (SZ, [ctypes.POINTER(jet_sizes), ctypes.POINTER(jet_dims)]),
+        "jet_score_candidates_mxfp8": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
+                                           P, P, P, P, P, SZ, P]),
         "jet_stack_workspace_bytes": (SZ, [ctypes.POINTER(jet_sizes), ctypes.POINTER(jet_dims),
                                            I]),
         "jet_stack_forward": (I, [ctypes.POINTER(jet_layout), ctypes.POINTER(jet_dims),
@@ -126,6 +131,8 @@ DECLARED = ("jet_abi_version", "jet_status_string", "jet_layout_plan", "jet_layo
             "jet_fork_state", "jet_fork_state_rule", "jet_score_candidates", "jet_score_candidates_noalloc",
             "jet_quantize_rows_e4m3", "jet_workspace_bytes_e4m3", "jet_score_candidates_e4m3",
             "jet_w4_bytes", "jet_quantize_w4", "jet_score_candidates_w4",
+            "jet_mxfp8_bytes", "jet_quantize_mxfp8", "jet_workspace_bytes_mxfp8",
+            "jet_score_candidates_mxfp8",
             "jet_stack_workspace_bytes", "jet_stack_forward", "jet_decide", "jet_evaluate", "jet_device_status",
             "jet_set_wait_budget_ns", "jet_launch_count", "jet_set_test_stall")
 
@@ -359,13 +366,13 @@ def jet_score_candidates_e4m3(layout, dims: jet_dims, hidden, w_q, w_scale, tok_
 
 
 def jet_w4_bytes(V: int, D: int) -> int:
-    """Bytes of the tiled 4-bit codes of a [V, D] matrix (0 if invalid)."""
+    """Bytes of the 4-bit codes and scale factors of a [V, D] matrix (0 if invalid)."""
     return int(_lib.jet_w4_bytes(int(V), int(D)))
 
 
 def jet_quantize_w4(w, w4, scale, stream=None) -> None:
-    """Tiled 4-bit codes w4 (jet_w4_bytes(V, D) bytes) and row scales [V]
-    float32 of the bf16 matrix w [V, D] (see include/jet.h)."""
+    """4-bit codes and block scale factors w4 (jet_w4_bytes(V, D) bytes) and
+    row scales [V] float32 of the bf16 matrix w [V, D] (see include/jet.h)."""
     V, D = (int(w.shape[0]), int(w.shape[1])) if w.dim() == 2 else (0, 0)
     _check(_lib.jet_quantize_w4(_addr(w), V, D, _addr(w4), _addr(scale), _stream(stream)),
            "jet_quantize_w4")
@@ -379,6 +386,33 @@ def jet_score_candidates_w4(layout, dims: jet_dims, hidden, w4, w_scale, tok_log
                                         _addr(tok_logprob), _addr(cand_score), _addr(ws),
                                         int(ws_bytes), _stream(stream)),
            "jet_score_candidates_w4")
+
+
+def jet_mxfp8_bytes(V: int, D: int) -> int:
+    """Bytes of the MXFP8 codes and scale factors of a [V, D] matrix (0 if invalid)."""
+    return int(_lib.jet_mxfp8_bytes(int(V), int(D)))
+
+
+def jet_quantize_mxfp8(w, out, stream=None) -> None:
+    """MXFP8 codes and block scale factors (jet_mxfp8_bytes(V, D) bytes) of the
+    bf16 matrix w [V, D] (see include/jet.h)."""
+    V, D = (int(w.shape[0]), int(w.shape[1])) if w.dim() == 2 else (0, 0)
+    _check(_lib.jet_quantize_mxfp8(_addr(w), V, D, _addr(out), _stream(stream)),
+           "jet_quantize_mxfp8")
+
+
+def jet_workspace_bytes_mxfp8(sizes: jet_sizes, dims: jet_dims) -> int:
+    return int(_lib.jet_workspace_bytes_mxfp8(ctypes.byref(sizes), ctypes.byref(dims)))
+
+
+def jet_score_candidates_mxfp8(layout, dims: jet_dims, hidden, w_mx, tok_logprob, cand_score,
+                               ws, ws_bytes: Optional[int] = None, stream=None) -> None:
+    ws_bytes = ws.numel() * ws.element_size() if ws_bytes is None else ws_bytes
+    _check(_lib.jet_score_candidates_mxfp8(ctypes.byref(_lay(layout)), ctypes.byref(dims),
+                                           _addr(hidden), _addr(w_mx), _addr(tok_logprob),
+                                           _addr(cand_score), _addr(ws), int(ws_bytes),
+                                           _stream(stream)),
+           "jet_score_candidates_mxfp8")
 
 
 def jet_stack_workspace_bytes(sizes: jet_sizes, dims: jet_dims, Dff: int) -> int:

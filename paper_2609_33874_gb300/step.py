@@ -108,6 +108,16 @@ def quantize_lm_head_w4(w_lm: torch.Tensor, stream=None):
     return w4, w_scale
 
 
+def quantize_lm_head_mxfp8(w_lm: torch.Tensor, stream=None):
+    """MXFP8 codes and block scale factors (uint8, jet_mxfp8_bytes(V, D) bytes)
+    of the bf16 LM-head weights (jet_quantize_mxfp8), for a step built with
+    lm="mxfp8"."""
+    V, D = w_lm.shape
+    w_mx = torch.empty(jet.jet_mxfp8_bytes(V, D), dtype=torch.uint8, device=w_lm.device)
+    jet.jet_quantize_mxfp8(w_lm, w_mx, stream=stream)
+    return w_mx
+
+
 class ScoringStep:
     """Device state of one batch shape.
 
@@ -117,7 +127,8 @@ class ScoringStep:
     state. ``chain`` feeds the attention output to the LM head (requires
     Hq * d == D). ``lm`` selects the LM head: "bf16" (w_lm is the bf16 weight
     matrix), "e4m3" (w_lm is the pair returned by :func:`quantize_lm_head`) or
-    "w4" (the pair returned by :func:`quantize_lm_head_w4`).
+    "w4" (the pair returned by :func:`quantize_lm_head_w4`) or "mxfp8" (the
+    buffer returned by :func:`quantize_lm_head_mxfp8`).
     ``rule`` selects the fork's recurrence: "delta" (gated delta rule) or "gla"
     (plain gated linear attention).
     """
@@ -125,8 +136,8 @@ class ScoringStep:
     def __init__(self, layout: "jet.HostLayout", dims: "jet.jet_dims", mode: int,
                  device="cuda", hybrid: bool = False, keep_fork_state: bool = False,
                  chain: bool = False, lm: str = "bf16", rule: str = "delta"):
-        if lm not in ("bf16", "e4m3", "w4"):
-            raise ValueError("lm must be 'bf16', 'e4m3' or 'w4'")
+        if lm not in ("bf16", "e4m3", "w4", "mxfp8"):
+            raise ValueError("lm must be 'bf16', 'e4m3', 'w4' or 'mxfp8'")
         self.lm = lm
         self.rule = jet.RULES[rule]
         self.dev = torch.device(device)
@@ -148,7 +159,9 @@ class ScoringStep:
             ("value", torch.float32, (n.R,))])
         self._results = z(rb, dtype=torch.uint8)
         self._bind_results(self._results)
-        ws = (jet.jet_workspace_bytes if lm == "bf16" else jet.jet_workspace_bytes_e4m3)(n, dims)
+        ws = {"bf16": jet.jet_workspace_bytes, "e4m3": jet.jet_workspace_bytes_e4m3,
+              "w4": jet.jet_workspace_bytes_e4m3,
+              "mxfp8": jet.jet_workspace_bytes_mxfp8}[lm](n, dims)
         self.ws = z((ws + 15) // 16 * 4)  # float32 words, 16-byte multiple
         if hybrid:
             self.lo = z(self.F, dims.Hl, dims.dv, dtype=dt)
@@ -191,9 +204,12 @@ class ScoringStep:
                        stream=stream)
 
     def score(self, hidden: torch.Tensor, w_lm, stream=None, layout=None) -> None:
-        """The LM-head call of the step (bf16, e4m3 or w4, as the step was built)."""
+        """The LM-head call of the step (bf16, e4m3, w4 or mxfp8, as the step was built)."""
         lay = self.layout if layout is None else layout
-        if self.lm == "w4":
+        if self.lm == "mxfp8":
+            jet.jet_score_candidates_mxfp8(lay, self.dims, hidden, w_lm, self.tok_logprob,
+                                           self.cand_score, self.ws, stream=stream)
+        elif self.lm == "w4":
             w4, w_scale = w_lm
             jet.jet_score_candidates_w4(lay, self.dims, hidden, w4, w_scale, self.tok_logprob,
                                         self.cand_score, self.ws, stream=stream)
