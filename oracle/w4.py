@@ -24,8 +24,9 @@ tensor core can take exactly:
   one float32 multiplication rounded to nearest. A row of zeros has s = 0,
   zero codes and e_b = -5.
 * The dequantised weight is s * 2^e_b * value(code). Every 2^e_b * value(code)
-  is an E4M3 value (e_b >= -5 keeps it a normal number), which is what lets the
-  GPU widen the codes to E4M3 exactly.
+  is an E4M3 value (e_b >= -5 keeps it a normal number), so its product with an
+  E4M3 hidden code is exact whether 2^e_b is applied as a block scale factor by
+  the tensor core or folded into widened codes.
 * The logit is z[n, v] = s_h[n] s_w[v] sum_k decode_e4m3(h[n, k]) w~[v, k] with
   the hidden states quantised per token as in the E4M3 head; everything after
   the logits is the oracle of Eq. 1-5 on the dequantised matrices.
