@@ -94,6 +94,12 @@ cudaError_t launch_prefill_state(const jet_layout& lay, const jet_dims& d, int r
                                  const float* alpha, const float* beta, void* o, float* s_out,
                                  int* status, cudaStream_t st);
 // rule: JET_RECUR_DELTA or JET_RECUR_GLA
+// the chunked scan on the tensor cores (scan_tc.cu): bf16 inputs, dk = dv = 128
+bool scan_tc_supported(const jet_dims& d);
+cudaError_t launch_scan_tc(const jet_layout& lay, const jet_dims& d, int rule,
+                           const float* s_init, const void* q, const void* k, const void* v,
+                           const float* alpha, const float* beta, void* o, float* s_out,
+                           int* status, cudaStream_t st);
 // causal self-attention over every request's prefix (bf16, tensor cores);
 // the workspace holds the work list
 size_t prefill_workspace_bytes(const jet_sizes& n, const jet_dims& d);

@@ -110,6 +110,9 @@ cudaError_t launch_prefill_state(const jet_layout& lay, const jet_dims& d, int r
                                  const float* alpha, const float* beta, void* o, float* s_out,
                                  int* status, cudaStream_t st) {
   const jet_sizes& n = lay.n;
+  // bf16 with 128 x 128 states: the chunked form on the tensor cores
+  if (scan_tc_supported(d))
+    return launch_scan_tc(lay, d, rule, s_init, q, k, v, alpha, beta, o, s_out, status, st);
   dim3 grid(unsigned((d.dv + kCols - 1) / kCols), unsigned(d.Hl), unsigned(n.R));
 #define JET_SCAN(T, DELTA)                                                                   \
   return launch_pdl(scan_kernel<T, DELTA>, grid, dim3(kThreads), 0, st, lay.prefix_offset, n.R, \

@@ -168,3 +168,46 @@ def test_prefill_state_column_tails(cuda, dv):
     rel = np.abs(got_s - ref_s).max() / np.abs(ref_s).max()
     assert rel <= TOL_FORK_REL, f"state error {rel}"
     _check_scan_out(got_o, ref_o, True)
+
+
+@pytest.mark.parametrize("rule", ["delta", "gla"])
+@pytest.mark.parametrize("alpha_scale", [1.0, 0.1])
+def test_prefill_state_chunked(cuda, rule, alpha_scale):
+    # bf16 with 128 x 128 states runs the chunked scan on the tensor cores
+    # (chunks of 64 tokens): prefixes around the chunk edges, with and without
+    # a start state; alpha_scale 0.1 makes every decay strong (a ~ 0.09-0.1,
+    # products far below float32's normal range within a chunk)
+    import torch
+    w = dataclasses.replace(jet_synth.WORKLOADS["ordinal_hybrid"], Hl=3, dtype="bf16")
+    assert w.dk == 128 and w.dv == 128
+    pl = [1, 63, 64, 65, 128, 130, 200]
+    R = len(pl)
+    p = jet_synth.custom_problem(w, pl, [1] * R, [1] * R, [0] * R, seed=97)
+    hl = cuda.jet_layout_build(p.prefix_len, p.n_cand, p.cand_len, p.target_ids, w.V)
+    dims = cuda.make_dims(cuda.DTYPE_BF16, Hl=w.Hl, dk=w.dk, dv=w.dv, D=w.D)
+    t = {n: jet_synth.torch_tensor(p, n, device="cuda")
+         for n in ("lq_pre", "lk_pre", "lv_pre", "alpha_pre", "beta_pre")}
+    alpha = (p.f32("alpha_pre") * np.float32(alpha_scale)).astype(np.float32)
+    t["alpha_pre"] = torch.from_numpy(alpha).cuda()
+    for with_init in (False, True):
+        s_init = jet_synth.torch_tensor(p, "s_prefix", device="cuda") if with_init else None
+        o = torch.empty(p.total_prefix, w.Hl, w.dv, dtype=torch.bfloat16, device="cuda")
+        s_out = torch.empty(R, w.Hl, w.dk, w.dv, dtype=torch.float32, device="cuda")
+        outs = []
+        for _ in range(2):  # two calls in a row give the same answer
+            cuda.jet_prefill_state(hl.to_device("cuda"), dims, t["lq_pre"], t["lk_pre"],
+                                   t["lv_pre"], t["alpha_pre"], t["beta_pre"], o, s_out,
+                                   s_init=s_init, rule=cuda.RULES[rule])
+            torch.cuda.synchronize()
+            assert cuda.jet_device_status() == 0
+            outs.append((o.float().cpu().numpy(), s_out.cpu().numpy()))
+        np.testing.assert_array_equal(outs[0][1], outs[1][1])
+        got_o, got_s = outs[1]
+        ref_o, ref_s = O.prefill_state(p.prefix_len, p.f32("s_prefix") if with_init else None,
+                                       p.f32("lq_pre"), p.f32("lk_pre"), p.f32("lv_pre"), alpha,
+                                       p.f32("beta_pre"), rule)
+        rel = np.abs(got_s - ref_s).max() / np.abs(ref_s).max()
+        print(f"chunked scan {rule} alpha x{alpha_scale} init={with_init}: state rel {rel:.2e}, "
+              f"out max {np.abs(got_o - ref_o).max():.2e}")
+        assert rel <= TOL_FORK_REL, f"state error {rel}"
+        _check_scan_out(got_o, ref_o, True)

@@ -159,3 +159,38 @@ def test_stack_projection_wait_runs_out(cuda):
     torch.cuda.synchronize()
     assert cuda.jet_device_status() == JET_OK
     assert torch.equal(got, ref)
+
+
+@pytest.mark.parametrize("rule", ["delta", "gla"])
+def test_prefix_scan_wait_runs_out(cuda, rule):
+    # the chunked prefix-state scan on the tensor cores (bf16, 128 x 128
+    # states; several chunks per request, so copies of later chunks are in
+    # flight when the first wait gives up): the hooked call reports the
+    # timeout, the next one equals a run that never saw one
+    import torch
+    w = dataclasses.replace(jet_synth.WORKLOADS["ordinal_hybrid"], Hl=2, dtype="bf16")
+    pl = [200, 64, 130]
+    R = len(pl)
+    p = jet_synth.custom_problem(w, pl, [1] * R, [1] * R, [0] * R, seed=61)
+    hl = cuda.jet_layout_build(p.prefix_len, p.n_cand, p.cand_len, p.target_ids, w.V)
+    dims = cuda.make_dims(cuda.DTYPE_BF16, Hl=w.Hl, dk=w.dk, dv=w.dv, D=w.D)
+    t = {n: jet_synth.torch_tensor(p, n, device="cuda")
+         for n in ("lq_pre", "lk_pre", "lv_pre", "alpha_pre", "beta_pre", "s_prefix")}
+    o = torch.empty(p.total_prefix, w.Hl, w.dv, dtype=torch.bfloat16, device="cuda")
+    s_out = torch.empty(R, w.Hl, w.dk, w.dv, dtype=torch.float32, device="cuda")
+    lay = hl.to_device("cuda")
+
+    def fn():
+        cuda.jet_prefill_state(lay, dims, t["lq_pre"], t["lk_pre"], t["lv_pre"], t["alpha_pre"],
+                               t["beta_pre"], o, s_out, s_init=t["s_prefix"],
+                               rule=cuda.RULES[rule])
+
+    fn()
+    torch.cuda.synchronize()
+    assert cuda.jet_device_status() == JET_OK
+    ref_o, ref_s = o.clone(), s_out.clone()
+    assert _stalled(cuda, fn) == JET_ERR_TIMEOUT
+    fn()
+    torch.cuda.synchronize()
+    assert cuda.jet_device_status() == JET_OK
+    assert torch.equal(o, ref_o) and torch.equal(s_out, ref_s)
