@@ -84,6 +84,7 @@ struct AttArgs {
   float scale_log2;  // log2(e) / sqrt(d)
   uint64_t wait_ns;  // budget of one bounded wait (jet_set_wait_budget_ns)
   int hold_first;    // test hook (jet_set_test_stall): withhold the first query block
+  int static_only;   // 1: one slot per CTA (the grid covers every slot; no shared counter)
 };
 
 // SW128 K-major position of 16-byte chunk c of row i inside one 64-wide slice
@@ -265,10 +266,68 @@ attend_items_kernel(const AttArgs a, int qgroups, int splits) {
   }
 }
 
-// The shared item counter of the dynamic schedule starts at zero.
-__global__ void attend_reset_kernel(int* item_next) {
+// The shared item counter of the dynamic schedule starts at zero. The
+// layout arrays every work item's geometry is read from are pulled into L2 on
+// the way (the LM head's weight stream evicts them between steps), so that
+// the attention kernel's first claims do not wait on DRAM.
+__global__ void attend_reset_kernel(int* item_next, const int32_t* prefix_offset,
+                                    const int32_t* row_offset, const int32_t* req_order,
+                                    const int32_t* row_cand, const int32_t* cand_row_offset,
+                                    int R, int N, int C) {
   pdl_begin();
   if (threadIdx.x == 0) *item_next = 0;
+  auto pull = [](const int32_t* p, int n) {
+    for (int i = 32 * int(threadIdx.x); i < n; i += 32 * int(blockDim.x))
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(p + i));
+  };
+  pull(prefix_offset, R + 1);
+  pull(row_offset, R + 1);
+  if (req_order) pull(req_order, R);
+  if (row_cand) pull(row_cand, N);
+  if (cand_row_offset) pull(cand_row_offset, C + 1);
+}
+
+// The k-th work item of the unsorted order - requests by decreasing prefix
+// length (req_order); within a request kv head, query block and chunk, the
+// chunk fastest - counting only items that have keys and vectors. One warp
+// scans the requests' item counts 32 at a time; false past the last item.
+__device__ __forceinline__ bool nth_item(const AttArgs& a, int k, int lane, int4* out) {
+  int before = 0;
+  for (int base = 0; base < a.R; base += 32) {
+    const int ri = base + lane;
+    int cnt = 0, r = 0, nq = 0, sp = 0;
+    if (ri < a.R) {
+      r = a.req_order[ri];
+      if (r >= 0 && r < a.R) {
+        const int P = a.prefix_offset[r + 1] - a.prefix_offset[r];
+        const int nr = a.row_offset[r + 1] - a.row_offset[r];
+        int per = 0;
+        sp = P >= 1 ? req_splits(P, a.chunk, &per) : 0;
+        nq = nr >= 1 ? (nr + a.rb - 1) / a.rb : 0;
+        cnt = a.Hkv * nq * sp;
+      }
+    }
+    int inc = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += y;
+    }
+    const int total = __shfl_sync(0xffffffffu, inc, 31);
+    if (k < before + total) {
+      const unsigned hit = __ballot_sync(0xffffffffu, k < before + inc);
+      const int src = __ffs(hit) - 1;
+      const int kk = k - before - __shfl_sync(0xffffffffu, inc - cnt, src);
+      r = __shfl_sync(0xffffffffu, r, src);
+      nq = __shfl_sync(0xffffffffu, nq, src);
+      sp = __shfl_sync(0xffffffffu, sp, src);
+      const int split = kk % sp, rest = kk / sp;
+      *out = make_int4(r, rest / nq, rest % nq, split);
+      return true;
+    }
+    before += total;
+  }
+  return false;
 }
 
 // One work item as the scheduler warp publishes it: the item and the geometry
@@ -367,57 +426,67 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
 
   if (warp == kSchedWarp) {
     // ---------------------------------------------------------------- scheduler
-    if (lane == 0) {
-      const int count = a.sorted ? *a.item_count : 0;
-      for (int u = 0;; ++u) {
-        const int slot = u & 1;
-        if (!mbar_wait(item_empty + slot, ((u >> 1) & 1) ^ 1u, a.wait_ns, abort_flag)) {
+    const int count = a.sorted ? *a.item_count : 0;
+    for (int u = 0;; ++u) {
+      const int slot = u & 1;
+      bool okw = true;
+      if (lane == 0) okw = mbar_wait(item_empty + slot, ((u >> 1) & 1) ^ 1u, a.wait_ns, abort_flag);
+      if (!__shfl_sync(0xffffffffu, okw ? 1 : 0, 0)) {
+        if (lane == 0) {
           *abort_flag = 1;
           flag(a.status, JET_ERR_TIMEOUT);
-          break;
         }
-        // the CTA's first item is slot blockIdx.x; later ones come from the
-        // shared counter, past the grid's first items
-        int4 it = kDone;
-        ItemGeo e{};
-        for (bool first = (u == 0);; first = false) {
-          int4 cand;
-          if (a.sorted) {
+        break;
+      }
+      // the CTA's first item is number blockIdx.x; later ones come from the
+      // shared counter, past the grid's first items
+      int4 it = kDone;
+      ItemGeo e{};
+      if (a.sorted) {
+        if (lane == 0) {
+          for (bool first = (u == 0);; first = false) {
             const int idx = first ? int(blockIdx.x) : int(gridDim.x) + atomicAdd(a.item_next, 1);
             if (idx >= count) break;
-            cand = a.items[idx];
-          } else {
-            // slots run over the requests by decreasing prefix length (query
-            // blocks past the first, mostly empty, last)
-            const long long sl =
-                first ? (long long)blockIdx.x : (long long)gridDim.x + atomicAdd(a.item_next, 1);
-            if (sl >= a.n_all) break;
-            const int split = int(sl % a.splits);
-            const long long rest = sl / a.splits;
-            const int kh = int(rest % a.Hkv);
-            const long long rest2 = rest / a.Hkv;
-            const int ri = int(rest2 % a.R);
-            const int qb = int(rest2 / a.R);
-            cand = make_int4(a.req_order[ri], kh, qb, split);
+            const int4 cand = a.items[idx];
+            const ItemGeo ce = item_geo(a, cand);
+            if (ce.ok) {
+              it = cand;
+              e = ce;
+              break;
+            }
+            flag(a.status, JET_ERR_DEVICE);  // the list holds an item the layout lacks
           }
+        }
+      } else {
+        int k = u == 0 ? int(blockIdx.x) : -1;
+        if (u > 0 && !a.static_only) {
+          if (lane == 0) k = int(gridDim.x) + atomicAdd(a.item_next, 1);
+          k = __shfl_sync(0xffffffffu, k, 0);
+        }
+        int4 cand;
+        if (k >= 0 && nth_item(a, k, lane, &cand)) {
           const ItemGeo ce = item_geo(a, cand);
           if (ce.ok) {
             it = cand;
             e = ce;
-            break;
+          } else if (lane == 0) {
+            flag(a.status, JET_ERR_DEVICE);
           }
-          if (a.sorted) flag(a.status, JET_ERR_DEVICE);  // the list holds an item the layout lacks
         }
+      }
+      if (lane == 0) {
         ring[slot].it = it;
         ring[slot].e = e;
         mbar_arrive(item_full + slot);
-        if (it.x < 0) break;
         // start the query block on its way into L2 (K/V tiles are not
         // prefetched: extra requests in flight only delay the demand loads)
+        if (it.x >= 0) {
 #pragma unroll
-        for (int sl = 0; sl < G::kSlices; ++sl)
-          tma_prefetch_3d(&tmQ, sl * 64, e.kh * g, e.n0 + e.row0);
+          for (int sl = 0; sl < G::kSlices; ++sl)
+            tma_prefetch_3d(&tmQ, sl * 64, e.kh * g, e.n0 + e.row0);
+        }
       }
+      if (__shfl_sync(0xffffffffu, it.x, 0) < 0) break;
     }
   } else if (warp == 0) {
     // ---------------------------------------------------------------- producer
@@ -772,45 +841,52 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         }
       }
       const float inv = l > 0.f ? 1.f / l : 0.f;
+      // 64 columns of O per TMEM round trip, written as two 32-column pieces
 #pragma unroll 1
-      for (int c0 = 0; c0 < DH; c0 += 32) {
-        float ov[32];
-        tmem_ld_32cols(tmem + lane_off + G::kOCol + c0, ov);
+      for (int c0 = 0; c0 < DH; c0 += 64) {
+        float ovp[2][32];
+        tmem_ld_32cols(tmem + lane_off + G::kOCol + c0, ovp[0]);
+        tmem_ld_32cols(tmem + lane_off + G::kOCol + c0 + 32, ovp[1]);
         tmem_wait_ld();
-        if (direct) {
-          // 32 bf16 = four 16-byte pieces per vector; two vectors per 128-byte
-          // row of the stage, pieces rotated so that 8 lanes hit 8 bank groups
 #pragma unroll
-          for (int q = 0; q < 4; ++q)
-            stage[(lane >> 1) * 8 + (lane & 1) * 4 + (q ^ ((lane >> 1) & 3))] =
-                make_uint4(pack_bf16(ov[8 * q] * inv, ov[8 * q + 1] * inv),
-                           pack_bf16(ov[8 * q + 2] * inv, ov[8 * q + 3] * inv),
-                           pack_bf16(ov[8 * q + 4] * inv, ov[8 * q + 5] * inv),
-                           pack_bf16(ov[8 * q + 6] * inv, ov[8 * q + 7] * inv));
-          __syncwarp();
+        for (int hp = 0; hp < 2; ++hp) {
+          const float* ov = ovp[hp];
+          const int cc0 = c0 + 32 * hp;
+          if (direct) {
+            // 32 bf16 = four 16-byte pieces per vector; two vectors per 128-byte
+            // row of the stage, pieces rotated so that 8 lanes hit 8 bank groups
 #pragma unroll
-          for (int s = 0; s < 4; ++s) {
-            const int iv = 8 * s + (lane >> 2), c = lane & 3;
-            const uint4 val = stage[(iv >> 1) * 8 + (iv & 1) * 4 + (c ^ ((iv >> 1) & 3))];
-            if (dst[s] >= 0) *reinterpret_cast<uint4*>(a.o + dst[s] + c0 + c * 8) = val;
+            for (int q = 0; q < 4; ++q)
+              stage[(lane >> 1) * 8 + (lane & 1) * 4 + (q ^ ((lane >> 1) & 3))] =
+                  make_uint4(pack_bf16(ov[8 * q] * inv, ov[8 * q + 1] * inv),
+                             pack_bf16(ov[8 * q + 2] * inv, ov[8 * q + 3] * inv),
+                             pack_bf16(ov[8 * q + 4] * inv, ov[8 * q + 5] * inv),
+                             pack_bf16(ov[8 * q + 6] * inv, ov[8 * q + 7] * inv));
+            __syncwarp();
+#pragma unroll
+            for (int s = 0; s < 4; ++s) {
+              const int iv = 8 * s + (lane >> 2), c = lane & 3;
+              const uint4 val = stage[(iv >> 1) * 8 + (iv & 1) * 4 + (c ^ ((iv >> 1) & 3))];
+              if (dst[s] >= 0) *reinterpret_cast<uint4*>(a.o + dst[s] + cc0 + c * 8) = val;
+            }
+          } else {
+            // 32 f32 = eight 16-byte pieces per vector, one vector per 128-byte
+            // row of the stage, pieces rotated by the row
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              stage[lane * 8 + (q ^ (lane & 7))] =
+                  make_uint4(__float_as_uint(ov[4 * q]), __float_as_uint(ov[4 * q + 1]),
+                             __float_as_uint(ov[4 * q + 2]), __float_as_uint(ov[4 * q + 3]));
+            __syncwarp();
+#pragma unroll
+            for (int s = 0; s < 8; ++s) {
+              const int iv = 4 * s + (lane >> 3), c = lane & 7;
+              const uint4 val = stage[iv * 8 + (c ^ (iv & 7))];
+              if (dst[s] >= 0) *reinterpret_cast<uint4*>(a.o_part + dst[s] + cc0 + c * 4) = val;
+            }
           }
-        } else {
-          // 32 f32 = eight 16-byte pieces per vector, one vector per 128-byte
-          // row of the stage, pieces rotated by the row
-#pragma unroll
-          for (int q = 0; q < 8; ++q)
-            stage[lane * 8 + (q ^ (lane & 7))] =
-                make_uint4(__float_as_uint(ov[4 * q]), __float_as_uint(ov[4 * q + 1]),
-                           __float_as_uint(ov[4 * q + 2]), __float_as_uint(ov[4 * q + 3]));
           __syncwarp();
-#pragma unroll
-          for (int s = 0; s < 8; ++s) {
-            const int iv = 4 * s + (lane >> 3), c = lane & 7;
-            const uint4 val = stage[iv * 8 + (c ^ (iv & 7))];
-            if (dst[s] >= 0) *reinterpret_cast<uint4*>(a.o_part + dst[s] + c0 + c * 4) = val;
-          }
         }
-        __syncwarp();
       }
       // O may be overwritten by the next item's first P V; the ring slot is free
       tc_fence_before();
@@ -965,25 +1041,27 @@ cudaError_t launch_dh(const jet_layout& lay, const jet_dims& d, const AttnPlan& 
   a.items = reinterpret_cast<int4*>(ctrl + 16);
   a.splits = plan.splits;
   a.n_all = (long long)n.R * d.Hkv * plan.qgroups * plan.splits;
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+    return cudaErrorInvalidValue;
+  const int grid = int(std::max<long long>(1, std::min<long long>(sms, a.n_all)));
   // longest-first dynamic order pays for its extra launch only when items are
-  // long and uneven (chunks of 16 key tiles or more)
+  // long and uneven (chunks of 16 key tiles or more); a grid that covers every
+  // slot takes one slot per CTA and needs no shared counter
   a.sorted = plan.chunk >= 16 * kBN;
+  a.static_only = !a.sorted && a.n_all <= grid;
   cudaError_t e = cudaSuccess;
   if (a.sorted)
     e = launch_pdl(attend_items_kernel, dim3(1), dim3(1024), 0, st, a, plan.qgroups, plan.splits);
-  else
-    e = launch_pdl(attend_reset_kernel, dim3(1), dim3(32), 0, st, a.item_next);
+  else if (!a.static_only)
+    e = launch_pdl(attend_reset_kernel, dim3(1), dim3(128), 0, st, a.item_next, a.prefix_offset,
+                   a.row_offset, a.req_order, a.row_cand, a.cand_row_offset, a.R, a.N, a.C);
   if (e != cudaSuccess) return e;
   const size_t smem = Geo<DH>::kBytes + 1024;
   e = cudaFuncSetAttribute(attend_prefix_tc_kernel<DH>,
                            cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
   if (e != cudaSuccess) return e;
-  int dev = 0, sms = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
-    return cudaErrorInvalidValue;
-  const long long max_items = (long long)n.R * d.Hkv * plan.qgroups * plan.splits;
-  const int grid = int(std::max<long long>(1, std::min<long long>(sms, max_items)));
   e = launch_pdl(attend_prefix_tc_kernel<DH>, dim3(grid), dim3(kThreads), smem, st, tmQ, tmK, tmV,
                  tmKc, tmVc, a);
   if (e != cudaSuccess || plan.splits <= 1) return e;
