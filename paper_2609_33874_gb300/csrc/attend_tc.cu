@@ -969,16 +969,32 @@ attend_combine_kernel(const int32_t* __restrict__ prefix_offset, const int32_t* 
 #pragma unroll
   for (int i = 0; i < PER; ++i) acc[i] = 0.f;
   float m = -INFINITY, l = 0.f;
-  for (int s = 0; s < splits_r; ++s) {
-    const size_t base = (size_t(s) * N + n) * Hq + h;
-    const float2 ml = ml_part[base];
-    if (!(ml.y > 0.f)) continue;
-    const float mn = fmaxf(m, ml.x);
-    const float fa = exp2f(m - mn), fb = exp2f(ml.x - mn);
+  // four chunks' partials at a time, every load issued before the first is
+  // used (the chunks are combined in order)
+  constexpr int kGroup = 4;
+  for (int s0 = 0; s0 < splits_r; s0 += kGroup) {
+    float2 ml[kGroup];
+    float v[kGroup][PER];
 #pragma unroll
-    for (int i = 0; i < PER; ++i) acc[i] = acc[i] * fa + o_part[base * DH + lane + 32 * i] * fb;
-    l = l * fa + ml.y * fb;
-    m = mn;
+    for (int q = 0; q < kGroup; ++q) {
+      ml[q] = make_float2(-INFINITY, 0.f);
+      if (s0 + q < splits_r) {
+        const size_t base = (size_t(s0 + q) * N + n) * Hq + h;
+        ml[q] = ml_part[base];
+#pragma unroll
+        for (int i = 0; i < PER; ++i) v[q][i] = o_part[base * DH + lane + 32 * i];
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < kGroup; ++q) {
+      if (!(ml[q].y > 0.f)) continue;
+      const float mn = fmaxf(m, ml[q].x);
+      const float fa = exp2f(m - mn), fb = exp2f(ml[q].x - mn);
+#pragma unroll
+      for (int i = 0; i < PER; ++i) acc[i] = acc[i] * fa + v[q][i] * fb;
+      l = l * fa + ml[q].y * fb;
+      m = mn;
+    }
   }
   const float inv = l > 0.f ? 1.f / l : 0.f;
 #pragma unroll

@@ -143,10 +143,6 @@ __device__ __forceinline__ uint32_t a_off(int r, int chunk) {
   return uint32_t(r) * kC + (uint32_t(chunk ^ (r & 15)) << 2);
 }
 
-__device__ __forceinline__ float a_at(const float* A, int r, int i) {
-  return A[a_off(r, i >> 2) + (i & 3)];
-}
-
 // T = (I + A)^{-1} (unit lower triangular) in f32, 64 floats a row, in the
 // token tiles' two 8 KB Q slots (rows 32 s .. 32 s + 31 in slice s): the Q of
 // the chunk is no longer needed when it is formed
@@ -158,7 +154,9 @@ __device__ __forceinline__ float* t_row(uint8_t* sm, int r) {
 // (i, j): column j of T_ii), then the blocks below them level by level
 // (d = i - j = 1, 2, 3): T_ij = -T_ii P_ij with P_ij = sum_{k=j}^{i-1} A_ik T_kj,
 // P_ij held in the unused block (j, i) above the diagonal. Every block of T
-// at or below the diagonal is written (zeros above the diagonal of T_ii).
+// at or below the diagonal is written (zeros above the diagonal of T_ii). In
+// the block products a thread forms four adjacent outputs of one row from
+// 16-byte loads.
 __device__ __forceinline__ void invert_unit_lower(const float* __restrict__ A, uint8_t* sm,
                                                   int tid) {
   if (tid < 64) {
@@ -168,7 +166,15 @@ __device__ __forceinline__ void invert_unit_lower(const float* __restrict__ A, u
     for (int r = 0; r < 16; ++r) {
       float s = r == jj ? 1.f : 0.f;
 #pragma unroll
-      for (int i = 0; i < r; ++i) s = fmaf(-a_at(A, 16 * bi + r, 16 * bi + i), x[i], s);
+      for (int q = 0; q < 4; ++q) {
+        if (4 * q < r) {
+          const float4 a4 = *reinterpret_cast<const float4*>(A + a_off(16 * bi + r, 4 * bi + q));
+          const float av[4] = {a4.x, a4.y, a4.z, a4.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            if (4 * q + e < r) s = fmaf(-av[e], x[4 * q + e], s);
+        }
+      }
       x[r] = s;
     }
 #pragma unroll
@@ -177,22 +183,47 @@ __device__ __forceinline__ void invert_unit_lower(const float* __restrict__ A, u
   __syncthreads();
 #pragma unroll
   for (int d = 1; d < 4; ++d) {
-    for (int e = tid; e < (4 - d) * 256; e += kThreads) {
-      const int jb = e >> 8, ib = jb + d, r = (e >> 4) & 15, cc = e & 15;
-      float s = 0.f;
-#pragma unroll 4
-      for (int k = 16 * jb; k < 16 * ib; ++k)
-        s = fmaf(a_at(A, 16 * ib + r, k), t_row(sm, k)[16 * jb + cc], s);
-      t_row(sm, 16 * jb + r)[16 * ib + cc] = s;
+    // task t: block (jb, jb + d), row r, columns 4 c4 .. 4 c4 + 3
+    const int t = tid;
+    const bool act = t < (4 - d) * 64;
+    const int jb = t >> 6, ib = jb + d, r = (t >> 2) & 15, c4 = t & 3;
+    if (act) {
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int k4 = 4 * jb; k4 < 4 * ib; ++k4) {
+        const float4 a4 = *reinterpret_cast<const float4*>(A + a_off(16 * ib + r, k4));
+        const float av[4] = {a4.x, a4.y, a4.z, a4.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float4 t4 =
+              *reinterpret_cast<const float4*>(t_row(sm, 4 * k4 + e) + 16 * jb + 4 * c4);
+          acc.x = fmaf(av[e], t4.x, acc.x);
+          acc.y = fmaf(av[e], t4.y, acc.y);
+          acc.z = fmaf(av[e], t4.z, acc.z);
+          acc.w = fmaf(av[e], t4.w, acc.w);
+        }
+      }
+      *reinterpret_cast<float4*>(t_row(sm, 16 * jb + r) + 16 * ib + 4 * c4) = acc;
     }
     __syncthreads();
-    for (int e = tid; e < (4 - d) * 256; e += kThreads) {
-      const int jb = e >> 8, ib = jb + d, r = (e >> 4) & 15, cc = e & 15;
+    if (act) {
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
       const float* ti = t_row(sm, 16 * ib + r) + 16 * ib;
-      float s = 0.f;
 #pragma unroll
-      for (int k = 0; k < 16; ++k) s = fmaf(ti[k], t_row(sm, 16 * jb + k)[16 * ib + cc], s);
-      t_row(sm, 16 * ib + r)[16 * jb + cc] = -s;
+      for (int k4 = 0; k4 < 4; ++k4) {
+        const float4 a4 = *reinterpret_cast<const float4*>(ti + 4 * k4);
+        const float av[4] = {a4.x, a4.y, a4.z, a4.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float4 p4 =
+              *reinterpret_cast<const float4*>(t_row(sm, 16 * jb + 4 * k4 + e) + 16 * ib + 4 * c4);
+          acc.x = fmaf(av[e], p4.x, acc.x);
+          acc.y = fmaf(av[e], p4.y, acc.y);
+          acc.z = fmaf(av[e], p4.z, acc.z);
+          acc.w = fmaf(av[e], p4.w, acc.w);
+        }
+      }
+      *reinterpret_cast<float4*>(t_row(sm, 16 * ib + r) + 16 * jb + 4 * c4) =
+          make_float4(-acc.x, -acc.y, -acc.z, -acc.w);
     }
     __syncthreads();
   }
