@@ -24,7 +24,7 @@ namespace {
 constexpr int kDK = 128;        // key dimension handled (rows of S)
 constexpr int kCols = 32;       // value columns per CTA
 constexpr int kThreads = 128;   // 4 warps x 32 rows
-constexpr int kWin = 32;        // fed tokens staged in shared memory at a time
+constexpr int kWin = 16;        // fed tokens staged in shared memory at a time
 constexpr int kMeta = 64;       // candidates whose lengths are staged at a time
 
 __device__ __forceinline__ float4 f4_fma(float a, float4 x, float4 y) {
@@ -153,8 +153,11 @@ __device__ __forceinline__ float4 token_step(float4 (&S)[8], int wt, const T (*w
 // q_rows (optional, [N, Hl, dk]): every row's q; the request's shared row then
 // reads the prefix state, o = S_r^T q / sqrt(dk), and o holds all N rows
 // (fed token f at row f + r + 1) instead of the fed tokens alone.
+// bf16: 72 registers and 28 KB of shared memory, so that seven CTAs share an
+// SM (a (32 requests x 16 heads x 4 slices) grid then fills 1.93 waves of
+// 1,064 CTAs instead of 2.25 waves of 912)
 template <typename T, bool DELTA>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, sizeof(T) == 2 ? 7 : 3)
 fork_kernel(const int32_t* __restrict__ cand_offset, const int32_t* __restrict__ cand_row_offset,
             const int32_t* __restrict__ tgt_offset, const int32_t* __restrict__ row_offset,
             int R, int C, int F, int Hl, int dv, const float* __restrict__ s_prefix,
