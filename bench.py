@@ -782,15 +782,21 @@ def run_prefill(args):
                   + 2 * R * w.Hl * w.dk * w.dv * 4)
         # per token and head: u = k^T S, the rank-one update, o = S^T q
         sflops = float(p.total_prefix * w.Hl * w.dk * w.dv * (6 if args.rule == "delta" else 4))
-        # the scan is sequential per (request, head): it is bound by fp32 FMA
-        # issue, 152 SMs x 128 lanes x 2 flop per clock at the maximum SM clock
+        # the recurrence's own work against the fp32 FMA peak (152 SMs x 128
+        # lanes x 2 flop per clock at the maximum SM clock), the bound of the
+        # sequential form; bf16 128 x 128 states run the chunked form, which
+        # moves most of that work onto the tensor cores and is bound by its
+        # per-chunk chain of MMAs and barriers
         alu_peak = 152 * 128 * 2 * peaks["sm_max_mhz"] * 1e6 / 1e12
         tf_s = sflops / (ms_s / 1e3) / 1e12
         sroof = dict(bound="alu", achieved=round(tf_s, 2), peak=round(alu_peak, 1),
                      unit="TFLOP/s", frac=round(tf_s / alu_peak, 4),
                      hbm_frac=round(sbytes / (ms_s / 1e3) / 1e9 / peaks["hbm"], 4))
-        sroof.update(kernel=f"jet_prefill_state (scan_kernel, {args.rule} rule)",
-                     peak_basis="fp32 FMA: 152 SMs x 128 lanes x 2 flop x max SM clock",
+        chunked = w.dtype == "bf16" and w.dk == 128 and w.dv == 128
+        sroof.update(kernel=(f"jet_prefill_state ({'scan_tc_kernel, chunked' if chunked else 'scan_kernel'}"
+                             f", {args.rule} rule)"),
+                     peak_basis="recurrence work (6 or 4 dk dv flop per token and head) against "
+                                "fp32 FMA: 152 SMs x 128 lanes x 2 flop x max SM clock",
                      algorithmic_flops=sflops, algorithmic_bytes=sbytes, traffic=None,
                      peak_source=peaks["source"])
         parts["state"] = dict(ms=round(ms_s, 4), roofline=sroof, launches=n_scan)

@@ -241,8 +241,11 @@ jet_status jet_prefill_attend(const jet_layout* lay, const jet_dims* dims, const
  *   o       [total_prefix, Hl, dv] dims.dtype  each prefix token's output
  *   s_out   [R, Hl, dk, dv] float32   the state after the prefix: the
  *           s_prefix every candidate forks from (Sec. 4.1)
- * Tokens run one after another within a request (requests, heads and
- * 32-column slices of the state run in parallel).
+ * Requests and heads run in parallel. bf16 states of 128 x 128 take the
+ * chunked form on the tensor cores (64 tokens at a time, one CTA per
+ * request and head; an exact rearrangement of the recurrence with float32-
+ * like accuracy); float32 and other state shapes run the tokens one after
+ * another (32- or 64-column slices of the state in parallel).
  */
 jet_status jet_prefill_state(const jet_layout* lay, const jet_dims* dims, int32_t rule,
                              const float* s_init, const void* q, const void* k, const void* v,
