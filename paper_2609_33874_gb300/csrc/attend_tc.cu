@@ -11,10 +11,12 @@
 //   warp 1      TMEM allocator, MMA issuer:
 //                 S_j  = Q K_j^T   (M 128 vectors, N 64 keys, K d)   -> TMEM
 //                 O   += P_j V_j   (M 128 vectors, N d, K 64 keys)   -> TMEM
-//               V_j is the MN-major B operand (d contiguous in memory).
+//               P_j is read from TMEM, V_j is the MN-major B operand (d
+//               contiguous in memory).
 //   warps 2..5  softmax: thread = query vector = TMEM lane. Reads S_j, keeps a
 //               running max m and sum l in base 2, writes P_j = 2^(s - m) as
-//               bf16 into a 128-byte-swizzled shared tile; O is rescaled in
+//               bf16 pairs into its own TMEM lane, where the P V MMA reads it
+//               as its A operand (no shared-memory round trip); O is rescaled in
 //               TMEM only when the row max grows by more than 8 (a factor 256),
 //               so P stays <= 256 and rescales are rare; at the item's end
 //               they write its output through shared memory (coalesced).
@@ -50,13 +52,15 @@ struct Geo {
   static constexpr int kSlices = DH / 64;                   // 64-wide d slices
   static constexpr uint32_t kQBytes = kBV * DH * 2;         // query block
   static constexpr uint32_t kKVBytes = kBN * DH * 2;        // one K (or V) tile
-  static constexpr uint32_t kPBytes = kBV * kBN * 2;        // one P tile
   static constexpr uint32_t kOffK = kQBytes;                // stage s: K at kOffK + s * 2 kKV
-  static constexpr uint32_t kOffP = kQBytes + kStages * 2 * kKVBytes;
-  static constexpr uint32_t kOffBar = kOffP + 2 * kPBytes;
+  // the output stage: 32 rows of 128 bytes per softmax warp
+  static constexpr uint32_t kOffStage = kQBytes + kStages * 2 * kKVBytes;
+  static constexpr uint32_t kOffBar = kOffStage + 4 * 32 * 128;
   static constexpr uint32_t kBytes = kOffBar + 512;
-  static constexpr uint32_t kTmemCols = (2 * kBN + DH) <= 256 ? 256 : 512;
+  // TMEM: the two S buffers, O, then the two P buffers (bf16 pairs, 32 columns)
+  static constexpr uint32_t kTmemCols = (2 * kBN + DH + 2 * (kBN / 2)) <= 256 ? 256 : 512;
   static constexpr uint32_t kOCol = 2 * kBN;                // O after the two S buffers
+  static constexpr uint32_t kPCol = 2 * kBN + DH;           // P buffer b at kPCol + 32 b
 };
 
 struct AttArgs {
@@ -640,12 +644,13 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
             if (o_ready && mbar_test(p_full + b, (Tj >> 1) & 1) &&
                 mbar_test(v_full + s, (Tj / kStages) & 1)) {
               tc_fence_after();
-              const uint32_t ps = smem_u32(smem + G::kOffP + b * G::kPBytes);
+              // P_j from TMEM (8 columns = 16 keys per instruction), V_j from shared memory
+              const uint32_t pt = tmem + G::kPCol + uint32_t(b) * (kBN / 2);
               const uint32_t vs = smem_u32(smem + G::kOffK + s * 2 * G::kKVBytes + G::kKVBytes);
 #pragma unroll
               for (int k = 0; k < kBN / 16; ++k)
-                mma_f16(tmem + G::kOCol, desc_k_sw128(ps + 32 * k),
-                        desc_mn_sw128(vs + k * 16 * 128, kBN * 128), id_o, (jo | k) != 0);
+                mma_f16_ta(tmem + G::kOCol, pt + uint32_t(8 * k),
+                           desc_mn_sw128(vs + k * 16 * 128, kBN * 128), id_o, (jo | k) != 0);
               mma_commit(p_free + b);
               mma_commit(v_empty + s);
               ++jo;
@@ -671,10 +676,10 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
     const int q4 = warp & 3;
     const int i = q4 * 32 + lane;  // query vector within the block = TMEM lane
     const uint32_t lane_off = uint32_t(q4 * 32) << 16;
-    // the output is transposed through this warp's own 32 rows of P buffer 0
-    // (4 KB, free once the item's last P V has completed) so that every global
-    // store covers whole 64- or 128-byte pieces of one vector's output
-    uint4* stage = reinterpret_cast<uint4*>(smem + G::kOffP + q4 * 32 * 128);
+    // the output is transposed through this warp's own 4 KB of the output
+    // stage so that every global store covers whole 64- or 128-byte pieces of
+    // one vector's output
+    uint4* stage = reinterpret_cast<uint4*>(smem + G::kOffStage + q4 * 32 * 128);
     // the query blocks arrive by TMA (rows [0, rb g)); zero the rows past them
     // once so that no stale shared memory enters the MMA
     if (i >= rb * g) {
@@ -786,26 +791,26 @@ attend_prefix_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
           }
           m_used = m_new;
         }
-        // P = 2^(s - m_used) as bf16, 128-byte swizzled; the row sum uses the
-        // rounded values, which are what the tensor core multiplies
-        uint8_t* pb = smem + G::kOffP + b * G::kPBytes;
-        float ps[8];  // one partial sum per 16-byte chunk, added as a tree
+        // P = 2^(s - m_used) as bf16 pairs into this row's TMEM lane (the P V
+        // MMA's A operand); the row sum uses the rounded values, which are what
+        // the tensor core multiplies
+        uint32_t pw[kBN / 2];
+        float ps[8];  // one partial sum per 8 keys, added as a tree
 #pragma unroll
         for (int cc = 0; cc < 8; ++cc) {
-          uint32_t w[4];
           ps[cc] = 0.f;
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const float x0 = ex2(sv[cc * 8 + 2 * q] - m_used);
             const float x1 = ex2(sv[cc * 8 + 2 * q + 1] - m_used);
-            w[q] = pack_bf16(x0, x1);
-            const __nv_bfloat162 hb = *reinterpret_cast<const __nv_bfloat162*>(&w[q]);
+            pw[cc * 4 + q] = pack_bf16(x0, x1);
+            const __nv_bfloat162 hb = *reinterpret_cast<const __nv_bfloat162*>(&pw[cc * 4 + q]);
             ps[cc] += __bfloat162float(hb.x) + __bfloat162float(hb.y);
           }
-          *reinterpret_cast<uint4*>(pb + sw128(i, cc)) = make_uint4(w[0], w[1], w[2], w[3]);
         }
+        tmem_st_32cols_u32(tmem + lane_off + G::kPCol + uint32_t(b) * (kBN / 2), pw);
         l += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
-        fence_proxy_async_smem();
+        tmem_wait_st();
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(p_full + b);
