@@ -138,17 +138,19 @@ def test_prefill_state(cuda, rule, dtype):
         _check_scan_out(got_o, ref_o, p.bf16)
 
 
-def test_prefill_state_full_hybrid(cuda):
-    # the hybrid workload's prefixes (32 requests x 512 tokens, 16 heads)
+@pytest.mark.parametrize("rule", ["delta", "gla"])
+def test_prefill_state_full_hybrid(cuda, rule):
+    # the hybrid workload's prefixes (32 requests x 512 tokens, 16 heads): the
+    # chunked scan in the launch configuration the bench times
     p = jet_synth.make_problem("ordinal_hybrid")
-    got_o, got_s = _scan(cuda, p, "delta", True)
+    got_o, got_s = _scan(cuda, p, rule, True)
     sub = [0, 13, 31]
     off = np.concatenate([[0], np.cumsum(p.prefix_len)])
     rows = np.concatenate([np.arange(off[r], off[r + 1]) for r in sub])
     sel = lambda n: p.f32(n)[rows]  # noqa: E731
     ref_o, ref_s = O.prefill_state(p.prefix_len[sub], p.f32("s_prefix")[sub], sel("lq_pre"),
                                    sel("lk_pre"), sel("lv_pre"), sel("alpha_pre"),
-                                   sel("beta_pre"))
+                                   sel("beta_pre"), rule)
     rel = np.abs(got_s[sub] - ref_s).max() / np.abs(ref_s).max()
     assert rel <= TOL_FORK_REL, f"state error {rel}"
     _check_scan_out(got_o[rows], ref_o, True)
@@ -211,3 +213,21 @@ def test_prefill_state_chunked(cuda, rule, alpha_scale):
               f"out max {np.abs(got_o - ref_o).max():.2e}")
         assert rel <= TOL_FORK_REL, f"state error {rel}"
         _check_scan_out(got_o, ref_o, True)
+
+
+def test_prefill_state_chunked_long(cuda):
+    # long prefixes through the chunked scan: 2,000 and 1,500 tokens (32 and
+    # 24 chunks, the last ones ragged), so a start state is carried through
+    # many chunk boundaries and both K buffers are reused many times
+    w = dataclasses.replace(jet_synth.WORKLOADS["ordinal_hybrid"], Hl=2, dtype="bf16")
+    pl = [2000, 1500]
+    R = len(pl)
+    p = jet_synth.custom_problem(w, pl, [1] * R, [1] * R, [0] * R, seed=98)
+    got_o, got_s = _scan(cuda, p, "delta", True)
+    ref_o, ref_s = O.prefill_state(p.prefix_len, p.f32("s_prefix"), p.f32("lq_pre"),
+                                   p.f32("lk_pre"), p.f32("lv_pre"), p.f32("alpha_pre"),
+                                   p.f32("beta_pre"), "delta")
+    rel = np.abs(got_s - ref_s).max() / np.abs(ref_s).max()
+    print(f"chunked scan over 2,000 / 1,500 tokens: state rel {rel:.2e}")
+    assert rel <= TOL_FORK_REL, f"state error {rel}"
+    _check_scan_out(got_o, ref_o, True)
