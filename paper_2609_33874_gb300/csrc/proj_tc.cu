@@ -46,7 +46,7 @@ constexpr int kThreads = 192;
 constexpr int kMaxNt = 256;
 constexpr uint64_t kDrainNs = 200000000ull;
 constexpr int kSmemLimit = 232448;
-// up-half exchange (64 lanes x 32 columns f32) + barriers and flags
+// gate/up exchange (16 columns x 128 lanes f32) + barriers and flags
 constexpr int kFixedSmem = 64 * 32 * 4 + 32 * 8 + 64;
 
 struct ProjArgs {
@@ -79,16 +79,24 @@ __device__ __forceinline__ Unit unit_of(const ProjArgs& a, int u) {
   return x;
 }
 
-template <int EPI>
+// P2: clusters of two CTAs, each unit a 256-row weight slice (the even CTA's
+// 128 rows, then the odd one's) against one token tile; each CTA loads its own
+// weight tile and half of the token tile (the even CTA the first Nt / 2 rows),
+// both CTAs' loads complete on the even CTA's stage barrier, the even CTA
+// issues M = 256 MMAs (cta_group::2) into both CTAs' TMEM, the commits reach
+// both CTAs' barriers, and each CTA runs the epilogue of its own 128 rows. Per
+// stage a CTA takes in 16 KB of weights and Nt x 64 bytes of rows for
+// 128 x Nt outputs, against 16 KB + Nt x 128 bytes alone.
+template <int EPI, bool P2>
 __global__ void __launch_bounds__(kThreads, 1)
 proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
                const ProjArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  const uint32_t a_bytes = kBM * 128, b_bytes = uint32_t(a.Nt) * 128;
+  const uint32_t a_bytes = kBM * 128, b_bytes = uint32_t(P2 ? a.Nt / 2 : a.Nt) * 128;
   const uint32_t stage_bytes = a.pair * a_bytes + b_bytes;
-  float* upx = reinterpret_cast<float*>(smem + size_t(a.stages) * stage_bytes);  // [64][32]
+  float* upx = reinterpret_cast<float*>(smem + size_t(a.stages) * stage_bytes);  // [16][128]
   uint64_t* full = reinterpret_cast<uint64_t*>(upx + 64 * 32);
   uint64_t* empty = full + a.stages;
   uint64_t* tfull = empty + a.stages;
@@ -99,6 +107,10 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
   volatile int* epi_abort = abort_flag + 1;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // P2: this CTA's rank in its pair, the pair's number and the pairs
+  const uint32_t rank = P2 ? cluster_rank() : 0u;
+  const int cid = P2 ? int(blockIdx.x >> 1) : int(blockIdx.x);
+  const int ncl = P2 ? int(gridDim.x >> 1) : int(gridDim.x);
   if (threadIdx.x == 0) {
     for (int s = 0; s < a.stages; ++s) {
       mbar_init(full + s, 1);
@@ -106,7 +118,7 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(tfull + b, 1);
-      mbar_init(tempty + b, 4);
+      mbar_init(tempty + b, P2 ? 8 : 4);  // P2: both CTAs' epilogue warps
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -119,11 +131,17 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
   }
   pdl_begin();
   if (warp == 1) {
-    tmem_alloc(tmem_slot, a.tmem_cols);
-    tmem_relinquish();
+    if (P2) {
+      tmem_alloc_pair(tmem_slot, a.tmem_cols);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(tmem_slot, a.tmem_cols);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
   __syncthreads();
+  if (P2) cluster_sync();  // the even CTA's barriers are initialised before any remote use
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -134,9 +152,10 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
       int s = 0;
       uint32_t ph = 0, issued = 0, issued_par = 0;
       bool ok = true, hold = a.hold_first != 0;
-      for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x) {
+      for (int u = cid; ok && u < a.units; u += ncl) {
         const Unit x = unit_of(a, u);
-        const int o0 = x.ot * a.pair * kBM, t0 = x.t0;
+        const int o0 = P2 ? (2 * x.ot + int(rank)) * kBM : x.ot * a.pair * kBM;
+        const int t0 = x.t0 + (P2 ? int(rank) * (a.Nt / 2) : 0);
         for (int kb = x.kb0; kb < x.kb1; ++kb) {
           if (!mbar_wait(empty + s, ph ^ 1u, a.wait_ns, abort_flag)) {
             ok = false;
@@ -145,6 +164,15 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
           uint8_t* sa = smem + size_t(s) * stage_bytes;
           if (hold) {
             hold = false;  // test hook: this stage never fills
+          } else if (P2) {
+            // both CTAs' bytes complete on the even CTA's barrier, which
+            // expects them all; the odd CTA's may land before that arrive
+            const uint32_t bar = mapa_shared(full + s, 0);
+            if (rank == 0) mbar_arrive_expect_tx(full + s, 2 * stage_bytes);
+            tma_load_2d_pair(sa, &tmW, bar, kb * kBK, o0, pol_w);
+            tma_load_2d_pair(sa + a_bytes, &tmX, bar, kb * kBK, t0, pol_x);
+            issued |= 1u << s;
+            issued_par = (issued_par & ~(1u << s)) | (ph << s);
           } else {
             mbar_arrive_expect_tx(full + s, stage_bytes);
             for (int t = 0; t < a.pair; ++t)
@@ -162,18 +190,26 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
       if (!ok) {
         *abort_flag = 1;
         flag(a.status, JET_ERR_TIMEOUT);
-        for (int t = 0; t < a.stages; ++t)
-          if (issued & (1u << t)) mbar_wait(full + t, (issued_par >> t) & 1u, kDrainNs, nullptr);
+        // let the copies in flight land (P2: the even CTA's barriers count
+        // both CTAs' bytes; the odd CTA waits out a fixed bounded time)
+        if (!P2 || rank == 0) {
+          for (int t = 0; t < a.stages; ++t)
+            if (issued & (1u << t)) mbar_wait(full + t, (issued_par >> t) & 1u, kDrainNs, nullptr);
+        } else if (issued) {
+          const uint64_t t0 = global_timer_ns();
+          while (global_timer_ns() - t0 < kDrainNs / 16) {
+          }
+        }
       }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      const uint32_t idesc = idesc_bf16_f32(kBM, a.Nt);
+    if (lane == 0 && (!P2 || rank == 0)) {
+      const uint32_t idesc = idesc_bf16_f32(P2 ? 2 * kBM : kBM, a.Nt);
       int s = 0, local = 0;
       uint32_t ph = 0;
       bool ok = true;
-      for (int u = blockIdx.x; ok && u < a.units; u += gridDim.x, ++local) {
+      for (int u = cid; ok && u < a.units; u += ncl, ++local) {
         const int buf = local % a.nbuf;
         const uint32_t tph = (local / a.nbuf) & 1;
         if (!mbar_wait(tempty + buf, tph ^ 1u, a.wait_ns, abort_flag)) {
@@ -191,33 +227,49 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
           tc_fence_after();
           const uint32_t sa = smem_u32(smem + size_t(s) * stage_bytes);
           const uint32_t sb = sa + a.pair * a_bytes;
-          for (int t = 0; t < a.pair; ++t) {
+          if (P2) {
 #pragma unroll
             for (int k = 0; k < 4; ++k)
-              mma_f16(d_tmem + t * a.acc_cols, desc_k_sw128(sa + t * a_bytes + 32 * k),
-                      desc_k_sw128(sb + 32 * k), idesc, (kb - x.kb0) != 0 || k != 0);
+              mma_f16_pair(d_tmem, desc_k_sw128(sa + 32 * k), desc_k_sw128(sb + 32 * k), idesc,
+                           (kb - x.kb0) != 0 || k != 0);
+            mma_commit_pair(empty + s, 0x3);  // both CTAs' stage s is free
+          } else {
+            for (int t = 0; t < a.pair; ++t) {
+#pragma unroll
+              for (int k = 0; k < 4; ++k)
+                mma_f16(d_tmem + t * a.acc_cols, desc_k_sw128(sa + t * a_bytes + 32 * k),
+                        desc_k_sw128(sb + 32 * k), idesc, (kb - x.kb0) != 0 || k != 0);
+            }
+            mma_commit(empty + s);
           }
-          mma_commit(empty + s);
           if (++s == a.stages) {
             s = 0;
             ph ^= 1u;
           }
         }
         if (!ok) break;
-        mma_commit(tfull + buf);
+        if (P2)
+          mma_commit_pair(tfull + buf, 0x3);
+        else
+          mma_commit(tfull + buf);
       }
       if (!ok) {
         *abort_flag = 1;
         flag(a.status, JET_ERR_TIMEOUT);
-        mma_commit(drain);
+        if (P2)
+          mma_commit_pair(drain, 0x1);
+        else
+          mma_commit(drain);
         mbar_wait(drain, 0, kDrainNs, nullptr);
       }
     }
   } else {
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;            // TMEM lane quadrant this warp may access
+    // P2: the odd CTA's warps release the accumulator on the even CTA's barrier
+    const uint32_t tempty_even = P2 ? mapa_shared(tempty, 0) : 0u;
     int local = 0;
-    for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++local) {
+    for (int u = cid; u < a.units; u += ncl, ++local) {
       const int buf = local % a.nbuf;
       const uint32_t tph = (local / a.nbuf) & 1;
       const Unit x = unit_of(a, u);
@@ -229,7 +281,8 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
       tc_fence_after();
       const int ncols = min(a.Nt, a.N - t0);
       for (int pt = 0; pt < a.pair; ++pt) {
-      const int ot = x.ot * a.pair + pt;  // this accumulator's weight tile
+      // this accumulator's weight tile
+      const int ot = P2 ? 2 * x.ot + int(rank) : x.ot * a.pair + pt;
       const uint32_t tl = tmem_base + uint32_t(buf * a.pair + pt) * a.acc_cols +
                           (uint32_t(32 * q) << 16);
       for (int c0 = 0; c0 < ncols; c0 += 32) {
@@ -247,23 +300,29 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
               if (i < nc) pp[size_t(i) * a.O] = v[i];
           }
         } else if (EPI == kProjSwiGLU) {
-          // lanes 64..127 hold the up features: hand them to the gate lanes
-          if (q >= 2) {
+          // lanes 0..63 hold the gate features, lanes 64..127 the matching up
+          // features: each half hands the other its values of 16 of the 32
+          // columns (column-major exchange, one 128-word row per column), then
+          // every warp forms SiLU(gate) * up for its 16 columns - the gate half
+          // columns 0..15, the up half 16..31
+          const bool gate = q < 2;
+          const int hb = gate ? 16 : 0;  // the columns this thread hands over
 #pragma unroll
-            for (int i = 0; i < 32; ++i) upx[(32 * (q - 2) + lane) * 32 + ((i + lane) & 31)] = v[i];
-          }
+          for (int j = 0; j < 16; ++j) upx[j * 128 + 32 * q + lane] = v[hb + j];
           named_bar_sync(1, 128);
-          if (q < 2) {
-            const int f = ot * 64 + 32 * q + lane;  // output feature
-            if (f < a.O / 2) {
+          const int f = ot * 64 + 32 * (q & 1) + lane;  // output feature
+          const int cb = gate ? 0 : 16;                 // the columns this thread forms
+          if (f < a.O / 2) {
 #pragma unroll
-              for (int i = 0; i < 32; ++i) {
-                if (i < nc) {
-                  const float up = upx[(32 * q + lane) * 32 + ((i + lane) & 31)];
-                  const float g = v[i];
-                  const float y = g / (1.f + __expf(-g)) * up;
-                  a.out[size_t(t0 + c0 + i) * a.ldo + f] = __float2bfloat16_rn(y);
-                }
+            for (int j = 0; j < 16; ++j) {
+              if (cb + j < nc) {
+                const float other = upx[j * 128 + 32 * (q ^ 2) + lane];
+                const float g = gate ? v[j] : other;
+                const float up = gate ? other : v[16 + j];
+                // SiLU(g) up = g up / (1 + e^-g), the quotient by the fast
+                // reciprocal (the result is rounded to bf16)
+                const float y = __fdividef(g * up, 1.f + __expf(-g));
+                a.out[size_t(t0 + c0 + cb + j) * a.ldo + f] = __float2bfloat16_rn(y);
               }
             }
           }
@@ -286,16 +345,27 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
       }  // the unit's weight tiles
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(tempty + buf);
+      if (lane == 0) {
+        if (P2 && rank != 0)
+          mbar_arrive_cluster(tempty_even + uint32_t(buf) * 8u);
+        else
+          mbar_arrive(tempty + buf);
+      }
     }
     if (*epi_abort) flag(a.status, JET_ERR_TIMEOUT);
   }
 
   tc_fence_before();
   __syncthreads();
+  // P2: neither CTA leaves (or frees its TMEM) while the partner's MMAs or
+  // copies may still use its shared memory or TMEM
+  if (P2) cluster_sync();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, a.tmem_cols);
+    if (P2)
+      tmem_dealloc_pair(tmem_base, a.tmem_cols);
+    else
+      tmem_dealloc(tmem_base, a.tmem_cols);
   }
 }
 
@@ -318,7 +388,7 @@ __global__ void proj_reduce_kernel(const float* __restrict__ part, int splits, i
       g += row[gr];
       up += row[gr + 64];
     }
-    out[size_t(n) * ldo + c] = __float2bfloat16_rn(g / (1.f + __expf(-g)) * up);
+    out[size_t(n) * ldo + c] = __float2bfloat16_rn(__fdividef(g * up, 1.f + __expf(-g)));
   } else {
     float acc = 0.f;
     for (int s = 0; s < splits; ++s) acc += part[(size_t(s) * N + n) * O + c];
@@ -435,6 +505,30 @@ int sm_count() {
   return n;
 }
 
+// clusters of two CTAs of `kern` that can be resident at once (one CTA per SM:
+// the SM pairs the GPCs offer); asked once per kernel
+template <typename K>
+int max_pairs(K kern, size_t smem) {
+  static int cached = 0;
+  if (cached > 0) return cached;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(2);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute cl{};
+  cl.id = cudaLaunchAttributeClusterDimension;
+  cl.val.clusterDim.x = 2;
+  cl.val.clusterDim.y = 1;
+  cl.val.clusterDim.z = 1;
+  cfg.attrs = &cl;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n < 1)
+    n = std::max(1, sm_count() / 2);
+  cached = n;
+  return n;
+}
+
 // the RMSNorm a residual projection's output feeds (h null: none)
 struct Norm {
   const void* g;
@@ -448,11 +542,14 @@ cudaError_t launch_reduce(const ProjArgs& a, float* part, int N, int O, void* ou
 
 struct Tiling {
   int n_tt, Nt, otiles, pair, groups, nkb, splits;
+  bool p2;  // clusters of two CTAs, 256 weight rows per unit
 };
 
-// token tiles of at most 256 rows; K split until the units cover 152 SMs
-// twice, keeping at least 8 K slices per unit. A function of the shapes only,
-// so that the workspace planned for a call matches the launch.
+// token tiles of at most 256 rows (a multiple of 16: each CTA of a pair holds
+// half); units of 256 weight rows on CTA pairs; K split while the units still
+// fit the 76 SM pairs once, keeping at least 8 K slices per unit. A function
+// of the shapes only, so that the workspace planned for a call matches the
+// launch.
 constexpr int kPlanSMs = 152;
 Tiling tiling(int N, int O, int K, bool split) {
   Tiling t{};
@@ -460,14 +557,14 @@ Tiling tiling(int N, int O, int K, bool split) {
   t.Nt = ((N + t.n_tt - 1) / t.n_tt + 15) / 16 * 16;
   t.n_tt = (N + t.Nt - 1) / t.Nt;
   t.otiles = (O + kBM - 1) / kBM;
-  // pairs only where both accumulator sets still fit (Nt <= 128): without the
-  // overlap of the epilogue with the next unit a pair was measured slower
-  t.pair = (t.otiles >= 2 && t.Nt <= 128) ? 2 : 1;
-  t.groups = (t.otiles + t.pair - 1) / t.pair;
+  t.p2 = true;
+  t.pair = 1;
+  t.groups = (t.otiles + 1) / 2;
   t.nkb = (K + kBK - 1) / kBK;
   const int units = t.groups * t.n_tt;
   t.splits = 1;
-  while (split && units * t.splits < 2 * kPlanSMs && t.nkb / (t.splits + 1) >= 8) ++t.splits;
+  while (split && units * (t.splits + 1) <= kPlanSMs / 2 && t.nkb / (t.splits + 1) >= 8)
+    ++t.splits;
   return t;
 }
 
@@ -497,17 +594,28 @@ cudaError_t launch_epi(const void* x, int N, int K, int ldx, const void* w, int 
   a.acc_cols = Nt <= 128 ? 128 : 256;
   a.nbuf = 2 * a.pair * int(a.acc_cols) <= 512 ? 2 : 1;
   a.tmem_cols = uint32_t(a.nbuf * a.pair) * a.acc_cols;
-  const int stage_bytes = a.pair * kBM * 128 + Nt * 128;
+  const int b_rows = tl.p2 ? Nt / 2 : Nt;  // token-tile rows one CTA loads
+  const int stage_bytes = a.pair * kBM * 128 + b_rows * 128;
   a.stages = std::min(8, (kSmemLimit - 1024 - kFixedSmem) / stage_bytes);
   const size_t smem = 1024 + size_t(a.stages) * stage_bytes + kFixedSmem;
   CUtensorMap tmW, tmX;
-  if (!encode_rows(&tmW, w, O, K, K, kBM) || !encode_rows(&tmX, x, N, K, ldx, Nt))
+  if (!encode_rows(&tmW, w, O, K, K, kBM) || !encode_rows(&tmX, x, N, K, ldx, b_rows))
     return cudaErrorInvalidValue;
-  cudaError_t e = cudaFuncSetAttribute(proj_tc_kernel<EPI>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-  if (e != cudaSuccess) return e;
-  const int grid = std::max(1, std::min(a.units, sm_count()));
-  e = launch_pdl(proj_tc_kernel<EPI>, dim3(grid), dim3(kThreads), smem, st, tmW, tmX, a);
+  cudaError_t e;
+  if (tl.p2) {
+    auto kern = proj_tc_kernel<EPI, true>;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    if (e != cudaSuccess) return e;
+    const int clusters = std::max(1, std::min(a.units, max_pairs(kern, smem)));
+    e = launch_pdl_pairs(kern, dim3(unsigned(2 * clusters)), dim3(kThreads), smem, st, tmW, tmX,
+                         a);
+  } else {
+    auto kern = proj_tc_kernel<EPI, false>;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    if (e != cudaSuccess) return e;
+    const int grid = std::max(1, std::min(a.units, sm_count()));
+    e = launch_pdl(kern, dim3(grid), dim3(kThreads), smem, st, tmW, tmX, a);
+  }
   if (e != cudaSuccess) return e;
   if (splits_out) {
     // the caller reduces the partials itself
