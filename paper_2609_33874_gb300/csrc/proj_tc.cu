@@ -2,29 +2,33 @@
 // out[N, O] = epilogue(X[N, K] W[O, K]^T) with bf16 X and W and f32
 // accumulation, for the mixer, output and MLP projections of every layer.
 //
-// The mainloop is the LM head's: weight rows on the MMA's M side (128 rows per
-// tile = the 128 TMEM lanes), the step's rows on N (a token tile of up to 256),
-// one persistent CTA per SM working through (weight tile, token tile) units.
-//   warp 0      TMA producer: 128 x 64 weight tile + Nt x 64 row tile per
-//               stage, both 128-byte swizzled, into a ring of stages
-//   warp 1      TMEM allocator and MMA issuer: 4 x tcgen05.mma kind::f16 (K =
-//               16) per stage into one of two TMEM accumulators
-//   warps 2..5  epilogue: each warp reads its 32 TMEM lanes (32 output
-//               features) x 32 rows at a time and writes bf16 outputs
+// Clusters of two CTAs (one per SM) work through units of (256 weight rows,
+// one token tile of up to 256 of the step's rows, a K range): each CTA loads
+// its own 128 weight rows and half of the token tile (the even CTA the first
+// Nt / 2 rows) into a ring of stages, both CTAs' loads complete on the even
+// CTA's stage barrier, and the even CTA issues M = 256 MMAs
+// (tcgen05.mma.cta_group::2) whose products land in both CTAs' TMEM, each CTA
+// holding its own 128 weight rows over all Nt columns. Per stage a CTA takes in
+// 16 KB of weights and Nt x 64 bytes of rows for 128 x Nt outputs (alone it
+// would take Nt x 128 bytes of rows): the tile bytes one SM takes in, not HBM,
+// bound these small-N GEMMs.
+//   warp 0      TMA producer (each CTA): its 128 x 64 weight tile and
+//               Nt / 2 x 64 row tile per stage, both 128-byte swizzled
+//   warp 1      TMEM allocator (each CTA, together) and, in the even CTA,
+//               the MMA issuer: 4 x tcgen05.mma kind::f16 (K = 16) per stage
+//               into one of two TMEM accumulators; the commits reach both
+//               CTAs' barriers
+//   warps 2..5  epilogue (each CTA): each warp reads its 32 TMEM lanes (32
+//               output features) x 32 rows at a time and writes bf16 outputs
 // Epilogues: kStore (out = acc), kResid (out = res + acc, one rounding; res
 // may be out itself: every element is read and written by one thread) and
 // kSwiGLU: the weight rows come interleaved in blocks of 64 (tile rows 0..63
-// gate features 64 t .., rows 64..127 the matching up features), the warps
-// holding the up half pass their values through shared memory, and
+// gate features 64 t .., rows 64..127 the matching up features), the halves
+// exchange half of their columns through shared memory, and
 // out[n, 64 t + f] = SiLU(gate) * up.
-// Split K: when the (weight tile, token tile) units are too few to occupy the
-// SMs (few output features, long K), each unit covers a range of K and writes
-// its f32 partial; a reduce kernel sums the partials and applies the epilogue.
-// Tile pairs: with at most 128 rows per row tile, a unit covers two weight
-// tiles that share every row tile (two TMEM accumulators, still double
-// buffered), which halves the row-tile bytes a weight byte costs - the row
-// tile is re-read from L2 for every weight tile, and the bytes one SM can take
-// in, not HBM, bound these small-N GEMMs.
+// Split K: when the units are too few to occupy the SM pairs (few output
+// features, long K), each unit covers a range of K and writes its f32 partial;
+// a reduce kernel sums the partials and applies the epilogue.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -40,14 +44,14 @@ namespace {
 
 using namespace sm100;
 
-constexpr int kBM = 128;            // weight rows per tile (MMA M, TMEM lanes)
+constexpr int kBM = 128;            // weight rows per CTA (MMA M per CTA, TMEM lanes)
 constexpr int kBK = 64;             // bf16 elements per stage: 128 bytes
 constexpr int kThreads = 192;
 constexpr int kMaxNt = 256;
 constexpr uint64_t kDrainNs = 200000000ull;
 constexpr int kSmemLimit = 232448;
 // gate/up exchange (16 columns x 128 lanes f32) + barriers and flags
-constexpr int kFixedSmem = 64 * 32 * 4 + 32 * 8 + 64;
+constexpr int kFixedSmem = 16 * 128 * 4 + 32 * 8 + 64;
 
 struct ProjArgs {
   __nv_bfloat16* out;
@@ -56,15 +60,13 @@ struct ProjArgs {
   int* status;
   int N, O, K, ldo;     // rows, weight rows, reduction length, output row stride
   int Nt, n_tt, units, nkb, stages, splits;
-  int pair;             // weight tiles per unit (1 or 2)
-  int nbuf;             // accumulator sets (2: the epilogue overlaps the next unit)
-  uint32_t tmem_cols, acc_cols;
+  uint32_t tmem_cols, acc_cols;  // two accumulators of acc_cols columns
   uint64_t wait_ns;  // budget of one bounded wait (jet_set_wait_budget_ns)
   int hold_first;    // test hook (jet_set_test_stall): withhold the first stage's loads
 };
 
-// unit u -> (weight tile, K split, token tile); the token tiles of one weight
-// slice are consecutive, so they share it through L2
+// unit u -> (256-row weight slice, K split, token tile); the token tiles of one
+// weight slice are consecutive, so they share it through L2
 struct Unit {
   int ot, sp, t0, kb0, kb1;
 };
@@ -79,25 +81,17 @@ __device__ __forceinline__ Unit unit_of(const ProjArgs& a, int u) {
   return x;
 }
 
-// P2: clusters of two CTAs, each unit a 256-row weight slice (the even CTA's
-// 128 rows, then the odd one's) against one token tile; each CTA loads its own
-// weight tile and half of the token tile (the even CTA the first Nt / 2 rows),
-// both CTAs' loads complete on the even CTA's stage barrier, the even CTA
-// issues M = 256 MMAs (cta_group::2) into both CTAs' TMEM, the commits reach
-// both CTAs' barriers, and each CTA runs the epilogue of its own 128 rows. Per
-// stage a CTA takes in 16 KB of weights and Nt x 64 bytes of rows for
-// 128 x Nt outputs, against 16 KB + Nt x 128 bytes alone.
-template <int EPI, bool P2>
+template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
 proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
                const ProjArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  const uint32_t a_bytes = kBM * 128, b_bytes = uint32_t(P2 ? a.Nt / 2 : a.Nt) * 128;
-  const uint32_t stage_bytes = a.pair * a_bytes + b_bytes;
+  const uint32_t a_bytes = kBM * 128, b_bytes = uint32_t(a.Nt / 2) * 128;
+  const uint32_t stage_bytes = a_bytes + b_bytes;
   float* upx = reinterpret_cast<float*>(smem + size_t(a.stages) * stage_bytes);  // [16][128]
-  uint64_t* full = reinterpret_cast<uint64_t*>(upx + 64 * 32);
+  uint64_t* full = reinterpret_cast<uint64_t*>(upx + 16 * 128);
   uint64_t* empty = full + a.stages;
   uint64_t* tfull = empty + a.stages;
   uint64_t* tempty = tfull + 2;
@@ -107,10 +101,9 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
   volatile int* epi_abort = abort_flag + 1;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // P2: this CTA's rank in its pair, the pair's number and the pairs
-  const uint32_t rank = P2 ? cluster_rank() : 0u;
-  const int cid = P2 ? int(blockIdx.x >> 1) : int(blockIdx.x);
-  const int ncl = P2 ? int(gridDim.x >> 1) : int(gridDim.x);
+  // this CTA's rank in its pair, the pair's number and the number of pairs
+  const uint32_t rank = cluster_rank();
+  const int cid = int(blockIdx.x >> 1), ncl = int(gridDim.x >> 1);
   if (threadIdx.x == 0) {
     for (int s = 0; s < a.stages; ++s) {
       mbar_init(full + s, 1);
@@ -118,7 +111,7 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(tfull + b, 1);
-      mbar_init(tempty + b, P2 ? 8 : 4);  // P2: both CTAs' epilogue warps
+      mbar_init(tempty + b, 8);  // both CTAs' epilogue warps
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -131,17 +124,12 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
   }
   pdl_begin();
   if (warp == 1) {
-    if (P2) {
-      tmem_alloc_pair(tmem_slot, a.tmem_cols);
-      tmem_relinquish_pair();
-    } else {
-      tmem_alloc(tmem_slot, a.tmem_cols);
-      tmem_relinquish();
-    }
+    tmem_alloc_pair(tmem_slot, a.tmem_cols);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
   __syncthreads();
-  if (P2) cluster_sync();  // the even CTA's barriers are initialised before any remote use
+  cluster_sync();  // the even CTA's barriers are initialised before any remote use
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -154,8 +142,8 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
       bool ok = true, hold = a.hold_first != 0;
       for (int u = cid; ok && u < a.units; u += ncl) {
         const Unit x = unit_of(a, u);
-        const int o0 = P2 ? (2 * x.ot + int(rank)) * kBM : x.ot * a.pair * kBM;
-        const int t0 = x.t0 + (P2 ? int(rank) * (a.Nt / 2) : 0);
+        const int o0 = (2 * x.ot + int(rank)) * kBM;
+        const int t0 = x.t0 + int(rank) * (a.Nt / 2);
         for (int kb = x.kb0; kb < x.kb1; ++kb) {
           if (!mbar_wait(empty + s, ph ^ 1u, a.wait_ns, abort_flag)) {
             ok = false;
@@ -164,20 +152,13 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
           uint8_t* sa = smem + size_t(s) * stage_bytes;
           if (hold) {
             hold = false;  // test hook: this stage never fills
-          } else if (P2) {
+          } else {
             // both CTAs' bytes complete on the even CTA's barrier, which
             // expects them all; the odd CTA's may land before that arrive
             const uint32_t bar = mapa_shared(full + s, 0);
             if (rank == 0) mbar_arrive_expect_tx(full + s, 2 * stage_bytes);
             tma_load_2d_pair(sa, &tmW, bar, kb * kBK, o0, pol_w);
             tma_load_2d_pair(sa + a_bytes, &tmX, bar, kb * kBK, t0, pol_x);
-            issued |= 1u << s;
-            issued_par = (issued_par & ~(1u << s)) | (ph << s);
-          } else {
-            mbar_arrive_expect_tx(full + s, stage_bytes);
-            for (int t = 0; t < a.pair; ++t)
-              tma_load_2d(sa + t * a_bytes, &tmW, full + s, kb * kBK, o0 + t * kBM, pol_w);
-            tma_load_2d(sa + a.pair * a_bytes, &tmX, full + s, kb * kBK, t0, pol_x);
             issued |= 1u << s;
             issued_par = (issued_par & ~(1u << s)) | (ph << s);
           }
@@ -190,9 +171,9 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
       if (!ok) {
         *abort_flag = 1;
         flag(a.status, JET_ERR_TIMEOUT);
-        // let the copies in flight land (P2: the even CTA's barriers count
-        // both CTAs' bytes; the odd CTA waits out a fixed bounded time)
-        if (!P2 || rank == 0) {
+        // let the copies in flight land: the even CTA's barriers count both
+        // CTAs' bytes; the odd CTA waits out a fixed bounded time
+        if (rank == 0) {
           for (int t = 0; t < a.stages; ++t)
             if (issued & (1u << t)) mbar_wait(full + t, (issued_par >> t) & 1u, kDrainNs, nullptr);
         } else if (issued) {
@@ -204,20 +185,20 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0 && (!P2 || rank == 0)) {
-      const uint32_t idesc = idesc_bf16_f32(P2 ? 2 * kBM : kBM, a.Nt);
+    if (lane == 0 && rank == 0) {
+      const uint32_t idesc = idesc_bf16_f32(2 * kBM, a.Nt);
       int s = 0, local = 0;
       uint32_t ph = 0;
       bool ok = true;
       for (int u = cid; ok && u < a.units; u += ncl, ++local) {
-        const int buf = local % a.nbuf;
-        const uint32_t tph = (local / a.nbuf) & 1;
+        const int buf = local & 1;
+        const uint32_t tph = (local >> 1) & 1;
         if (!mbar_wait(tempty + buf, tph ^ 1u, a.wait_ns, abort_flag)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + uint32_t(buf * a.pair) * a.acc_cols;
+        const uint32_t d_tmem = tmem_base + uint32_t(buf) * a.acc_cols;
         const Unit x = unit_of(a, u);
         for (int kb = x.kb0; kb < x.kb1; ++kb) {
           if (!mbar_wait(full + s, ph, a.wait_ns, abort_flag)) {
@@ -225,53 +206,40 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
             break;
           }
           tc_fence_after();
+          // one thread issues every MMA, so the loop stays lean: the
+          // descriptors are built once per stage and stepped along K by
+          // adding to their start-address field (16-byte units)
           const uint32_t sa = smem_u32(smem + size_t(s) * stage_bytes);
-          const uint32_t sb = sa + a.pair * a_bytes;
-          if (P2) {
-#pragma unroll
-            for (int k = 0; k < 4; ++k)
-              mma_f16_pair(d_tmem, desc_k_sw128(sa + 32 * k), desc_k_sw128(sb + 32 * k), idesc,
-                           (kb - x.kb0) != 0 || k != 0);
-            mma_commit_pair(empty + s, 0x3);  // both CTAs' stage s is free
-          } else {
-            for (int t = 0; t < a.pair; ++t) {
-#pragma unroll
-              for (int k = 0; k < 4; ++k)
-                mma_f16(d_tmem + t * a.acc_cols, desc_k_sw128(sa + t * a_bytes + 32 * k),
-                        desc_k_sw128(sb + 32 * k), idesc, (kb - x.kb0) != 0 || k != 0);
-            }
-            mma_commit(empty + s);
-          }
+          const uint64_t da = desc_k_sw128(sa), db = desc_k_sw128(sa + a_bytes);
+          mma_f16_pair(d_tmem, da, db, idesc, kb != x.kb0);
+          mma_f16_pair(d_tmem, da + 2, db + 2, idesc, 1u);
+          mma_f16_pair(d_tmem, da + 4, db + 4, idesc, 1u);
+          mma_f16_pair(d_tmem, da + 6, db + 6, idesc, 1u);
+          mma_commit_pair(empty + s, 0x3);  // both CTAs' stage s is free
           if (++s == a.stages) {
             s = 0;
             ph ^= 1u;
           }
         }
         if (!ok) break;
-        if (P2)
-          mma_commit_pair(tfull + buf, 0x3);
-        else
-          mma_commit(tfull + buf);
+        mma_commit_pair(tfull + buf, 0x3);
       }
       if (!ok) {
         *abort_flag = 1;
         flag(a.status, JET_ERR_TIMEOUT);
-        if (P2)
-          mma_commit_pair(drain, 0x1);
-        else
-          mma_commit(drain);
+        mma_commit_pair(drain, 0x1);
         mbar_wait(drain, 0, kDrainNs, nullptr);
       }
     }
   } else {
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;            // TMEM lane quadrant this warp may access
-    // P2: the odd CTA's warps release the accumulator on the even CTA's barrier
-    const uint32_t tempty_even = P2 ? mapa_shared(tempty, 0) : 0u;
+    // the odd CTA's warps release the accumulator on the even CTA's barrier
+    const uint32_t tempty_even = mapa_shared(tempty, 0);
     int local = 0;
     for (int u = cid; u < a.units; u += ncl, ++local) {
-      const int buf = local % a.nbuf;
-      const uint32_t tph = (local / a.nbuf) & 1;
+      const int buf = local & 1;
+      const uint32_t tph = (local >> 1) & 1;
       const Unit x = unit_of(a, u);
       const int t0 = x.t0;
       const bool ok = warp_mbar_wait(tfull + buf, tph, a.wait_ns, abort_flag);
@@ -280,11 +248,8 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
       if (*epi_abort) break;
       tc_fence_after();
       const int ncols = min(a.Nt, a.N - t0);
-      for (int pt = 0; pt < a.pair; ++pt) {
-      // this accumulator's weight tile
-      const int ot = P2 ? 2 * x.ot + int(rank) : x.ot * a.pair + pt;
-      const uint32_t tl = tmem_base + uint32_t(buf * a.pair + pt) * a.acc_cols +
-                          (uint32_t(32 * q) << 16);
+      const int ot = 2 * x.ot + int(rank);  // this CTA's 128-row weight tile
+      const uint32_t tl = tmem_base + uint32_t(buf) * a.acc_cols + (uint32_t(32 * q) << 16);
       for (int c0 = 0; c0 < ncols; c0 += 32) {
         float v[32];
         tmem_ld_32cols(tl + uint32_t(c0), v);
@@ -306,9 +271,9 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
           // every warp forms SiLU(gate) * up for its 16 columns - the gate half
           // columns 0..15, the up half 16..31
           const bool gate = q < 2;
-          const int hb = gate ? 16 : 0;  // the columns this thread hands over
+          // the columns this thread hands over: 16..31 (gate half) or 0..15
 #pragma unroll
-          for (int j = 0; j < 16; ++j) upx[j * 128 + 32 * q + lane] = v[hb + j];
+          for (int j = 0; j < 16; ++j) upx[j * 128 + 32 * q + lane] = gate ? v[16 + j] : v[j];
           named_bar_sync(1, 128);
           const int f = ot * 64 + 32 * (q & 1) + lane;  // output feature
           const int cb = gate ? 0 : 16;                 // the columns this thread forms
@@ -342,11 +307,10 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
           }
         }
       }
-      }  // the unit's weight tiles
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
-        if (P2 && rank != 0)
+        if (rank != 0)
           mbar_arrive_cluster(tempty_even + uint32_t(buf) * 8u);
         else
           mbar_arrive(tempty + buf);
@@ -357,15 +321,12 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
 
   tc_fence_before();
   __syncthreads();
-  // P2: neither CTA leaves (or frees its TMEM) while the partner's MMAs or
+  // neither CTA leaves (or frees its TMEM) while the partner's MMAs or
   // copies may still use its shared memory or TMEM
-  if (P2) cluster_sync();
+  cluster_sync();
   if (warp == 1) {
     tc_fence_after();
-    if (P2)
-      tmem_dealloc_pair(tmem_base, a.tmem_cols);
-    else
-      tmem_dealloc(tmem_base, a.tmem_cols);
+    tmem_dealloc_pair(tmem_base, a.tmem_cols);
   }
 }
 
@@ -541,8 +502,7 @@ cudaError_t launch_reduce(const ProjArgs& a, float* part, int N, int O, void* ou
                           const void* res, cudaStream_t st);
 
 struct Tiling {
-  int n_tt, Nt, otiles, pair, groups, nkb, splits;
-  bool p2;  // clusters of two CTAs, 256 weight rows per unit
+  int n_tt, Nt, otiles, groups, nkb, splits;  // groups: 256-row weight slices
 };
 
 // token tiles of at most 256 rows (a multiple of 16: each CTA of a pair holds
@@ -557,8 +517,6 @@ Tiling tiling(int N, int O, int K, bool split) {
   t.Nt = ((N + t.n_tt - 1) / t.n_tt + 15) / 16 * 16;
   t.n_tt = (N + t.Nt - 1) / t.Nt;
   t.otiles = (O + kBM - 1) / kBM;
-  t.p2 = true;
-  t.pair = 1;
   t.groups = (t.otiles + 1) / 2;
   t.nkb = (K + kBK - 1) / kBK;
   const int units = t.groups * t.n_tt;
@@ -588,34 +546,22 @@ cudaError_t launch_epi(const void* x, int N, int K, int ldx, const void* w, int 
   a.ldo = ldo;
   a.Nt = Nt;
   a.n_tt = n_tt;
-  a.pair = tl.pair;
   a.units = tl.groups * n_tt * a.splits;
   a.nkb = (K + kBK - 1) / kBK;
   a.acc_cols = Nt <= 128 ? 128 : 256;
-  a.nbuf = 2 * a.pair * int(a.acc_cols) <= 512 ? 2 : 1;
-  a.tmem_cols = uint32_t(a.nbuf * a.pair) * a.acc_cols;
-  const int b_rows = tl.p2 ? Nt / 2 : Nt;  // token-tile rows one CTA loads
-  const int stage_bytes = a.pair * kBM * 128 + b_rows * 128;
+  a.tmem_cols = 2 * a.acc_cols;
+  const int b_rows = Nt / 2;  // token-tile rows one CTA loads
+  const int stage_bytes = kBM * 128 + b_rows * 128;
   a.stages = std::min(8, (kSmemLimit - 1024 - kFixedSmem) / stage_bytes);
   const size_t smem = 1024 + size_t(a.stages) * stage_bytes + kFixedSmem;
   CUtensorMap tmW, tmX;
   if (!encode_rows(&tmW, w, O, K, K, kBM) || !encode_rows(&tmX, x, N, K, ldx, b_rows))
     return cudaErrorInvalidValue;
-  cudaError_t e;
-  if (tl.p2) {
-    auto kern = proj_tc_kernel<EPI, true>;
-    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-    if (e != cudaSuccess) return e;
-    const int clusters = std::max(1, std::min(a.units, max_pairs(kern, smem)));
-    e = launch_pdl_pairs(kern, dim3(unsigned(2 * clusters)), dim3(kThreads), smem, st, tmW, tmX,
-                         a);
-  } else {
-    auto kern = proj_tc_kernel<EPI, false>;
-    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-    if (e != cudaSuccess) return e;
-    const int grid = std::max(1, std::min(a.units, sm_count()));
-    e = launch_pdl(kern, dim3(grid), dim3(kThreads), smem, st, tmW, tmX, a);
-  }
+  auto kern = proj_tc_kernel<EPI>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  if (e != cudaSuccess) return e;
+  const int clusters = std::max(1, std::min(a.units, max_pairs(kern, smem)));
+  e = launch_pdl_pairs(kern, dim3(unsigned(2 * clusters)), dim3(kThreads), smem, st, tmW, tmX, a);
   if (e != cudaSuccess) return e;
   if (splits_out) {
     // the caller reduces the partials itself
