@@ -145,9 +145,12 @@ __device__ __forceinline__ uint32_t a_off(int r, int chunk) {
 
 // T = (I + A)^{-1} (unit lower triangular) in f32, 64 floats a row, in the
 // token tiles' two 8 KB Q slots (rows 32 s .. 32 s + 31 in slice s): the Q of
-// the chunk is no longer needed when it is formed
-__device__ __forceinline__ float* t_row(uint8_t* sm, int r) {
-  return reinterpret_cast<float*>(sm + kOffKQ + (r >> 5) * kKQSlice + 8192 + (r & 31) * 256);
+// the chunk is no longer needed when it is formed. Element (r, col): the
+// 16-byte chunks of row r permuted by r & 15, so that the rows one warp
+// reads or writes at the same columns fall in different banks.
+__device__ __forceinline__ float* t_at(uint8_t* sm, int r, int col) {
+  return reinterpret_cast<float*>(sm + kOffKQ + (r >> 5) * kKQSlice + 8192 + (r & 31) * 256 +
+                                  ((((col >> 2) ^ (r & 15)) << 4) | ((col & 3) << 2)));
 }
 
 // T in 16 x 16 blocks: the diagonal blocks T_ii by substitution (thread
@@ -178,7 +181,7 @@ __device__ __forceinline__ void invert_unit_lower(const float* __restrict__ A, u
       x[r] = s;
     }
 #pragma unroll
-    for (int r = 0; r < 16; ++r) t_row(sm, 16 * bi + r)[16 * bi + jj] = x[r];
+    for (int r = 0; r < 16; ++r) *t_at(sm, 16 * bi + r, 16 * bi + jj) = x[r];
   }
   __syncthreads();
 #pragma unroll
@@ -189,40 +192,41 @@ __device__ __forceinline__ void invert_unit_lower(const float* __restrict__ A, u
     const int jb = t >> 6, ib = jb + d, r = (t >> 2) & 15, c4 = t & 3;
     if (act) {
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int k4 = 4 * jb; k4 < 4 * ib; ++k4) {
+      // 4 d chunks of k (a compile-time count: the loads can all be issued early)
+#pragma unroll
+      for (int kk = 0; kk < 4 * d; ++kk) {
+        const int k4 = 4 * jb + kk;
         const float4 a4 = *reinterpret_cast<const float4*>(A + a_off(16 * ib + r, k4));
         const float av[4] = {a4.x, a4.y, a4.z, a4.w};
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          const float4 t4 =
-              *reinterpret_cast<const float4*>(t_row(sm, 4 * k4 + e) + 16 * jb + 4 * c4);
+          const float4 t4 = *reinterpret_cast<const float4*>(t_at(sm, 4 * k4 + e, 16 * jb + 4 * c4));
           acc.x = fmaf(av[e], t4.x, acc.x);
           acc.y = fmaf(av[e], t4.y, acc.y);
           acc.z = fmaf(av[e], t4.z, acc.z);
           acc.w = fmaf(av[e], t4.w, acc.w);
         }
       }
-      *reinterpret_cast<float4*>(t_row(sm, 16 * jb + r) + 16 * ib + 4 * c4) = acc;
+      *reinterpret_cast<float4*>(t_at(sm, 16 * jb + r, 16 * ib + 4 * c4)) = acc;
     }
     __syncthreads();
     if (act) {
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      const float* ti = t_row(sm, 16 * ib + r) + 16 * ib;
 #pragma unroll
       for (int k4 = 0; k4 < 4; ++k4) {
-        const float4 a4 = *reinterpret_cast<const float4*>(ti + 4 * k4);
+        const float4 a4 = *reinterpret_cast<const float4*>(t_at(sm, 16 * ib + r, 16 * ib + 4 * k4));
         const float av[4] = {a4.x, a4.y, a4.z, a4.w};
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const float4 p4 =
-              *reinterpret_cast<const float4*>(t_row(sm, 16 * jb + 4 * k4 + e) + 16 * ib + 4 * c4);
+              *reinterpret_cast<const float4*>(t_at(sm, 16 * jb + 4 * k4 + e, 16 * ib + 4 * c4));
           acc.x = fmaf(av[e], p4.x, acc.x);
           acc.y = fmaf(av[e], p4.y, acc.y);
           acc.z = fmaf(av[e], p4.z, acc.z);
           acc.w = fmaf(av[e], p4.w, acc.w);
         }
       }
-      *reinterpret_cast<float4*>(t_row(sm, 16 * ib + r) + 16 * jb + 4 * c4) =
+      *reinterpret_cast<float4*>(t_at(sm, 16 * ib + r, 16 * jb + 4 * c4)) =
           make_float4(-acc.x, -acc.y, -acc.z, -acc.w);
     }
     __syncthreads();
@@ -468,15 +472,17 @@ scan_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
       invert_unit_lower(Am, sm, tid);
       {
         const int row = tid >> 2;
-        const float* tr = t_row(sm, row);
 #pragma unroll
         for (int h2 = 0; h2 < 2; ++h2) {
           const int jj = 2 * (tid & 3) + h2;
           float x1[8], x2[8];
+          const float4 t0 = *reinterpret_cast<const float4*>(t_at(sm, row, 8 * jj));
+          const float4 t1 = *reinterpret_cast<const float4*>(t_at(sm, row, 8 * jj + 4));
+          const float tv[8] = {t0.x, t0.y, t0.z, t0.w, t1.x, t1.y, t1.z, t1.w};
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             const int i = 8 * jj + e;
-            const float t = i <= row ? tr[i] : 0.f;
+            const float t = i <= row ? tv[e] : 0.f;
             x1[e] = t * vb[i];
             x2[e] = x1[e] * vg[i];
           }
