@@ -154,12 +154,12 @@ __device__ __forceinline__ float* t_at(uint8_t* sm, int r, int col) {
 }
 
 // T in 16 x 16 blocks: the diagonal blocks T_ii by substitution (thread
-// (i, j): column j of T_ii), then the blocks below them level by level
-// (d = i - j = 1, 2, 3): T_ij = -T_ii P_ij with P_ij = sum_{k=j}^{i-1} A_ik T_kj,
-// P_ij held in the unused block (j, i) above the diagonal. Every block of T
-// at or below the diagonal is written (zeros above the diagonal of T_ii). In
-// the block products a thread forms four adjacent outputs of one row from
-// 16-byte loads.
+// (i, j): column j of T_ii), the products T_ii A_ik (k < i) in the unused
+// blocks above the diagonal, then the blocks below the diagonal level by level
+// (d = i - j = 1, 2, 3): T_ij = -sum_{k=j}^{i-1} (T_ii A_ik) T_kj - five
+// barrier-separated steps. Every block of T at or below the diagonal is
+// written (zeros above the diagonal of T_ii). In the block products a thread
+// forms four adjacent outputs of one row from 16-byte loads.
 __device__ __forceinline__ void invert_unit_lower(const float* __restrict__ A, uint8_t* sm,
                                                   int tid) {
   if (tid < 64) {
@@ -184,46 +184,52 @@ __device__ __forceinline__ void invert_unit_lower(const float* __restrict__ A, u
     for (int r = 0; r < 16; ++r) *t_at(sm, 16 * bi + r, 16 * bi + jj) = x[r];
   }
   __syncthreads();
+  // the six products T_ii A_ik (k < i), each kept in the unused block (k, i)
+  // above the diagonal: task (block b, row r, columns 4 c4 ..)
+  for (int task = tid; task < 6 * 64; task += kThreads) {
+    const int b = task >> 6, r = (task >> 2) & 15, c4 = task & 3;
+    const int ib = b < 1 ? 1 : b < 3 ? 2 : 3, kb = b - ib * (ib - 1) / 2;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int k4 = 0; k4 < 4; ++k4) {
+      const float4 t4 = *reinterpret_cast<const float4*>(t_at(sm, 16 * ib + r, 16 * ib + 4 * k4));
+      const float tv[4] = {t4.x, t4.y, t4.z, t4.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float4 a4 =
+            *reinterpret_cast<const float4*>(A + a_off(16 * ib + 4 * k4 + e, 4 * kb + c4));
+        acc.x = fmaf(tv[e], a4.x, acc.x);
+        acc.y = fmaf(tv[e], a4.y, acc.y);
+        acc.z = fmaf(tv[e], a4.z, acc.z);
+        acc.w = fmaf(tv[e], a4.w, acc.w);
+      }
+    }
+    *reinterpret_cast<float4*>(t_at(sm, 16 * kb + r, 16 * ib + 4 * c4)) = acc;
+  }
+  __syncthreads();
+  // then the blocks below the diagonal level by level (d = i - j = 1, 2, 3):
+  // T_ij = -sum_{k=j}^{i-1} (T_ii A_ik) T_kj, one barrier a level
 #pragma unroll
   for (int d = 1; d < 4; ++d) {
-    // task t: block (jb, jb + d), row r, columns 4 c4 .. 4 c4 + 3
+    // task t: block (jb + d, jb), row r, columns 4 c4 .. 4 c4 + 3
     const int t = tid;
-    const bool act = t < (4 - d) * 64;
     const int jb = t >> 6, ib = jb + d, r = (t >> 2) & 15, c4 = t & 3;
-    if (act) {
+    if (t < (4 - d) * 64) {
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
       // 4 d chunks of k (a compile-time count: the loads can all be issued early)
 #pragma unroll
       for (int kk = 0; kk < 4 * d; ++kk) {
-        const int k4 = 4 * jb + kk;
-        const float4 a4 = *reinterpret_cast<const float4*>(A + a_off(16 * ib + r, k4));
-        const float av[4] = {a4.x, a4.y, a4.z, a4.w};
+        const int kb = jb + (kk >> 2), k4 = kk & 3;
+        const float4 p4 = *reinterpret_cast<const float4*>(t_at(sm, 16 * kb + r, 16 * ib + 4 * k4));
+        const float pv[4] = {p4.x, p4.y, p4.z, p4.w};
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          const float4 t4 = *reinterpret_cast<const float4*>(t_at(sm, 4 * k4 + e, 16 * jb + 4 * c4));
-          acc.x = fmaf(av[e], t4.x, acc.x);
-          acc.y = fmaf(av[e], t4.y, acc.y);
-          acc.z = fmaf(av[e], t4.z, acc.z);
-          acc.w = fmaf(av[e], t4.w, acc.w);
-        }
-      }
-      *reinterpret_cast<float4*>(t_at(sm, 16 * jb + r, 16 * ib + 4 * c4)) = acc;
-    }
-    __syncthreads();
-    if (act) {
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-      for (int k4 = 0; k4 < 4; ++k4) {
-        const float4 a4 = *reinterpret_cast<const float4*>(t_at(sm, 16 * ib + r, 16 * ib + 4 * k4));
-        const float av[4] = {a4.x, a4.y, a4.z, a4.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float4 p4 =
-              *reinterpret_cast<const float4*>(t_at(sm, 16 * jb + 4 * k4 + e, 16 * ib + 4 * c4));
-          acc.x = fmaf(av[e], p4.x, acc.x);
-          acc.y = fmaf(av[e], p4.y, acc.y);
-          acc.z = fmaf(av[e], p4.z, acc.z);
-          acc.w = fmaf(av[e], p4.w, acc.w);
+          const float4 t4 =
+              *reinterpret_cast<const float4*>(t_at(sm, 16 * kb + 4 * k4 + e, 16 * jb + 4 * c4));
+          acc.x = fmaf(pv[e], t4.x, acc.x);
+          acc.y = fmaf(pv[e], t4.y, acc.y);
+          acc.z = fmaf(pv[e], t4.z, acc.z);
+          acc.w = fmaf(pv[e], t4.w, acc.w);
         }
       }
       *reinterpret_cast<float4*>(t_at(sm, 16 * ib + r, 16 * jb + 4 * c4)) =
