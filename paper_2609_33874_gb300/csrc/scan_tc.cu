@@ -256,6 +256,8 @@ scan_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   float* vgc = vg + 64;                                // G[C-1][i]
   float* gC = vgc + 64;                                // g_{C-1}
   float* Am = reinterpret_cast<float*>(sm + kOffA);
+  // the chunk's outputs [64 tokens][kD] bf16, staged in the A buffer
+  __nv_bfloat16* ost = reinterpret_cast<__nv_bfloat16*>(sm + kOffA);
   uint64_t* bar_k = reinterpret_cast<uint64_t*>(sm + kOffBar);  // K buffers 0 and 1
   uint64_t* bar_q = bar_k + 2;
   uint64_t* bar_v = bar_k + 3;
@@ -670,11 +672,10 @@ scan_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
       tmem_ld_32cols(scol, s0);
       tmem_ld_32cols(scol + 32, s1);
       tmem_wait_ld();
+      // the chunk's outputs through the solve's A buffer (free until the next
+      // chunk), [token][value] as they are stored, for 16-byte global stores
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const int t = 32 * grp + i;
-        if (t < n) o[(size_t(c0 + t) * Hl + h) * kD + c] = __float2bfloat16_rn(ov[i] * rs);
-      }
+      for (int i = 0; i < 32; ++i) ost[(32 * grp + i) * kD + c] = __float2bfloat16_rn(ov[i] * rs);
       if (last) {
         const size_t row0 = head + 64 * grp;
 #pragma unroll
@@ -694,6 +695,13 @@ scan_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    // each token's 128 outputs are 256 contiguous bytes of o (the next
+    // chunk's first barrier comes before its A lands in the buffer)
+    for (int e = tid; e < n * (kD / 8); e += kThreads) {
+      const int t = e / (kD / 8), q = e % (kD / 8);
+      *reinterpret_cast<uint4*>(o + (size_t(c0 + t) * Hl + h) * kD + 8 * q) =
+          reinterpret_cast<const uint4*>(ost)[e];
+    }
   }
   if (!ok) {
     // a wait ran out: let the copies and tensor-core work already issued
