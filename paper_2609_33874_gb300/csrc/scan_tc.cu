@@ -64,8 +64,7 @@ constexpr uint32_t kKQSlice = 3 * 8192;
 constexpr uint32_t kOffKQ = 0;
 constexpr uint32_t kOffV = 2 * kKQSlice;            // V: 64 rows x 2 dv-slices
 constexpr uint32_t kVSlice = 8192;
-constexpr uint32_t kOffS0h = 65536, kOffS0l = 98304;  // S0^T hi, lo: 128 rows x 2 dk-slices
-constexpr uint32_t kS0Slice = 16384;
+// 65536 .. 131071: free (the state's hi/lo operand lives in TMEM)
 // [-W | g Q] hi, lo: MN-major (dk rows of 64 tokens), two N slices (-W, then
 // g Q) of 128 rows; the first slices hold T diag(b) and T diag(b g) until W
 constexpr uint32_t kOffWQh = 131072, kOffWQl = 163840;
@@ -82,8 +81,11 @@ constexpr uint32_t kSmemBytes = kOffBar + 64 + 1024;
 static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
 
 // TMEM columns: [K; Q] K^T at 0 (64), X = [d^T | O^T] at 64 (128), the state
-// at 256 (128)
+// at 256 (128), the state's hi and lo bf16 operand at 384 and 448 (64 each)
 constexpr uint32_t kColGM = 0, kColX = 64, kColO = 128, kColSt = 256;
+// the state as the X MMA's A operand: bf16 pairs (dk elements 2k, 2k + 1 of
+// lane c in column k), hi then lo
+constexpr uint32_t kColS0h = 384, kColS0l = 448;
 
 // byte offset of element (row, k) in a 128-byte swizzled K-major tile
 __device__ __forceinline__ uint32_t sw_off(int row, int k, uint32_t slice_bytes) {
@@ -107,6 +109,21 @@ __device__ __forceinline__ void split2(float x, float y, uint32_t& hi, uint32_t&
   const __nv_bfloat162 l = __floats2bfloat162_rn(x - hf.x, y - hf.y);
   hi = *reinterpret_cast<const uint32_t*>(&h);
   lo = *reinterpret_cast<const uint32_t*>(&l);
+}
+
+// 32 consecutive state values of this thread's lane (dk i0 .. i0 + 31) as hi
+// and lo bf16 pairs in 16 TMEM columns each
+__device__ __forceinline__ void put32_tmem(uint32_t hi_col, uint32_t lo_col, const float* x) {
+  float h[16], l[16];
+#pragma unroll
+  for (int k = 0; k < 16; ++k) {
+    uint32_t hh, ll;
+    split2(x[2 * k], x[2 * k + 1], hh, ll);
+    h[k] = __uint_as_float(hh);
+    l[k] = __uint_as_float(ll);
+  }
+  tmem_st_16cols(hi_col, h);
+  tmem_st_16cols(lo_col, l);
 }
 
 // eight consecutive values (chunk j of a 64-element slice row) as hi and lo
@@ -295,8 +312,6 @@ scan_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   }
   const int nch = (p1 - p0 + kC - 1) / kC;
   const size_t head = (size_t(r) * Hl + h) * kD;  // row 0 of this (request, head)'s state
-  uint8_t* const s0h = sm + kOffS0h;
-  uint8_t* const s0l = sm + kOffS0l;
   const uint64_t pol = policy_evict_first();
 
   // TMA copies of chunk j's K (into buffer j & 1), Q and V, issued by thread 0;
@@ -343,9 +358,7 @@ scan_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] = s_init ? s_init[(head + i0 + i) * kD + c] : 0.f;
     tmem_st_32cols(tmem + lane_off + kColSt + i0, v);
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-      put8(s0h + grp * kS0Slice, s0l + grp * kS0Slice, c, ((i0 & 63) >> 3) + j, v + 8 * j);
+    put32_tmem(tmem + lane_off + kColS0h + (i0 >> 1), tmem + lane_off + kColS0l + (i0 >> 1), v);
   }
   tmem_wait_st();
   fence_proxy_async_shared();
@@ -570,18 +583,17 @@ scan_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
       tc_fence_after();
 #pragma unroll
       for (int pass = 0; pass < 3; ++pass) {
-        const uint32_t a = smem_u32(pass == 2 ? s0l : s0h);
+        // A (the state, K = dk) from TMEM: 8 packed columns per K = 16 step
+        const uint32_t a = tmem + (pass == 2 ? kColS0l : kColS0h);
         const uint32_t b = smem_u32(sm + (pass == 1 ? kOffWQl : kOffWQh));
 #pragma unroll
         for (int st = 0; st < 8; ++st) {
-          const uint32_t oa = (st >> 2) * kS0Slice + 32 * (st & 3);
           if (DELTA)
-            mma_f16(tmem + kColX, desc_k_sw128(a + oa), desc_mn_sw128(b + st * 2048, kWQSlice),
-                    idesc_bf16_f32(128, 128) | (1u << 16), 1u);
+            mma_f16_ta(tmem + kColX, a + 8 * st, desc_mn_sw128(b + st * 2048, kWQSlice),
+                       idesc_bf16_f32(128, 128) | (1u << 16), 1u);
           else
-            mma_f16(tmem + kColO, desc_k_sw128(a + oa),
-                    desc_mn_sw128(b + kWQSlice + st * 2048, kWQSlice),
-                    idesc_bf16_f32(128, 64) | (1u << 16), (pass | st) != 0);
+            mma_f16_ta(tmem + kColO, a + 8 * st, desc_mn_sw128(b + kWQSlice + st * 2048, kWQSlice),
+                       idesc_bf16_f32(128, 64) | (1u << 16), (pass | st) != 0);
         }
       }
       mma_commit(bar_mma);
@@ -684,11 +696,11 @@ scan_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
           s_out[(row0 + 32 + i) * kD + c] = s1[i];
         }
       } else {
-#pragma unroll
-        for (int jj = 0; jj < 4; ++jj) {
-          put8(s0h + grp * kS0Slice, s0l + grp * kS0Slice, c, jj, s0 + 8 * jj);
-          put8(s0h + grp * kS0Slice, s0l + grp * kS0Slice, c, 4 + jj, s1 + 8 * jj);
-        }
+        // this warpgroup's 64 dk columns: packed columns 32 grp .. 32 grp + 31
+        put32_tmem(tmem + lane_off + kColS0h + 32 * grp, tmem + lane_off + kColS0l + 32 * grp, s0);
+        put32_tmem(tmem + lane_off + kColS0h + 32 * grp + 16,
+                   tmem + lane_off + kColS0l + 32 * grp + 16, s1);
+        tmem_wait_st();
       }
     }
     fence_proxy_async_shared();
