@@ -63,6 +63,7 @@ struct ProjArgs {
   uint32_t tmem_cols, acc_cols;  // two accumulators of acc_cols columns
   uint64_t wait_ns;  // budget of one bounded wait (jet_set_wait_budget_ns)
   int hold_first;    // test hook (jet_set_test_stall): withhold the first stage's loads
+  int vec;           // out 16-byte aligned and ldo % 8 == 0: 16-byte output stores
 };
 
 // unit u -> (256-row weight slice, K split, token tile); the token tiles of one
@@ -292,6 +293,22 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ 
             }
           }
           named_bar_sync(1, 128);
+        } else if (EPI == kProjStore && a.vec && ot * kBM + 32 * q + 32 <= a.O) {
+          // this warp's 32 features x 32 rows through its 2 KB of the exchange
+          // buffer (unused by this epilogue), then 16-byte pieces of each row
+          __nv_bfloat16* stg = reinterpret_cast<__nv_bfloat16*>(upx) + q * 1024;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) stg[i * 32 + lane] = __float2bfloat16_rn(v[i]);
+          __syncwarp();
+          const int f0 = ot * kBM + 32 * q;  // the warp's first output feature
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const int e = lane + 32 * k, row = e >> 2, pc = e & 3;
+            if (row < nc)
+              *reinterpret_cast<uint4*>(a.out + size_t(t0 + c0 + row) * a.ldo + f0 + 8 * pc) =
+                  *reinterpret_cast<const uint4*>(stg + row * 32 + 8 * pc);
+          }
+          __syncwarp();
         } else {
           const int o = ot * kBM + 32 * q + lane;  // output feature
           if (o < a.O) {
@@ -544,6 +561,7 @@ cudaError_t launch_epi(const void* x, int N, int K, int ldx, const void* w, int 
   a.O = O;
   a.K = K;
   a.ldo = ldo;
+  a.vec = (ldo % 8 == 0) && (reinterpret_cast<uintptr_t>(out) % 16 == 0);
   a.Nt = Nt;
   a.n_tt = n_tt;
   a.units = tl.groups * n_tt * a.splits;
