@@ -110,7 +110,7 @@ struct IdleClock {
   }
 };
 
-// mbar_wait by every lane of a warp, with one verdict for the whole warp
+// mbar_wait by every lane of a warp, with one outcome for the whole warp
 __device__ __forceinline__ bool warp_mbar_wait(uint64_t* bar, uint32_t parity, uint64_t budget_ns,
                                                volatile int* abort) {
   const bool ok = mbar_wait(bar, parity, budget_ns, abort);
