@@ -171,10 +171,10 @@ __device__ __forceinline__ float* t_at(uint8_t* sm, int r, int col) {
 }
 
 // T in 16 x 16 blocks: the diagonal blocks T_ii by substitution (thread
-// (i, j): column j of T_ii), the products T_ii A_ik (k < i) in the unused
-// blocks above the diagonal, then the blocks below the diagonal level by level
-// (d = i - j = 1, 2, 3): T_ij = -sum_{k=j}^{i-1} (T_ii A_ik) T_kj - five
-// barrier-separated steps. Every block of T at or below the diagonal is
+// (i, j): column j of T_ii) and, in the same step, the products T_ii A_ik
+// (k < i) by substitution too, in the unused blocks above the diagonal; then
+// the blocks below the diagonal level by level (d = i - j = 1, 2, 3):
+// T_ij = -sum_{k=j}^{i-1} (T_ii A_ik) T_kj - four barrier-separated steps. Every block of T at or below the diagonal is
 // written (zeros above the diagonal of T_ii). In the block products a thread
 // forms four adjacent outputs of one row from 16-byte loads.
 __device__ __forceinline__ void invert_unit_lower(const float* __restrict__ A, uint8_t* sm,
@@ -199,29 +199,30 @@ __device__ __forceinline__ void invert_unit_lower(const float* __restrict__ A, u
     }
 #pragma unroll
     for (int r = 0; r < 16; ++r) *t_at(sm, 16 * bi + r, 16 * bi + jj) = x[r];
-  }
-  __syncthreads();
-  // the six products T_ii A_ik (k < i), each kept in the unused block (k, i)
-  // above the diagonal: task (block b, row r, columns 4 c4 ..)
-  for (int task = tid; task < 6 * 64; task += kThreads) {
-    const int b = task >> 6, r = (task >> 2) & 15, c4 = task & 3;
+  } else if (tid < 64 + 6 * 16) {
+    // in the same step, the six products T_ii A_ik (k < i), column by column as
+    // the solutions of (I + A_ii) x = A_ik[:, col], each kept in the unused
+    // block (k, i) above the diagonal
+    const int task = tid - 64, b = task >> 4, col = task & 15;
     const int ib = b < 1 ? 1 : b < 3 ? 2 : 3, kb = b - ib * (ib - 1) / 2;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    float x[16];
 #pragma unroll
-    for (int k4 = 0; k4 < 4; ++k4) {
-      const float4 t4 = *reinterpret_cast<const float4*>(t_at(sm, 16 * ib + r, 16 * ib + 4 * k4));
-      const float tv[4] = {t4.x, t4.y, t4.z, t4.w};
+    for (int r = 0; r < 16; ++r) {
+      float s = A[a_off(16 * ib + r, 4 * kb + (col >> 2)) + (col & 3)];
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float4 a4 =
-            *reinterpret_cast<const float4*>(A + a_off(16 * ib + 4 * k4 + e, 4 * kb + c4));
-        acc.x = fmaf(tv[e], a4.x, acc.x);
-        acc.y = fmaf(tv[e], a4.y, acc.y);
-        acc.z = fmaf(tv[e], a4.z, acc.z);
-        acc.w = fmaf(tv[e], a4.w, acc.w);
+      for (int q = 0; q < 4; ++q) {
+        if (4 * q < r) {
+          const float4 a4 = *reinterpret_cast<const float4*>(A + a_off(16 * ib + r, 4 * ib + q));
+          const float av[4] = {a4.x, a4.y, a4.z, a4.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            if (4 * q + e < r) s = fmaf(-av[e], x[4 * q + e], s);
+        }
       }
+      x[r] = s;
     }
-    *reinterpret_cast<float4*>(t_at(sm, 16 * kb + r, 16 * ib + 4 * c4)) = acc;
+#pragma unroll
+    for (int r = 0; r < 16; ++r) *t_at(sm, 16 * kb + r, 16 * ib + col) = x[r];
   }
   __syncthreads();
   // then the blocks below the diagonal level by level (d = i - j = 1, 2, 3):
